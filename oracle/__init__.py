@@ -1,0 +1,229 @@
+"""CPU oracle for the W4/W2-GateUp decode MLP path (plain C, fp64).
+
+TEST INFRASTRUCTURE.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
+package.  The product path (``paper_2606_04238_gb300``) never imports it and
+shares no code with it.
+
+What it computes (paper sections cited in ``wq_oracle.c``):
+  * ``quantize``   Stage-1 group-wise asymmetric min-max RTN (Sec. 4.1), fp32,
+                   bit-exact definition of codes / scales / zeros.
+  * ``tile_pack``  the packed storage format (byte layout definition).
+  * ``gateup``     g,u = x W^T + alpha (x A^T) B^T (Eq. 1) on the dequantized
+                   gate/up weights, h = SiLU(g) * u (Sec. 3.3), fp64.
+  * ``down``       y = residual + h Wd^T on the dequantized 4-bit down weights.
+  * ``prenorm``    unit-weight RMSNorm of the MLP input, rounded to bf16.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "wq_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+RMS_EPS = 1e-6
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (IEEE arithmetic: no fast-math, no FMA contraction)."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
+               "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I = ctypes.c_int
+            D = ctypes.c_double
+            S = ctypes.c_size_t
+            sig = {
+                "orc_quantize": (I, [P, I, I, I, I, P, P, P]),
+                "orc_tile_pack": (I, [P, P, P, I, I, I, I, P, P]),
+                "orc_tile_unpack": (I, [P, P, I, I, I, I, P, P, P]),
+                "orc_dequant": (I, [P, P, P, I, I, I, P]),
+                "orc_prenorm": (I, [P, I, I, D, P]),
+                "orc_gateup": (I, [P, I, I, I, P, P, P, P, P, P, I, P, P, P, I, D, I, D, P, P]),
+                "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
+                "orc_threads": (I, []),
+                "orc_set_threads": (None, [I]),
+                "orc_f32_to_f16_array": (None, [P, S, P]),
+                "orc_f16_to_f64_array": (None, [P, S, P]),
+                "orc_f64_to_bf16_array": (None, [P, S, P]),
+                "orc_bf16_to_f64_array": (None, [P, S, P]),
+            }
+            for name, (res, args) in sig.items():
+                fn = getattr(lib, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = lib
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# ---------------------------------------------------------------- conversions
+def f32_to_f16_bits(a) -> np.ndarray:
+    a = _c(a, np.float32)
+    out = np.empty(a.shape, np.uint16)
+    _load().orc_f32_to_f16_array(_p(a), a.size, _p(out))
+    return out
+
+
+def f16_bits_to_f64(a) -> np.ndarray:
+    a = _c(a, np.uint16)
+    out = np.empty(a.shape, np.float64)
+    _load().orc_f16_to_f64_array(_p(a), a.size, _p(out))
+    return out
+
+
+def f64_to_bf16_bits(a) -> np.ndarray:
+    a = _c(a, np.float64)
+    out = np.empty(a.shape, np.uint16)
+    _load().orc_f64_to_bf16_array(_p(a), a.size, _p(out))
+    return out
+
+
+def bf16_bits_to_f64(a) -> np.ndarray:
+    a = _c(a, np.uint16)
+    out = np.empty(a.shape, np.float64)
+    _load().orc_bf16_to_f64_array(_p(a), a.size, _p(out))
+    return out
+
+
+# --------------------------------------------------------------- quantization
+def quantize(w, group: int, bits: int):
+    """Stage-1 RTN quantization of an fp32 [n, k] matrix -> (q u8, s f16 bits, z f16 bits, nonfinite)."""
+    w = _c(w, np.float32)
+    n, k = w.shape
+    q = np.empty((n, k), np.uint8)
+    s = np.empty((n, k // group), np.uint16)
+    z = np.empty((n, k // group), np.uint16)
+    rc = _load().orc_quantize(_p(w), n, k, group, bits, _p(q), _p(s), _p(z))
+    if rc < 0:
+        raise ValueError("orc_quantize: bad arguments")
+    return q, s, z, rc
+
+
+def packed_sizes(n: int, k: int, group: int, bits: int):
+    """(code words, meta halves) of the packed format for an [n, k] matrix."""
+    rt, kb = (n + 15) // 16, (k + 127) // 128
+    wpb = 128 if bits == 2 else 256
+    return rt * kb * wpb, rt * (kb * 128 // group) * 32
+
+
+def tile_pack(q, s, z, group: int, bits: int):
+    q = _c(q, np.uint8)
+    s = _c(s, np.uint16)
+    z = _c(z, np.uint16)
+    n, k = q.shape
+    nw, nm = packed_sizes(n, k, group, bits)
+    codes = np.empty(nw, np.uint32)
+    meta = np.empty(nm, np.uint16)
+    if _load().orc_tile_pack(_p(q), _p(s), _p(z), n, k, group, bits, _p(codes), _p(meta)) < 0:
+        raise ValueError("orc_tile_pack: bad arguments")
+    return codes, meta
+
+
+def tile_unpack(codes, meta, n: int, k: int, group: int, bits: int):
+    codes = _c(codes, np.uint32)
+    meta = _c(meta, np.uint16)
+    q = np.empty((n, k), np.uint8)
+    s = np.empty((n, k // group), np.uint16)
+    z = np.empty((n, k // group), np.uint16)
+    if _load().orc_tile_unpack(_p(codes), _p(meta), n, k, group, bits, _p(q), _p(s), _p(z)) < 0:
+        raise ValueError("orc_tile_unpack: bad arguments")
+    return q, s, z
+
+
+def dequant(q, s, z, group: int) -> np.ndarray:
+    q = _c(q, np.uint8)
+    s = _c(s, np.uint16)
+    z = _c(z, np.uint16)
+    n, k = q.shape
+    w = np.empty((n, k), np.float64)
+    if _load().orc_dequant(_p(q), _p(s), _p(z), n, k, group, _p(w)) < 0:
+        raise ValueError("orc_dequant: bad arguments")
+    return w
+
+
+# -------------------------------------------------------------------- forward
+def prenorm(x_bits, eps: float = RMS_EPS) -> np.ndarray:
+    x = _c(x_bits, np.uint16)
+    m, d = x.shape
+    out = np.empty_like(x)
+    _load().orc_prenorm(_p(x), m, d, eps, _p(out))
+    return out
+
+
+def gateup(x_bits, gate, up, group: int, lora_a=None, lora_bg=None, lora_bu=None,
+           lora_scale: float = 0.0, prenorm: bool = False, eps: float = RMS_EPS):
+    """h = SiLU(g) * u with unmerged LoRA.  gate / up are (q, s, z) tuples.
+
+    Returns (h_f64 [m, inter], h_bf16_bits [m, inter]).
+    """
+    x = _c(x_bits, np.uint16)
+    m, d = x.shape
+    qg, sg, zg = (_c(gate[0], np.uint8), _c(gate[1], np.uint16), _c(gate[2], np.uint16))
+    qu, su, zu = (_c(up[0], np.uint8), _c(up[1], np.uint16), _c(up[2], np.uint16))
+    inter = qg.shape[0]
+    if lora_a is None:
+        r = 0
+        la = lbg = lbu = np.zeros(1, np.uint16)
+    else:
+        la, lbg, lbu = _c(lora_a, np.uint16), _c(lora_bg, np.uint16), _c(lora_bu, np.uint16)
+        r = lbg.shape[1]
+    h = np.empty((m, inter), np.float64)
+    hb = np.empty((m, inter), np.uint16)
+    rc = _load().orc_gateup(_p(x), m, d, inter, _p(qg), _p(sg), _p(zg), _p(qu), _p(su), _p(zu),
+                            group, _p(la), _p(lbg), _p(lbu), r, float(lora_scale), int(bool(prenorm)),
+                            float(eps), _p(h), _p(hb))
+    if rc < 0:
+        raise ValueError("orc_gateup: bad arguments")
+    return h, hb
+
+
+def down(h_bits, wd, group: int, residual_bits=None):
+    """y = residual + h deq(Wd)^T.  wd is a (q, s, z) tuple.  Returns (y_f64, y_bf16_bits)."""
+    h = _c(h_bits, np.uint16)
+    m, inter = h.shape
+    q, s, z = (_c(wd[0], np.uint8), _c(wd[1], np.uint16), _c(wd[2], np.uint16))
+    d = q.shape[0]
+    res = None if residual_bits is None else _c(residual_bits, np.uint16)
+    y = np.empty((m, d), np.float64)
+    yb = np.empty((m, d), np.uint16)
+    rc = _load().orc_down(_p(h), m, inter, d, _p(q), _p(s), _p(z), group, _p(res), _p(y), _p(yb))
+    if rc < 0:
+        raise ValueError("orc_down: bad arguments")
+    return y, yb
+
+
+def threads() -> int:
+    return _load().orc_threads()
+
+
+def set_threads(n: int) -> None:
+    _load().orc_set_threads(int(n))

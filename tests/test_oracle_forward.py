@@ -1,0 +1,139 @@
+"""Pins for the oracle's forward pass (Eq. 1 LoRA, Sec. 3.3 gated MLP).
+
+Checked against library routines and closed forms: numpy fp64 matmul of a
+dequantized matrix written out independently, torch's fp64 SiLU and RMSNorm,
+the LoRA-zero and B = 0 special cases, and a rank-1 closed form.
+"""
+import numpy as np
+import pytest
+import torch
+
+
+def _np_deq(q, s_bits, z_bits, group):
+    s = np.repeat(s_bits.view(np.float16).astype(np.float64), group, axis=1)
+    z = np.repeat(z_bits.view(np.float16).astype(np.float64), group, axis=1)
+    return s * (q.astype(np.float64) - z)
+
+
+def _bf16_to_f64(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).double().numpy()
+
+
+def _rand_bf16(rng, shape, std=1.0):
+    t = torch.from_numpy(rng.standard_normal(shape) * std).float().to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def _layer(orc, rng, d, inter, group_gu, group_d, bits_gu=2):
+    wg = (rng.standard_normal((inter, d)) * 0.02).astype(np.float32)
+    wu = (rng.standard_normal((inter, d)) * 0.02).astype(np.float32)
+    wd = (rng.standard_normal((d, inter)) * 0.02).astype(np.float32)
+    g = orc.quantize(wg, group_gu, bits_gu)[:3]
+    u = orc.quantize(wu, group_gu, bits_gu)[:3]
+    dn = orc.quantize(wd, group_d, 4)[:3] if inter % group_d == 0 else None
+    return g, u, dn
+
+
+def test_dequant_matches_numpy(orc):
+    rng = np.random.default_rng(0)
+    w = (rng.standard_normal((40, 256)) * 0.02).astype(np.float32)
+    q, s, z, _ = orc.quantize(w, 64, 2)
+    np.testing.assert_array_equal(orc.dequant(q, s, z, 64), _np_deq(q, s, z, 64))
+
+
+@pytest.mark.parametrize("m", [1, 3])
+def test_gateup_no_lora_matches_numpy_matmul(orc, m):
+    rng = np.random.default_rng(m)
+    d, inter = 256, 96
+    g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    x = _rand_bf16(rng, (m, d))
+    h, hb = orc.gateup(x, g, u, 64)
+    xf = _bf16_to_f64(x)
+    gg = xf @ _np_deq(*g, 64).T
+    uu = xf @ _np_deq(*u, 64).T
+    want = torch.nn.functional.silu(torch.from_numpy(gg)).numpy() * uu
+    np.testing.assert_allclose(h, want, rtol=1e-12, atol=1e-14)
+    # the bf16 output is the round-to-nearest of the fp64 value
+    np.testing.assert_array_equal(hb, orc.f64_to_bf16_bits(h))
+
+
+def test_lora_special_cases(orc):
+    rng = np.random.default_rng(3)
+    d, inter, r = 256, 80, 8
+    g, u, _ = _layer(orc, rng, d, inter, 128, 128)
+    x = _rand_bf16(rng, (2, d))
+    a = _rand_bf16(rng, (2 * r, d), 0.01)
+    bg = _rand_bf16(rng, (inter, r), 0.01)
+    bu = _rand_bf16(rng, (inter, r), 0.01)
+    base, _ = orc.gateup(x, g, u, 128)
+    h0, _ = orc.gateup(x, g, u, 128, a, bg, bu, lora_scale=0.0)
+    np.testing.assert_array_equal(h0, base)
+    zeros = np.zeros_like(bg)
+    hz, _ = orc.gateup(x, g, u, 128, a, zeros, zeros, lora_scale=2.0)
+    np.testing.assert_array_equal(hz, base)
+    h1, _ = orc.gateup(x, g, u, 128, a, bg, bu, lora_scale=2.0)
+    assert np.max(np.abs(h1 - base)) > 1e-6
+
+
+def test_lora_rank1_closed_form(orc):
+    # r = 1: g = x Wg^T + alpha (x . a_g) b_g, u likewise.
+    rng = np.random.default_rng(4)
+    d, inter = 128, 48
+    g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    x = _rand_bf16(rng, (1, d))
+    a = _rand_bf16(rng, (2, d), 0.1)
+    bg = _rand_bf16(rng, (inter, 1), 0.1)
+    bu = _rand_bf16(rng, (inter, 1), 0.1)
+    alpha = 1.75
+    h, _ = orc.gateup(x, g, u, 64, a, bg, bu, lora_scale=alpha)
+    xf, af = _bf16_to_f64(x)[0], _bf16_to_f64(a)
+    gg = _np_deq(*g, 64) @ xf + alpha * (xf @ af[0]) * _bf16_to_f64(bg)[:, 0]
+    uu = _np_deq(*u, 64) @ xf + alpha * (xf @ af[1]) * _bf16_to_f64(bu)[:, 0]
+    want = gg / (1 + np.exp(-gg)) * uu
+    np.testing.assert_allclose(h[0], want, rtol=1e-12, atol=1e-14)
+
+
+def test_prenorm_matches_torch_rms_norm(orc):
+    rng = np.random.default_rng(5)
+    x = _rand_bf16(rng, (4, 512), 3.0)
+    got = _bf16_to_f64(orc.prenorm(x))
+    xt = torch.from_numpy(_bf16_to_f64(x))
+    want = torch.nn.functional.rms_norm(xt, (512,), eps=1e-6).numpy()
+    # the oracle rounds once to bf16: within half a bf16 ulp of the fp64 value
+    spacing = 2.0 ** (np.floor(np.log2(np.abs(want))) - 7)
+    assert np.all(np.abs(got - want) <= spacing * 0.5 * (1 + 1e-9))
+
+
+def test_gateup_prenorm_equals_gateup_of_normalized(orc):
+    rng = np.random.default_rng(6)
+    d, inter = 256, 64
+    g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    x = _rand_bf16(rng, (2, d), 5.0)
+    h1, _ = orc.gateup(x, g, u, 64, prenorm=True)
+    h2, _ = orc.gateup(orc.prenorm(x), g, u, 64, prenorm=False)
+    np.testing.assert_array_equal(h1, h2)
+
+
+def test_down_with_residual_matches_numpy(orc):
+    rng = np.random.default_rng(7)
+    d, inter = 96, 256
+    wd = (rng.standard_normal((d, inter)) * 0.02).astype(np.float32)
+    dn = orc.quantize(wd, 64, 4)[:3]
+    h = _rand_bf16(rng, (3, inter))
+    res = _rand_bf16(rng, (3, d))
+    y, yb = orc.down(h, dn, 64, res)
+    want = _bf16_to_f64(res) + _bf16_to_f64(h) @ _np_deq(*dn, 64).T
+    np.testing.assert_allclose(y, want, rtol=1e-12, atol=1e-13)
+    y0, _ = orc.down(h, dn, 64, None)
+    np.testing.assert_allclose(y0, _bf16_to_f64(h) @ _np_deq(*dn, 64).T, rtol=1e-12, atol=1e-13)
+    np.testing.assert_array_equal(yb, orc.f64_to_bf16_bits(y))
+
+
+def test_empty_token_batch(orc):
+    rng = np.random.default_rng(8)
+    g, u, dn = _layer(orc, rng, 128, 64, 64, 64)
+    x = np.zeros((0, 128), np.uint16)
+    h, hb = orc.gateup(x, g, u, 64)
+    assert h.shape == (0, 64)
+    y, _ = orc.down(hb, dn, 64, x)
+    assert y.shape == (0, 128)
