@@ -1,0 +1,202 @@
+/*
+ * wq.h -- C ABI of the W4/W2-GateUp decode MLP library (libwq.so, sm_103a).
+ *
+ * The library computes the decode-regime gated-MLP block of the W4/W2-GateUp
+ * scheme: gate and up projections quantized to 2 bits, the down projection
+ * to 4 bits (Sec. 3.3), with the Recover-LoRA adapters left unmerged on gate
+ * and up (Eq. 1, Y = W X + alpha B A X; Sec. 4.2 allows deploying them either
+ * merged or as an extra low-rank path, and this library takes the second
+ * option).  The quantizer is the Stage-1 group-wise post-training
+ * quantization of Sec. 4.1.
+ *
+ * Conventions shared by every call:
+ *   - All tensor arguments are DEVICE pointers owned by the caller.  The
+ *     library never allocates device memory and never synchronizes; every
+ *     call is asynchronous on `stream` (a cudaStream_t, NULL = legacy default
+ *     stream).  Argument errors are detected on the host before any launch.
+ *   - Device pointers must be 16-byte aligned (WQ_ERR_ALIGN otherwise).
+ *   - Weights are row-major [out, in] (W in R^{d x k}, Y = W X, Eq. 1).
+ *     Activations are token-major [m, features].  bf16 tensors are passed as
+ *     `void*` holding IEEE bfloat16 values.
+ *   - Quantized weights use the packed format described at wq_qweight.
+ *   - Supported: group in {32, 64, 128}; in-features a multiple of the group
+ *     (WQ_ERR_SHAPE otherwise); 1 <= m <= 64 tokens (m == 0 is a no-op);
+ *     LoRA rank r a multiple of 8, r <= 64 (r == 0: no adapter).
+ *   - On error the call returns a negative wq_status and wq_last_error()
+ *     describes it (per host thread).  Kernel-side waits are bounded; a wait
+ *     that runs out records WQ_ERR_TIMEOUT, read back by wq_device_status().
+ */
+#ifndef WQ_H
+#define WQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    WQ_OK = 0,
+    WQ_ERR_ARG = -1,          /* null pointer, negative size, bad flag */
+    WQ_ERR_SHAPE = -2,        /* shapes inconsistent or outside the supported set */
+    WQ_ERR_ALIGN = -3,        /* a device pointer is not 16-byte aligned */
+    WQ_ERR_UNSUPPORTED = -4,  /* valid request this build does not implement */
+    WQ_ERR_CUDA = -5,         /* a CUDA runtime call or launch failed */
+    WQ_ERR_TIMEOUT = -6,      /* a bounded device-side wait ran out */
+    WQ_ERR_WORKSPACE = -7     /* workspace missing or smaller than required */
+} wq_status;
+
+/* Flags of wq_gateup_* and wq_mlp_forward. */
+#define WQ_PRENORM 1u   /* unit-weight RMSNorm (eps 1e-6) of the MLP input first */
+
+/* Output element types of wq_down_w4. */
+#define WQ_BF16 0
+#define WQ_F32 1
+
+/*
+ * A group-quantized weight matrix W[n, k] (n output rows, k input features)
+ * in the packed format (device memory, caller-owned):
+ *
+ *   Rows are padded to a multiple of 16 and k to a multiple of 128 with
+ *   codes 0 and scales/zeros 0.  RT = ceil(n/16) row tiles, KB = ceil(k/128)
+ *   feature blocks, NG = KB*128/group groups per row.
+ *
+ *   codes: uint32 words; block (rt, kb) of 16 rows x 128 features starts at
+ *   word (rt*KB + kb) * WPB, WPB = 128 (bits 2) or 256 (bits 4).  The code of
+ *   local row i and local feature c sits at
+ *       lane = (i%8)*4 + (c%8)/2,  half = c%2
+ *       bits 2: word = lane*4 + c/32,
+ *               bit  = 16*half + 8*(i/8) + 2*(2*((c%32)/16) + (c%16)/8)
+ *       bits 4: word = (c/64)*128 + lane*4 + (c%64)/16,
+ *               bit  = 16*half + 8*(i/8) + 4*((c%16)/8)
+ *   so that one 16-byte load per lane yields that lane's m16n8k16 tensor-core
+ *   A fragments for a whole 128-feature block (64 codes of 2 bits) or a
+ *   64-feature half block (32 codes of 4 bits).
+ *
+ *   meta: binary16 scale s and zero z per (row, group): 32 values per
+ *   (rt, group j) at (rt*NG + j)*32, for e = 0..7:
+ *       [4e] = s[16rt+e], [4e+1] = s[16rt+e+8], [4e+2] = z[16rt+e], [4e+3] = z[16rt+e+8].
+ *
+ *   Dequantized weight: W[r, c] = s[r, c/group] * (code[r, c] - z[r, c/group]).
+ */
+typedef struct {
+    uint32_t *codes;
+    uint16_t *meta;
+    int32_t n, k, group, bits;
+} wq_qweight;
+
+/* One gated-MLP layer: h = SiLU(gate x + a_g) * (up x + a_u), y = x + down h,
+ * with the unmerged LoRA terms a_g = lora_scale * (x A_g^T) B_g^T and a_u likewise
+ * (Eq. 1; alpha of Eq. 1 is lora_scale, e.g. alpha/r in the PEFT convention). */
+typedef struct {
+    wq_qweight gate, up, down;   /* gate/up: n = inter, k = d.  down: n = d, k = inter */
+    const void *lora_a;          /* bf16 [2r, d]: rows 0..r-1 = A_gate, r..2r-1 = A_up; NULL if r == 0 */
+    const void *lora_b_gate;     /* bf16 [inter, r] */
+    const void *lora_b_up;       /* bf16 [inter, r] */
+    int32_t r;
+    float lora_scale;
+} wq_mlp_layer;
+
+/* Sizes in bytes of the packed codes and meta buffers of an [n, k] matrix.
+ * Returns WQ_ERR_SHAPE for an unsupported (bits, group) or k % group != 0. */
+wq_status wq_packed_sizes(int bits, int n, int k, int group, size_t *code_bytes, size_t *meta_bytes);
+
+/*
+ * Stage-1 quantization and packing (Sec. 4.1 selective INT2 quantization of
+ * gate/up; INT4 for the remaining layers, Sec. 3.3 and Sec. 6 step 4).
+ * Asymmetric min-max round-to-nearest per group of `group` consecutive input
+ * features of each row, in IEEE fp32:
+ *     s = fp16((max - min) / qmax)  (1.0 if that is zero),
+ *     z = clamp(rint(-min / s), 0, qmax),  q = clamp(rint(w / s) + z, 0, qmax),
+ * qmax = 2^bits - 1, rint ties-to-even, divisions IEEE-exact.
+ *   w:         fp32 [n, k] row-major, device.
+ *   out:       host struct whose codes/meta point to device buffers of the
+ *              sizes wq_packed_sizes() gives; n, k, group, bits are filled in.
+ *   nonfinite: optional device int; the kernel ORs 1 into it if any weight is
+ *              NaN or infinite (the caller reads it after synchronizing).
+ */
+wq_status wq_pack(const float *w, int n, int k, int group, int bits, wq_qweight *out,
+                  int *nonfinite, void *stream);
+wq_status wq_pack_w2(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream);
+wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream);
+
+/*
+ * Workspace (device scratch, caller-owned) needed by wq_gateup_*, wq_down_w4
+ * and wq_mlp_forward for up to m tokens of a layer of hidden size d,
+ * intermediate size inter and LoRA rank r, on the current device.  Before its
+ * first use a workspace must be zero-filled (wq_workspace_init); every call
+ * leaves its internal arrival counters at zero again (after a call whose
+ * device status reads WQ_ERR_TIMEOUT, zero it again).  Calls that share a
+ * workspace must not overlap in time on the GPU.
+ */
+size_t wq_workspace_bytes(int m, int d, int inter, int r);
+wq_status wq_workspace_init(void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * Fused 2-bit gate/up projection with unmerged LoRA and SiLU(gate) * up
+ * (Eq. 1 on gate and up; gated MLP of Sec. 3.3; gate, activation and product
+ * fused in one kernel as in the fused MLP modelling of Sec. 5):
+ *     xin = (flags & WQ_PRENORM) ? bf16(RMSNorm(x)) : x
+ *     g   = xin deq(Wg)^T + lora_scale * (xin A_g^T) B_g^T      (fp32 accumulate)
+ *     u   = xin deq(Wu)^T + lora_scale * (xin A_u^T) B_u^T
+ *     h   = bf16( g / (1 + exp(-g)) * u )
+ *   x: bf16 [m, d].  gate, up: bits 2, n = inter, k = d.  lora_*: see
+ *   wq_mlp_layer (r == 0 and NULLs: no adapter).  h: bf16 [m, inter].
+ */
+wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                            const void *lora_a, const void *lora_b_gate, const void *lora_b_up,
+                            int r, float lora_scale, unsigned flags, void *h,
+                            void *ws, size_t ws_bytes, void *stream);
+
+/* The uniform-W4 comparator: the same block with 4-bit gate/up and no LoRA. */
+wq_status wq_gateup_w4(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                       unsigned flags, void *h, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * 4-bit down projection with optional residual (Sec. 3.3: down stays INT4):
+ *     y = residual + h deq(Wd)^T
+ *   h: bf16 [m, inter].  down: bits 4, n = d, k = inter.  residual: bf16
+ *   [m, d] or NULL.  y: [m, d] of y_dtype (WQ_BF16 rounds to nearest even,
+ *   WQ_F32 stores the fp32 accumulator).
+ */
+wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *residual,
+                     void *y, int y_dtype, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * A stack of gated-MLP layers for one decode step of m tokens:
+ *     x_0 = x,  x_{l+1} = x_l + down_l( SiLU(gate_l(xin_l)) * up_l(xin_l) ),  y = x_L
+ * with xin_l = RMSNorm(x_l) when flags has WQ_PRENORM, else x_l.  Each layer's
+ * gate/up are 2-bit (with LoRA) or 4-bit (no LoRA); down is 4-bit.  x, y:
+ * bf16 [m, d]; the residual stream is stored in bf16 between layers.  The
+ * call launches every kernel on `stream` with programmatic dependent launch
+ * and can be captured into a CUDA graph.
+ */
+wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
+                         unsigned flags, void *y, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * Describes how a dequant-GEMV launch of the current device splits its work
+ * (for tests and tuning; launches nothing).  kind: 0 = 2-bit gate/up,
+ * 1 = 4-bit gate/up, 2 = 4-bit down.  n, k: matrix shape; m tokens; r LoRA
+ * rank.  info[0..9] receives: row tiles, 128-feature blocks, row tiles per
+ * CTA, blocks per panel, warps along k, panels, CTAs, threads per CTA,
+ * dynamic shared memory bytes, tokens per MMA chunk.
+ */
+wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t info[10]);
+
+/* Message of the last error returned on this host thread ("" if none). */
+const char *wq_last_error(void);
+
+/* Reads and clears the device-side status word (WQ_OK or WQ_ERR_TIMEOUT) of
+ * the current device.  Synchronizes the device. */
+wq_status wq_device_status(int *status);
+
+/* Library version string. */
+const char *wq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WQ_H */

@@ -1,0 +1,395 @@
+// wq_api.cu -- the C ABI of include/wq.h: argument validation, workspace
+// layout, launch sequencing.  Every check happens on the host before any
+// launch; nothing here allocates device memory or synchronizes (except
+// wq_device_status, which is documented to).
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <algorithm>
+#include <string>
+
+#include "wq.h"
+#include "wq_internal.h"
+
+using namespace wq;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+wq_status fail(wq_status st, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+wq_status ok() {
+  g_last_error.clear();
+  return WQ_OK;
+}
+
+wq_status cuda_fail(cudaError_t e, const char *what) {
+  return fail(WQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool group_ok(int g) { return g == 32 || g == 64 || g == 128; }
+
+int num_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cached[dev] = v;
+  }
+  return cached[dev];
+}
+
+wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
+  if (!q) return fail(WQ_ERR_ARG, "%s: null wq_qweight", name);
+  if (!q->codes || !q->meta) return fail(WQ_ERR_ARG, "%s: null codes or meta pointer", name);
+  if (!aligned16(q->codes) || !aligned16(q->meta)) return fail(WQ_ERR_ALIGN, "%s: codes/meta not 16-byte aligned", name);
+  if (q->bits != bits) return fail(WQ_ERR_SHAPE, "%s: bits %d, expected %d", name, q->bits, bits);
+  if (q->n <= 0 || q->k <= 0) return fail(WQ_ERR_SHAPE, "%s: bad shape [%d, %d]", name, q->n, q->k);
+  if (!group_ok(q->group)) return fail(WQ_ERR_SHAPE, "%s: group %d not in {32, 64, 128}", name, q->group);
+  if (q->k % q->group != 0) return fail(WQ_ERR_SHAPE, "%s: k=%d not a multiple of group %d", name, q->k, q->group);
+  return WQ_OK;
+}
+
+// Byte layout of the workspace for up to m tokens of a (d, inter) layer.
+struct WsLayout {
+  size_t t, xhat, xa, xb, h, cnt1, cnt2, part1, part2, total;
+};
+
+size_t up256(size_t v) { return (v + 255) / 256 * 256; }
+
+size_t partial_bytes(const GemvPlan &p, int nproj) {
+  return p.P > 1 ? (size_t)p.RT * p.P * nproj * 16 * p.MPAD * 4 : 0;
+}
+
+// Largest split-K partial buffer any plan of this shape can need.
+bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2) {
+  const int sms = num_sms();
+  if (sms <= 0) return false;
+  *p1 = *p2 = 0;
+  const int groups[3] = {32, 64, 128};
+  for (int g : groups) {
+    for (int r = 0; r <= kMaxRank; r += 8) {
+      GemvPlan pl;
+      if (d % g == 0) {
+        if (plan_gemv(kGateUpW2, inter, d, m, g, r, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
+        if (r == 0 && plan_gemv(kGateUpW4, inter, d, m, g, 0, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
+      }
+    }
+    GemvPlan pl;
+    if (inter % g == 0 && plan_gemv(kDownW4, d, inter, m, g, 0, sms, &pl)) *p2 = std::max(*p2, partial_bytes(pl, 1));
+  }
+  return true;
+}
+
+// The arrival counters come first: their offsets depend on (d, inter) only,
+// so a workspace zeroed once stays valid for every token count.
+bool ws_layout(int m, int d, int inter, WsLayout *L) {
+  size_t p1, p2;
+  if (!max_partials(m, d, inter, &p1, &p2)) return false;
+  size_t off = 0;
+  L->cnt1 = off; off = up256(off + (size_t)((inter + 15) / 16) * 4);
+  L->cnt2 = off; off = up256(off + (size_t)((d + 15) / 16) * 4);
+  L->t = off;    off = up256(off + (size_t)m * 2 * kMaxRank * 4);
+  L->xhat = off; off = up256(off + (size_t)m * d * 2);
+  L->xa = off;   off = up256(off + (size_t)m * d * 2);
+  L->xb = off;   off = up256(off + (size_t)m * d * 2);
+  L->h = off;    off = up256(off + (size_t)m * inter * 2);
+  L->part1 = off; off = up256(off + p1);
+  L->part2 = off; off = up256(off + p2);
+  L->total = off;
+  return true;
+}
+
+// gate/up (2-bit with LoRA, or 4-bit) for one layer.
+wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                     const void *lora_a, const void *lora_bg, const void *lora_bu, int r, float lora_scale,
+                     unsigned flags, void *h, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+  const int d = gate->k, inter = gate->n;
+  const bool prenorm = (flags & WQ_PRENORM) != 0;
+  GemvPlan plan;
+  if (!plan_gemv(kind, inter, d, m, gate->group, r, num_sms(), &plan))
+    return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits [%d x %d], m=%d, group %d", inter, d, m, gate->group);
+  float *t = reinterpret_cast<float *>(ws + L.t);
+  void *xhat = ws + L.xhat;
+  if (prenorm || r > 0) {
+    cudaError_t e = launch_prep(x, m, d, lora_a, r, prenorm ? 1 : 0, xhat, t, s, true);
+    if (e != cudaSuccess) return cuda_fail(e, "prologue launch");
+  }
+  GemvArgs a = {};
+  a.act = prenorm ? xhat : x;
+  a.M = m;
+  a.K = d;
+  a.N = inter;
+  a.group = gate->group;
+  a.codes[0] = gate->codes;
+  a.codes[1] = up->codes;
+  a.meta[0] = gate->meta;
+  a.meta[1] = up->meta;
+  a.t = t;
+  a.lora_b[0] = lora_bg;
+  a.lora_b[1] = lora_bu;
+  a.r = r;
+  a.lora_scale = lora_scale;
+  a.out = h;
+  a.partials = reinterpret_cast<float *>(ws + L.part1);
+  a.counters = reinterpret_cast<unsigned *>(ws + L.cnt1);
+  cudaError_t e = launch_gemv(kind, plan, a, s, true);
+  if (e != cudaSuccess) return cuda_fail(e, "gate/up launch");
+  return WQ_OK;
+}
+
+wq_status run_down(const void *h, int m, const wq_qweight *down, const void *residual, void *y, int y_f32,
+                   const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+  GemvPlan plan;
+  if (!plan_gemv(kDownW4, down->n, down->k, m, down->group, 0, num_sms(), &plan))
+    return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits [%d x %d], m=%d", down->n, down->k, m);
+  GemvArgs a = {};
+  a.act = h;
+  a.M = m;
+  a.K = down->k;
+  a.N = down->n;
+  a.group = down->group;
+  a.codes[0] = down->codes;
+  a.meta[0] = down->meta;
+  a.residual = residual;
+  a.out = y;
+  a.out_f32 = y_f32;
+  a.partials = reinterpret_cast<float *>(ws + L.part2);
+  a.counters = reinterpret_cast<unsigned *>(ws + L.cnt2);
+  cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);
+  if (e != cudaSuccess) return cuda_fail(e, "down launch");
+  return WQ_OK;
+}
+
+wq_status check_tokens(int m) {
+  if (m < 0) return fail(WQ_ERR_ARG, "m=%d is negative", m);
+  if (m > kMaxTokens) return fail(WQ_ERR_UNSUPPORTED, "m=%d exceeds the %d-token limit of this build", m, kMaxTokens);
+  return WQ_OK;
+}
+
+wq_status check_ws(void *ws, size_t ws_bytes, int m, int d, int inter, WsLayout *L) {
+  if (!ws_layout(m, d, inter, L)) return fail(WQ_ERR_CUDA, "cannot query the current device");
+  if (!ws) return fail(WQ_ERR_WORKSPACE, "null workspace");
+  if (!aligned16(ws)) return fail(WQ_ERR_ALIGN, "workspace not 16-byte aligned");
+  if (ws_bytes < L->total)
+    return fail(WQ_ERR_WORKSPACE, "workspace of %zu bytes, %zu needed (wq_workspace_bytes)", ws_bytes, L->total);
+  return WQ_OK;
+}
+
+wq_status check_lora(const void *lora_a, const void *bg, const void *bu, int r) {
+  if (r == 0) return WQ_OK;
+  if (r < 0 || r % 8 != 0 || r > kMaxRank) return fail(WQ_ERR_SHAPE, "LoRA rank %d not a multiple of 8 in [8, 64]", r);
+  if (!lora_a || !bg || !bu) return fail(WQ_ERR_ARG, "null LoRA pointer with r=%d", r);
+  if (!aligned16(lora_a) || !aligned16(bg) || !aligned16(bu)) return fail(WQ_ERR_ALIGN, "LoRA pointers not 16-byte aligned");
+  return WQ_OK;
+}
+
+wq_status check_gateup_pair(const wq_qweight *gate, const wq_qweight *up, int bits) {
+  wq_status st = check_qweight(gate, bits, "gate");
+  if (st != WQ_OK) return st;
+  if ((st = check_qweight(up, bits, "up")) != WQ_OK) return st;
+  if (gate->n != up->n || gate->k != up->k || gate->group != up->group)
+    return fail(WQ_ERR_SHAPE, "gate [%d x %d g%d] and up [%d x %d g%d] differ", gate->n, gate->k, gate->group, up->n,
+                up->k, up->group);
+  return WQ_OK;
+}
+
+wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                       const void *lora_a, const void *bg, const void *bu, int r, float lora_scale, unsigned flags,
+                       void *h, void *ws, size_t ws_bytes, void *stream) {
+  wq_status st = check_tokens(m);
+  if (st != WQ_OK) return st;
+  if ((st = check_gateup_pair(gate, up, kind == kGateUpW2 ? 2 : 4)) != WQ_OK) return st;
+  if ((st = check_lora(lora_a, bg, bu, r)) != WQ_OK) return st;
+  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (m == 0) return ok();
+  if (!x || !h) return fail(WQ_ERR_ARG, "null x or h");
+  if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
+  WsLayout L;
+  if ((st = check_ws(ws, ws_bytes, m, gate->k, gate->n, &L)) != WQ_OK) return st;
+  st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, L, static_cast<uint8_t *>(ws),
+                  static_cast<cudaStream_t>(stream));
+  return st == WQ_OK ? ok() : st;
+}
+
+}  // namespace
+
+extern "C" {
+
+wq_status wq_packed_sizes(int bits, int n, int k, int group, size_t *code_bytes, size_t *meta_bytes) {
+  if (bits != 2 && bits != 4) return fail(WQ_ERR_SHAPE, "bits %d not in {2, 4}", bits);
+  if (!group_ok(group)) return fail(WQ_ERR_SHAPE, "group %d not in {32, 64, 128}", group);
+  if (n < 0 || k < 0 || k % group != 0) return fail(WQ_ERR_SHAPE, "bad shape [%d, %d] for group %d", n, k, group);
+  const size_t RT = (size_t)(n + 15) / 16, KB = (size_t)(k + 127) / 128;
+  if (code_bytes) *code_bytes = RT * KB * (bits == 2 ? 512 : 1024);
+  if (meta_bytes) *meta_bytes = RT * (KB * 128 / group) * 64;
+  return ok();
+}
+
+wq_status wq_pack(const float *w, int n, int k, int group, int bits, wq_qweight *out, int *nonfinite, void *stream) {
+  size_t cb, mb;
+  wq_status st = wq_packed_sizes(bits, n, k, group, &cb, &mb);
+  if (st != WQ_OK) return st;
+  if (!out) return fail(WQ_ERR_ARG, "null output wq_qweight");
+  if (n == 0 || k == 0) return fail(WQ_ERR_SHAPE, "empty matrix [%d, %d]", n, k);
+  if (!w || !out->codes || !out->meta) return fail(WQ_ERR_ARG, "null weight, codes or meta pointer");
+  if (!aligned16(w) || !aligned16(out->codes) || !aligned16(out->meta))
+    return fail(WQ_ERR_ALIGN, "weight, codes or meta pointer not 16-byte aligned");
+  cudaError_t e = launch_pack(w, n, k, group, bits, out->codes, out->meta, nonfinite, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "pack launch");
+  out->n = n;
+  out->k = k;
+  out->group = group;
+  out->bits = bits;
+  return ok();
+}
+
+wq_status wq_pack_w2(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream) {
+  return wq_pack(w, n, k, group, 2, out, nonfinite, stream);
+}
+
+wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream) {
+  return wq_pack(w, n, k, group, 4, out, nonfinite, stream);
+}
+
+size_t wq_workspace_bytes(int m, int d, int inter, int r) {
+  (void)r;  // the LoRA-A product area is sized for the largest supported rank
+  if (m <= 0 || d <= 0 || inter <= 0 || m > kMaxTokens) return 0;
+  size_t most = 0;  // enough for every token count up to m
+  for (int mm = 1; mm <= m; ++mm) {
+    WsLayout L;
+    if (!ws_layout(mm, d, inter, &L)) return 0;
+    most = std::max(most, L.total);
+  }
+  return most;
+}
+
+wq_status wq_workspace_init(void *ws, size_t ws_bytes, void *stream) {
+  if (!ws) return fail(WQ_ERR_WORKSPACE, "null workspace");
+  cudaError_t e = cudaMemsetAsync(ws, 0, ws_bytes, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "workspace clear");
+  return ok();
+}
+
+wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const wq_qweight *up, const void *lora_a,
+                            const void *lora_b_gate, const void *lora_b_up, int r, float lora_scale, unsigned flags,
+                            void *h, void *ws, size_t ws_bytes, void *stream) {
+  return gateup_entry(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, ws, ws_bytes,
+                      stream);
+}
+
+wq_status wq_gateup_w4(const void *x, int m, const wq_qweight *gate, const wq_qweight *up, unsigned flags, void *h,
+                       void *ws, size_t ws_bytes, void *stream) {
+  return gateup_entry(kGateUpW4, x, m, gate, up, nullptr, nullptr, nullptr, 0, 0.f, flags, h, ws, ws_bytes, stream);
+}
+
+wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *residual, void *y, int y_dtype, void *ws,
+                     size_t ws_bytes, void *stream) {
+  wq_status st = check_tokens(m);
+  if (st != WQ_OK) return st;
+  if ((st = check_qweight(down, 4, "down")) != WQ_OK) return st;
+  if (y_dtype != WQ_BF16 && y_dtype != WQ_F32) return fail(WQ_ERR_ARG, "y_dtype %d not WQ_BF16 or WQ_F32", y_dtype);
+  if (m == 0) return ok();
+  if (!h || !y) return fail(WQ_ERR_ARG, "null h or y");
+  if (!aligned16(h) || !aligned16(y) || (residual && !aligned16(residual)))
+    return fail(WQ_ERR_ALIGN, "h, y or residual not 16-byte aligned");
+  WsLayout L;
+  if ((st = check_ws(ws, ws_bytes, m, down->n, down->k, &L)) != WQ_OK) return st;
+  st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
+                static_cast<cudaStream_t>(stream));
+  return st == WQ_OK ? ok() : st;
+}
+
+wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, void *y,
+                         void *ws, size_t ws_bytes, void *stream) {
+  wq_status st = check_tokens(m);
+  if (st != WQ_OK) return st;
+  if (n_layers < 0) return fail(WQ_ERR_ARG, "n_layers=%d is negative", n_layers);
+  if (n_layers > 0 && !layers) return fail(WQ_ERR_ARG, "null layer array");
+  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  int d = 0, inter = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    const wq_mlp_layer &Ly = layers[l];
+    const int bits = Ly.gate.bits;
+    if (bits != 2 && bits != 4) return fail(WQ_ERR_SHAPE, "layer %d: gate bits %d not in {2, 4}", l, bits);
+    if ((st = check_gateup_pair(&Ly.gate, &Ly.up, bits)) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    if ((st = check_qweight(&Ly.down, 4, "down")) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    if (bits == 4 && Ly.r != 0) return fail(WQ_ERR_UNSUPPORTED, "layer %d: LoRA on 4-bit gate/up is not supported", l);
+    if ((st = check_lora(Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r)) != WQ_OK)
+      return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    if (Ly.down.n != Ly.gate.k || Ly.down.k != Ly.gate.n)
+      return fail(WQ_ERR_SHAPE, "layer %d: down [%d x %d] does not match gate/up [%d x %d]", l, Ly.down.n, Ly.down.k,
+                  Ly.gate.n, Ly.gate.k);
+    if (l == 0) {
+      d = Ly.gate.k;
+      inter = Ly.gate.n;
+    } else if (Ly.gate.k != d || Ly.gate.n != inter) {
+      return fail(WQ_ERR_SHAPE, "layer %d: shape [%d x %d] differs from layer 0 [%d x %d]", l, Ly.gate.n, Ly.gate.k,
+                  inter, d);
+    }
+  }
+  if (m == 0 || n_layers == 0) {
+    if (n_layers == 0 && m > 0 && x != y) return fail(WQ_ERR_ARG, "n_layers=0 needs y == x");
+    return ok();
+  }
+  if (!x || !y) return fail(WQ_ERR_ARG, "null x or y");
+  if (!aligned16(x) || !aligned16(y)) return fail(WQ_ERR_ALIGN, "x or y not 16-byte aligned");
+  WsLayout L;
+  if ((st = check_ws(ws, ws_bytes, m, d, inter, &L)) != WQ_OK) return st;
+  uint8_t *w8 = static_cast<uint8_t *>(ws);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const void *cur = x;
+  void *hbuf = w8 + L.h;
+  for (int l = 0; l < n_layers; ++l) {
+    const wq_mlp_layer &Ly = layers[l];
+    void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
+    const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+    st = run_gateup(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale, flags,
+                    hbuf, L, w8, s);
+    if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    st = run_down(hbuf, m, &Ly.down, cur, out, 0, L, w8, s);
+    if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    cur = out;
+  }
+  return ok();
+}
+
+wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t info[10]) {
+  if (!info) return fail(WQ_ERR_ARG, "null info array");
+  if (kind < 0 || kind > 2) return fail(WQ_ERR_ARG, "kind %d not in {0, 1, 2}", kind);
+  if (!group_ok(group) || k % group != 0) return fail(WQ_ERR_SHAPE, "group %d / k %d unsupported", group, k);
+  const int sms = num_sms();
+  if (sms <= 0) return fail(WQ_ERR_CUDA, "cannot query the current device");
+  GemvPlan p;
+  if (!plan_gemv(static_cast<GemvKind>(kind), n, k, m, group, r, sms, &p))
+    return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits");
+  const int64_t v[10] = {p.RT, p.KB, p.RB, p.KP, p.WK, p.P, p.units, p.threads, p.smem, 8 * p.NT};
+  for (int i = 0; i < 10; ++i) info[i] = v[i];
+  return ok();
+}
+
+const char *wq_last_error(void) { return g_last_error.c_str(); }
+
+wq_status wq_device_status(int *status) {
+  if (!status) return fail(WQ_ERR_ARG, "null status pointer");
+  cudaError_t e = read_device_status(status);
+  if (e != cudaSuccess) return cuda_fail(e, "device status read");
+  return ok();
+}
+
+const char *wq_version(void) { return "wq 0.1 (sm_103a)"; }
+
+}  // extern "C"

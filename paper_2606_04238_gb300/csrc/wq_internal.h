@@ -1,0 +1,75 @@
+// wq_internal.h -- types shared by the host-side API (wq_api.cu) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace wq {
+
+constexpr int kMaxTokens = 64;      // tokens per call on the dequant-GEMV path
+constexpr int kMaxRank = 64;        // LoRA rank limit
+constexpr int kMaxWarps = 32;       // warps per CTA
+constexpr float kRmsEps = 1e-6f;    // RMSNorm epsilon of WQ_PRENORM
+
+// How one dequant-GEMV launch splits its work.
+//   Row tiles (16 output rows) are grouped into row blocks of RB tiles; the
+//   input features (128-wide blocks) into P panels of KP blocks.  One CTA
+//   computes one (row block, panel) unit with RB*WK warps: warp (rw, wk)
+//   owns row tile rw of the block and the wk-th share of the panel's blocks.
+//   With P > 1 the panel partial sums of a row tile are added by whichever
+//   CTA finishes that row tile last (arrival counter, fixed summation order).
+struct GemvPlan {
+  int RT, KB;          // row tiles, 128-feature blocks of the whole matrix
+  int RB, KP, WK;      // row tiles per unit, blocks per panel, warps along k
+  int P, NRB;          // panels, row blocks
+  int M, MPAD, NT;     // tokens, tokens padded to the token-chunk size, 8-token tiles per chunk
+  int threads;         // RB * WK * 32
+  int units;           // grid size = NRB * P
+  int lora_smem;       // LoRA B rows staged in shared memory (P == 1 and r > 0)
+  uint32_t smem;       // dynamic shared memory bytes
+  // byte offsets inside dynamic shared memory
+  uint32_t off_codes, off_meta, off_lorab, off_xp, off_xs, off_scale, off_slots, off_t, off_bar, off_last;
+  int xstride;         // halves per token row of the converted activation panel
+};
+
+struct GemvArgs {
+  const void *act;           // bf16 [M, K]
+  int M, K, N, group;
+  const uint32_t *codes[2];  // packed codes of the (one or two) matrices
+  const uint16_t *meta[2];   // packed binary16 scales / zeros
+  const float *t;            // LoRA-A products [M, 2r] fp32 (gate/up with LoRA)
+  const void *lora_b[2];     // bf16 [N, r]
+  int r;
+  float lora_scale;
+  const void *residual;      // bf16 [M, N] or null (down projection)
+  void *out;                 // bf16 or fp32 [M, N]
+  int out_f32;
+  float *partials;           // [RT][P][NPROJ][16][MPAD] fp32 (P > 1)
+  unsigned *counters;        // [RT] arrival counters, zero between calls
+};
+
+enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
+
+// Plans a launch; returns false if no configuration fits.
+bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *plan);
+
+// Launches the dequant-GEMV kernel of `kind` (programmatic dependent launch
+// when `pdl`).  Returns the CUDA error of the launch.
+cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl);
+
+// Launches the prologue kernel: RMSNorm of x (if prenorm) into xhat and the
+// LoRA-A products t = xin A^T (if r > 0).
+cudaError_t launch_prep(const void *x, int M, int d, const void *lora_a, int r, int prenorm, void *xhat,
+                        float *t, cudaStream_t stream, bool pdl);
+
+// Launches the quantizer / packer (two kernels).
+cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint32_t *codes, uint16_t *meta,
+                        int *nonfinite, cudaStream_t stream);
+
+// Reads and clears the device status word of the current device.
+cudaError_t read_device_status(int *status);
+
+}  // namespace wq

@@ -1,0 +1,114 @@
+// wq_pack.cu -- Stage-1 group-wise quantizer and packer (sm_103a).
+//
+// Sec. 4.1 quantizes gate/up to INT2 and (Sec. 3.3, Sec. 6 step 4) every
+// other linear layer to INT4.  The quantizer is asymmetric min-max
+// round-to-nearest per group of `group` consecutive input features of a row,
+// computed in IEEE fp32 with explicit round-to-nearest intrinsics so that the
+// codes, scales and zeros are reproducible bit for bit:
+//   s = fp16((max - min) / qmax) (1.0 if zero), z = clamp(rint(-min/s), 0, qmax),
+//   q = clamp(rint(w/s) + z, 0, qmax).
+// Two kernels: one warp per (row, group) computes s and z into the packed
+// meta layout; then one thread per packed 32-bit word gathers its 16 (2-bit)
+// or 8 (4-bit) codes.  Offline work: not on the decode path.
+#include <cuda_fp16.h>
+
+#include "wq_internal.h"
+
+namespace wq {
+namespace {
+
+__global__ void quant_meta_kernel(const float *__restrict__ w, int n, int k, int group, int bits, int RT, int NG,
+                                  uint16_t *__restrict__ meta, int *nonfinite) {
+  const long long gw = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (gw >= (long long)RT * 16 * NG) return;  // warp-uniform
+  const int row = (int)(gw / NG), j = (int)(gw % NG);
+  const int ngk = k / group;
+  unsigned short s16 = 0, z16 = 0;
+  if (row < n && j < ngk) {
+    const float *src = w + (size_t)row * k + (size_t)j * group;
+    float mn = INFINITY, mx = -INFINITY;
+    bool bad = false;
+    for (int i = lane; i < group; i += 32) {
+      const float v = src[i];
+      bad |= !isfinite(v);
+      mn = fminf(mn, v);
+      mx = fmaxf(mx, v);
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    const float qmax = (float)((1 << bits) - 1);
+    __half sh = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), qmax));
+    if (__half2float(sh) == 0.f) sh = __float2half_rn(1.f);
+    const float sf = __half2float(sh);
+    const float zf = __fadd_rn(fminf(fmaxf(rintf(__fdiv_rn(-mn, sf)), 0.f), qmax), 0.f);
+    s16 = __half_as_ushort(sh);
+    z16 = __half_as_ushort(__float2half_rn(zf));
+    if (bad && lane == 0 && nonfinite) atomicOr(nonfinite, 1);
+  }
+  if (lane == 0) {
+    const int rt = row >> 4, i = row & 15;
+    const size_t base = ((size_t)rt * NG + j) * 32 + 4 * (i & 7) + (i >> 3);
+    meta[base] = s16;
+    meta[base + 2] = z16;
+  }
+}
+
+__global__ void pack_codes_kernel(const float *__restrict__ w, int n, int k, int group, int bits, int RT, int KB,
+                                  int NG, const uint16_t *__restrict__ meta, uint32_t *__restrict__ codes) {
+  const int WPB = bits == 2 ? 128 : 256;
+  const size_t wid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (wid >= (size_t)RT * KB * WPB) return;
+  const size_t blk = wid / WPB;
+  const int wl = (int)(wid % WPB);
+  const int rt = (int)(blk / KB), kb = (int)(blk % KB);
+  const int tile = bits == 2 ? 0 : wl >> 7;  // 64-feature half of a 4-bit block
+  const int wl2 = wl & 127;
+  const int lane = wl2 >> 2, wi = wl2 & 3;
+  const float qmax = (float)((1 << bits) - 1);
+  uint32_t word = 0;
+  for (int bit = 0; bit < 32; bit += bits) {
+    const int half = bit >> 4, rowhalf = (bit >> 3) & 1;
+    int c;
+    if (bits == 2) {
+      const int cls = (bit & 7) >> 1;  // 2 * (16-feature step parity) + (upper 8 features)
+      c = wi * 32 + (cls >> 1) * 16 + (cls & 1) * 8 + (lane & 3) * 2 + half;
+    } else {
+      const int hi = (bit & 7) >> 2;
+      c = tile * 64 + wi * 16 + hi * 8 + (lane & 3) * 2 + half;
+    }
+    const int i = (lane >> 2) + 8 * rowhalf;
+    const int row = rt * 16 + i, col = kb * 128 + c;
+    if (row < n && col < k) {
+      const size_t mb = ((size_t)rt * NG + col / group) * 32 + 4 * (i & 7) + (i >> 3);
+      const float sf = __half2float(__ushort_as_half(meta[mb]));
+      const float zf = __half2float(__ushort_as_half(meta[mb + 2]));
+      const float qf = fminf(fmaxf(__fadd_rn(rintf(__fdiv_rn(w[(size_t)row * k + col], sf)), zf), 0.f), qmax);
+      word |= (uint32_t)qf << bit;
+    }
+  }
+  codes[wid] = word;
+}
+
+}  // namespace
+
+cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint32_t *codes, uint16_t *meta,
+                        int *nonfinite, cudaStream_t stream) {
+  const int RT = (n + 15) / 16, KB = (k + 127) / 128, NG = KB * 128 / group;
+  const long long warps = (long long)RT * 16 * NG;
+  const int tpb = 256;
+  quant_meta_kernel<<<(unsigned)((warps * 32 + tpb - 1) / tpb), tpb, 0, stream>>>(w, n, k, group, bits, RT, NG, meta,
+                                                                                 nonfinite);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const long long words = (long long)RT * KB * (bits == 2 ? 128 : 256);
+  pack_codes_kernel<<<(unsigned)((words + tpb - 1) / tpb), tpb, 0, stream>>>(w, n, k, group, bits, RT, KB, NG, meta,
+                                                                             codes);
+  return cudaGetLastError();
+}
+
+}  // namespace wq

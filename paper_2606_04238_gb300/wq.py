@@ -1,0 +1,263 @@
+"""Python binding of libwq.so (include/wq.h): argument marshalling only.
+
+Every function here converts torch tensors to device pointers and sizes,
+calls the C ABI of the same name on the current CUDA stream, and raises
+``WQError`` on a non-zero status.  All arithmetic runs in the CUDA kernels;
+there is no fallback: if the library is missing or no GPU is present the
+calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+from . import _build
+
+WQ_PRENORM = 1
+WQ_BF16 = 0
+WQ_F32 = 1
+
+_STATUS = {0: "WQ_OK", -1: "WQ_ERR_ARG", -2: "WQ_ERR_SHAPE", -3: "WQ_ERR_ALIGN", -4: "WQ_ERR_UNSUPPORTED",
+           -5: "WQ_ERR_CUDA", -6: "WQ_ERR_TIMEOUT", -7: "WQ_ERR_WORKSPACE"}
+
+
+class WQError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class _QWeight(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("meta", ctypes.c_void_p), ("n", ctypes.c_int32),
+                ("k", ctypes.c_int32), ("group", ctypes.c_int32), ("bits", ctypes.c_int32)]
+
+
+class _MLPLayer(ctypes.Structure):
+    _fields_ = [("gate", _QWeight), ("up", _QWeight), ("down", _QWeight), ("lora_a", ctypes.c_void_p),
+                ("lora_b_gate", ctypes.c_void_p), ("lora_b_up", ctypes.c_void_p), ("r", ctypes.c_int32),
+                ("lora_scale", ctypes.c_float)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def lib():
+    """The loaded libwq.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        path = _build.LIB_PATH
+        if not os.path.exists(path):
+            raise RuntimeError(f"libwq.so not found at {path}: run __graft_entry__.build() first")
+        L = ctypes.CDLL(path)
+        P, I, S, F, U = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float, ctypes.c_uint
+        QP = ctypes.POINTER(_QWeight)
+        sig = {
+            "wq_packed_sizes": (I, [I, I, I, I, ctypes.POINTER(S), ctypes.POINTER(S)]),
+            "wq_pack": (I, [P, I, I, I, I, QP, P, P]),
+            "wq_pack_w2": (I, [P, I, I, I, QP, P, P]),
+            "wq_pack_w4": (I, [P, I, I, I, QP, P, P]),
+            "wq_workspace_bytes": (S, [I, I, I, I]),
+            "wq_workspace_init": (I, [P, S, P]),
+            "wq_gateup_w2_lora": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P, S, P]),
+            "wq_gateup_w4": (I, [P, I, QP, QP, U, P, P, S, P]),
+            "wq_down_w4": (I, [P, I, QP, P, P, I, P, S, P]),
+            "wq_mlp_forward": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, S, P]),
+            "wq_plan_info": (I, [I, I, I, I, I, I, ctypes.POINTER(ctypes.c_int64)]),
+            "wq_last_error": (ctypes.c_char_p, []),
+            "wq_device_status": (I, [ctypes.POINTER(I)]),
+            "wq_version": (ctypes.c_char_p, []),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(status: int):
+    if status != 0:
+        raise WQError(status, lib().wq_last_error().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream():
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+@dataclass
+class QWeight:
+    """A packed group-quantized matrix [n, k] held in two device tensors."""
+    codes: torch.Tensor   # int32 words
+    meta: torch.Tensor    # int16 (binary16 bit patterns)
+    n: int
+    k: int
+    group: int
+    bits: int
+
+    def c(self) -> _QWeight:
+        return _QWeight(self.codes.data_ptr(), self.meta.data_ptr(), self.n, self.k, self.group, self.bits)
+
+    @property
+    def nbytes(self) -> int:
+        return self.codes.numel() * 4 + self.meta.numel() * 2
+
+
+def packed_sizes(bits: int, n: int, k: int, group: int):
+    cb, mb = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(lib().wq_packed_sizes(bits, n, k, group, ctypes.byref(cb), ctypes.byref(mb)))
+    return cb.value, mb.value
+
+
+def empty_qweight(n: int, k: int, group: int, bits: int, device="cuda") -> QWeight:
+    cb, mb = packed_sizes(bits, n, k, group)
+    return QWeight(torch.empty(cb // 4, dtype=torch.int32, device=device),
+                   torch.empty(mb // 2, dtype=torch.int16, device=device), n, k, group, bits)
+
+
+def pack(w: torch.Tensor, group: int, bits: int, nonfinite: torch.Tensor | None = None,
+         out: QWeight | None = None) -> QWeight:
+    """Quantize and pack an fp32 [n, k] device matrix (wq_pack)."""
+    assert w.dtype == torch.float32 and w.is_cuda and w.is_contiguous()
+    n, k = w.shape
+    q = out if out is not None else empty_qweight(n, k, group, bits, device=w.device)
+    cq = q.c()
+    _check(lib().wq_pack(_ptr(w), n, k, group, bits, ctypes.byref(cq), _ptr(nonfinite), _stream()))
+    return q
+
+
+def pack_w2(w, group, nonfinite=None):
+    return pack(w, group, 2, nonfinite)
+
+
+def pack_w4(w, group, nonfinite=None):
+    return pack(w, group, 4, nonfinite)
+
+
+def workspace_bytes(m: int, d: int, inter: int, r: int = 0) -> int:
+    return int(lib().wq_workspace_bytes(m, d, inter, r))
+
+
+def workspace(m: int, d: int, inter: int, r: int = 0, device="cuda") -> torch.Tensor:
+    """A zero-initialised workspace tensor for up to m tokens of a (d, inter) layer."""
+    nb = workspace_bytes(m, d, inter, r)
+    if nb == 0:
+        raise WQError(-2, f"no workspace size for m={m}, d={d}, inter={inter}")
+    ws = torch.empty(nb, dtype=torch.uint8, device=device)
+    _check(lib().wq_workspace_init(_ptr(ws), nb, _stream()))
+    return ws
+
+
+def gateup_w2_lora(x, gate: QWeight, up: QWeight, lora_a=None, lora_b_gate=None, lora_b_up=None,
+                   lora_scale: float = 0.0, prenorm: bool = False, h=None, ws=None):
+    m, d = x.shape
+    r = 0 if lora_b_gate is None else lora_b_gate.shape[1]
+    if h is None:
+        h = torch.empty((m, gate.n), dtype=torch.bfloat16, device=x.device)
+    if ws is None:
+        ws = workspace(max(m, 1), d, gate.n, r, device=x.device)
+    cg, cu = gate.c(), up.c()
+    _check(lib().wq_gateup_w2_lora(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), _ptr(lora_a), _ptr(lora_b_gate),
+                                   _ptr(lora_b_up), r, float(lora_scale), WQ_PRENORM if prenorm else 0, _ptr(h),
+                                   _ptr(ws), ws.numel(), _stream()))
+    return h
+
+
+def gateup_w4(x, gate: QWeight, up: QWeight, prenorm: bool = False, h=None, ws=None):
+    m, d = x.shape
+    if h is None:
+        h = torch.empty((m, gate.n), dtype=torch.bfloat16, device=x.device)
+    if ws is None:
+        ws = workspace(max(m, 1), d, gate.n, 0, device=x.device)
+    cg, cu = gate.c(), up.c()
+    _check(lib().wq_gateup_w4(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), WQ_PRENORM if prenorm else 0, _ptr(h),
+                              _ptr(ws), ws.numel(), _stream()))
+    return h
+
+
+def down_w4(h, down: QWeight, residual=None, out_f32: bool = False, y=None, ws=None):
+    m, inter = h.shape
+    if y is None:
+        y = torch.empty((m, down.n), dtype=torch.float32 if out_f32 else torch.bfloat16, device=h.device)
+    if ws is None:
+        ws = workspace(max(m, 1), down.n, inter, 0, device=h.device)
+    cd = down.c()
+    _check(lib().wq_down_w4(_ptr(h), m, ctypes.byref(cd), _ptr(residual), _ptr(y), WQ_F32 if out_f32 else WQ_BF16,
+                            _ptr(ws), ws.numel(), _stream()))
+    return y
+
+
+@dataclass
+class MLPLayer:
+    gate: QWeight
+    up: QWeight
+    down: QWeight
+    lora_a: torch.Tensor | None = None
+    lora_b_gate: torch.Tensor | None = None
+    lora_b_up: torch.Tensor | None = None
+    lora_scale: float = 0.0
+
+    @property
+    def r(self) -> int:
+        return 0 if self.lora_b_gate is None else self.lora_b_gate.shape[1]
+
+    def c(self) -> _MLPLayer:
+        return _MLPLayer(self.gate.c(), self.up.c(), self.down.c(),
+                         None if self.lora_a is None else self.lora_a.data_ptr(),
+                         None if self.lora_b_gate is None else self.lora_b_gate.data_ptr(),
+                         None if self.lora_b_up is None else self.lora_b_up.data_ptr(),
+                         self.r, float(self.lora_scale))
+
+
+class LayerTable:
+    """The C array of wq_mlp_layer for a stack (kept alive for graph replays)."""
+
+    def __init__(self, layers):
+        self.layers = list(layers)
+        self.array = (_MLPLayer * max(1, len(self.layers)))(*[l.c() for l in self.layers])
+
+
+def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTable | None = None):
+    """Stack of gated-MLP layers (wq_mlp_forward) on the current stream."""
+    m, d = x.shape
+    if table is None:
+        table = LayerTable(layers)
+    if y is None:
+        y = torch.empty_like(x)
+    if ws is None:
+        l0 = table.layers[0]
+        ws = workspace(max(m, 1), d, l0.gate.n, l0.r, device=x.device)
+    _check(lib().wq_mlp_forward(_ptr(x), m, table.array, len(table.layers), WQ_PRENORM if prenorm else 0, _ptr(y),
+                                _ptr(ws), ws.numel(), _stream()))
+    return y
+
+
+PLAN_FIELDS = ("row_tiles", "kblocks", "rb", "kp", "wk", "panels", "ctas", "threads", "smem", "tok_chunk")
+KIND_GATEUP_W2, KIND_GATEUP_W4, KIND_DOWN_W4 = 0, 1, 2
+
+
+def plan_info(kind: int, n: int, k: int, m: int, group: int, r: int = 0) -> dict:
+    """The launch decomposition the library would use on the current device."""
+    arr = (ctypes.c_int64 * 10)()
+    _check(lib().wq_plan_info(kind, n, k, m, group, r, arr))
+    return dict(zip(PLAN_FIELDS, list(arr)))
+
+
+def device_status() -> int:
+    v = ctypes.c_int(0)
+    _check(lib().wq_device_status(ctypes.byref(v)))
+    return v.value
+
+
+def version() -> str:
+    return lib().wq_version().decode()
