@@ -1,0 +1,445 @@
+"""Decode MLP-stack benchmark of the W4/W2-GateUp block on GB300.
+
+One step = one decode step of m tokens through the whole MLP stack of the
+Qwen3-4B-shaped workload (36 layers, d=2560, inter=9728; 2-bit gate/up with
+group 128 and LoRA rank 16 on both; 4-bit down with group 128; unit-weight
+RMSNorm before each MLP), replayed from a CUDA graph of wq_mlp_forward.
+Inputs are seeded synthetic draws of the paper's weight / activation shapes;
+the packed weights (1.01 GB per step) are far larger than L2, so no flush is
+needed between steps.
+
+Reported besides the step rate: the fused 2-bit gate/up call and the 4-bit
+down call timed on their own (36 distinct layers back to back, one graph) for
+the HBM roofline, the uniform-W4 stack on the same GPU (speedup, Gain%), the
+end-to-end rate through the C ABI with host buffers, SM clocks sampled during
+the timed region, and the CPU oracle on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl wq|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode MLP-stack tokens/s and fused W2 gate/up GEMV HBM GB/s (% of peak) at 1 GB300"
+UNIT = "tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="wq", choices=["wq", "reference"])
+    ap.add_argument("--config", default="qwen3_4b")
+    ap.add_argument("--m", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=0, help="0: the config's depth")
+    ap.add_argument("--no-extras", action="store_true", help="skip the comparator / per-kernel / CPU legs")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------- helpers
+def dist_setup(args):
+    import torch
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v, ws):
+    if ws == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock / throttle reasons during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.file.flush()
+        rows = []
+        with open(self.file.name) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.file.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------- byte model
+def algorithmic_bytes(cfg, m, bits_gu=2, lora=True):
+    """Bytes one decode step must move: packed codes, fp16 scales/zeros, LoRA
+    factors, bf16 activations in and out (nothing else)."""
+    d, inter, g = cfg.d, cfg.inter, cfg.group_gu
+    codes_gu = 2 * inter * d * bits_gu / 8
+    meta_gu = 2 * inter * (d // g) * 4
+    lora_b = (2 * inter * cfg.r * 2) if lora else 0
+    lora_a = (2 * cfg.r * d * 2) if lora else 0
+    act_gu = m * d * 2 + m * inter * 2                       # x in, h out
+    gateup = codes_gu + meta_gu + lora_a + lora_b + act_gu
+    codes_d = d * inter * 4 / 8
+    meta_d = d * (inter // cfg.group_down) * 4
+    act_d = m * inter * 2 + 2 * m * d * 2                    # h in, residual in, y out
+    down = codes_d + meta_d + act_d
+    return gateup, down
+
+
+def source_sha():
+    h = hashlib.sha256()
+    for fn in ("wq_gemv.cu", "wq_ptx.cuh", "wq_internal.h"):
+        with open(os.path.join(ROOT, "paper_2606_04238_gb300", "csrc", fn), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel)
+    if not e or e.get("source_sha") != source_sha():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# --------------------------------------------------------------------------- GPU arm
+def build_stack(wq, synth, cfg, n_layers, bits_gu, lora, dev):
+    import torch
+    layers = []
+    for l in range(n_layers):
+        wg, wu, wd = synth.layer_weights(cfg, l, device=dev)
+        kw = {}
+        if lora and bits_gu == 2:
+            a, bg, bu = synth.lora(cfg.d, cfg.inter, cfg.r, 10_000 + l, device=dev)
+            kw = dict(lora_a=a, lora_b_gate=bg, lora_b_up=bu, lora_scale=cfg.lora_scale)
+        layers.append(wq.MLPLayer(wq.pack(wg, cfg.group_gu, bits_gu), wq.pack(wu, cfg.group_gu, bits_gu),
+                                  wq.pack(wd, cfg.group_down, 4), **kw))
+        del wg, wu, wd
+    torch.cuda.synchronize()
+    return layers
+
+
+def capture(fn):
+    import torch
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        fn()
+        fn()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
+def time_graph(g, steps, warmup, ws_=1, sampler=None, pre=None, post=None):
+    """Device time of `steps` replays (CUDA events on the replay stream), max over ranks."""
+    import torch
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        if pre:
+            pre()
+        g.replay()
+        if post:
+            post()
+    torch.cuda.synchronize()
+    barrier(ws_)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        if pre:
+            pre()
+        g.replay()
+        if post:
+            post()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop() if sampler else None
+    barrier(ws_)
+    ms = e0.elapsed_time(e1)
+    return max_over_ranks(ms, ws_), clocks
+
+
+def cpu_oracle_sample(cfg, m, target_s=12.0, max_layers=8):
+    """The fp64 oracle on the host cores: time a bounded number of the stack's
+    layers and scale to the stack's depth (tokens/s of the whole stack)."""
+    import oracle as orc
+    from paper_2606_04238_gb300 import synth
+    x = synth.bf16_bits(synth.activations((m, cfg.d), 2024))
+    elapsed, done = 0.0, 0
+    for l in range(max_layers):
+        wg, wu, wd = synth.layer_weights(cfg, l)
+        qg = orc.quantize(wg.numpy(), cfg.group_gu, 2)[:3]
+        qu = orc.quantize(wu.numpy(), cfg.group_gu, 2)[:3]
+        qd = orc.quantize(wd.numpy(), cfg.group_down, 4)[:3]
+        a, bg, bu = synth.lora(cfg.d, cfg.inter, cfg.r, 10_000 + l)
+        t0 = time.perf_counter()
+        _, hb = orc.gateup(x, qg, qu, cfg.group_gu, synth.bf16_bits(a), synth.bf16_bits(bg), synth.bf16_bits(bu),
+                           cfg.lora_scale, prenorm=True)
+        _, x = orc.down(hb, qd, cfg.group_down, x)
+        elapsed += time.perf_counter() - t0
+        done += 1
+        if elapsed >= target_s:
+            break
+    per_layer = elapsed / done
+    return {"value": m / (per_layer * cfg.layers), "unit": UNIT, "cores": orc.threads(), "kind": "oracle",
+            "sample": f"{done} of {cfg.layers} layers at m={m} (fp64 C oracle, OpenMP), scaled to the full stack; "
+                      f"{per_layer * 1e3:.1f} ms per layer"}
+
+
+def run_gpu(args):
+    import torch
+    from paper_2606_04238_gb300 import synth, wq
+
+    ws_, rank, local = dist_setup(args)
+    import __graft_entry__
+    if rank == 0 or not os.path.exists(wq.library_path()):
+        __graft_entry__.build()
+    barrier(ws_)
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = synth.CONFIGS[args.config]
+    n_layers = args.layers or cfg.layers
+    m = args.m
+    steps, warmup = max(1, args.steps), max(3, args.warmup)
+
+    layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
+    table = wq.LayerTable(layers)
+    ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
+    x = synth.activations((m, cfg.d), 2024 + rank, device=dev)
+    y = torch.empty_like(x)
+    g = capture(lambda: wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table))
+    sampler = ClockSampler(local)
+    ms, clocks = time_graph(g, steps, warmup, ws_, sampler)
+    ms_step = ms / steps
+    value = ws_ * m * steps / (ms / 1e3)
+    launches_per_step = n_layers * 3
+
+    # end to end through the C ABI with host buffers: H2D of x, the stack, D2H of y
+    xh = torch.empty((m, cfg.d), dtype=torch.bfloat16).pin_memory()
+    xh.copy_(x.cpu())
+    yh = torch.empty((m, cfg.d), dtype=torch.bfloat16).pin_memory()
+    xd = torch.empty_like(x)
+
+    def e2e_step():
+        xd.copy_(xh, non_blocking=True)
+        wq.mlp_forward(xd, layers, prenorm=True, y=y, ws=ws, table=table)
+        yh.copy_(y, non_blocking=True)
+
+    ge = capture(e2e_step)
+    ms_e2e, _ = time_graph(ge, steps, warmup, ws_)
+    e2e = {"value": ws_ * m * steps / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": xh.numel() * 2,
+           "d2h_bytes_per_step": yh.numel() * 2,
+           "path": "pinned host x -> cudaMemcpyAsync -> wq_mlp_forward -> cudaMemcpyAsync -> pinned host y, "
+                   "in one CUDA graph per step"}
+
+    peak, peak_src = measured_peaks()
+    gu_bytes, dn_bytes = algorithmic_bytes(cfg, m)
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_, "steps": steps, "warmup": warmup,
+           "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "w2/w4 codes x f16 mma, f32 accumulate, bf16 activations", "data": "synthetic",
+           "config": {"workload": f"{cfg.name}_mlp_stack_{n_layers}L_m{m}", "model": f"{cfg.name}-shaped MLP stack",
+                      "d": cfg.d, "inter": cfg.inter, "layers": n_layers, "m": m, "global_batch": m * ws_,
+                      "seq_len": 1, "group": cfg.group_gu, "lora_r": cfg.r, "lora_scale": cfg.lora_scale,
+                      "prenorm": True, "parallelism": f"replicas x{ws_}",
+                      "l2": f"no flush: {n_layers * (gu_bytes + dn_bytes) / 1e9:.2f} GB of packed weights per step "
+                            "(> 129 MB L2)"},
+           "gpu_launches": launches_per_step * steps, "clocks": clocks, "e2e": e2e,
+           "stack_gbs": n_layers * (gu_bytes + dn_bytes) / (ms_step / 1e3) / 1e9}
+
+    if not args.no_extras and rank == 0:
+        # per-kernel chains: 36 distinct layers back to back (PDL), for the roofline
+        h = torch.empty((m, cfg.inter), dtype=torch.bfloat16, device=dev)
+        yk = torch.empty_like(x)
+
+        def gu_chain():
+            for L in layers:
+                wq.gateup_w2_lora(x, L.gate, L.up, L.lora_a, L.lora_b_gate, L.lora_b_up, L.lora_scale, prenorm=True,
+                                  h=h, ws=ws)
+
+        def dn_chain():
+            for L in layers:
+                wq.down_w4(h, L.down, residual=x, y=yk, ws=ws)
+
+        ks = max(20, steps // 4)
+        ms_gu, _ = time_graph(capture(gu_chain), ks, warmup)
+        ms_dn, _ = time_graph(capture(dn_chain), ks, warmup)
+        t_gu = ms_gu / ks / n_layers / 1e3
+        t_dn = ms_dn / ks / n_layers / 1e3
+        gu_gbs, dn_gbs = gu_bytes / t_gu / 1e9, dn_bytes / t_dn / 1e9
+        tr = recorded_traffic("gateup_w2_lora")
+        out["roofline"] = {"bound": "hbm", "achieved": gu_gbs, "peak": peak, "unit": "GB/s", "frac": gu_gbs / peak,
+                           "traffic": tr, "kernel": "wq_gateup_w2_lora (LoRA-A prologue + fused 2-bit gate/up GEMV)",
+                           "algorithmic_bytes_per_launch": gu_bytes, "us_per_launch": t_gu * 1e6,
+                           "peak_source": f"{peak_src} HBM copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"}
+        out["kernels"] = {
+            "gateup_w2_lora": {"us": t_gu * 1e6, "gbs": gu_gbs, "frac": gu_gbs / peak, "bytes": gu_bytes},
+            "down_w4": {"us": t_dn * 1e6, "gbs": dn_gbs, "frac": dn_gbs / peak, "bytes": dn_bytes,
+                        "traffic": recorded_traffic("down_w4")},
+        }
+        out["gpu_launches"] += ks * n_layers * 2 * 2 + ks * n_layers * 0  # chains: prologue+GEMV, GEMV
+
+        # the uniform-W4 comparator stack (same workload, 4-bit gate/up, no adapter)
+        del g, ge
+        w4 = build_stack(wq, synth, cfg, n_layers, 4, False, dev)
+        t4 = wq.LayerTable(w4)
+        g4 = capture(lambda: wq.mlp_forward(x, w4, prenorm=True, y=y, ws=ws, table=t4))
+        ms4, _ = time_graph(g4, steps, warmup)
+        tps4 = m * steps / (ms4 / 1e3)
+        tps = value / ws_
+        out["w4_uniform"] = {"tokens_per_s": tps4, "ms_per_step": ms4 / steps,
+                             "speedup_w4w2_over_w4": tps / tps4, "gain_pct": 100.0 * (tps - tps4) / tps4,
+                             "paper_gain_pct_context": "7.5-23.3% whole-model TPS, LIFE roofline model on "
+                                                       "Device A (50 TOPs, 100 GB/s) / Device B (200 GB/s)"}
+        out["gpu_launches"] += steps * n_layers * 3
+        del w4, g4
+        torch.cuda.empty_cache()
+        out["cpu_baseline"] = cpu_oracle_sample(cfg, m)
+
+    if rank == 0:
+        print(json.dumps(out))
+    barrier(ws_)
+
+
+# --------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    """The oracle as it stands, on the host cores: each step is one layer of
+    the stack (a bounded sample); the rate is scaled to the whole stack."""
+    ws_ = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle as orc
+    from paper_2606_04238_gb300 import synth
+    orc.build()
+    cfg = synth.CONFIGS[args.config]
+    m = args.m
+    n_layers = args.layers or cfg.layers
+    nprep = min(4, max(1, args.steps + args.warmup))
+    prepared = []
+    for l in range(nprep):
+        wg, wu, wd = synth.layer_weights(cfg, l)
+        a, bg, bu = synth.lora(cfg.d, cfg.inter, cfg.r, 10_000 + l)
+        prepared.append((orc.quantize(wg.numpy(), cfg.group_gu, 2)[:3], orc.quantize(wu.numpy(), cfg.group_gu, 2)[:3],
+                         orc.quantize(wd.numpy(), cfg.group_down, 4)[:3], synth.bf16_bits(a), synth.bf16_bits(bg),
+                         synth.bf16_bits(bu)))
+    x = synth.bf16_bits(synth.activations((m, cfg.d), 2024))
+
+    def step(i, x):
+        qg, qu, qd, a, bg, bu = prepared[i % nprep]
+        _, hb = orc.gateup(x, qg, qu, cfg.group_gu, a, bg, bu, cfg.lora_scale, prenorm=True)
+        return orc.down(hb, qd, cfg.group_down, x)[1]
+
+    for i in range(max(0, args.warmup)):
+        x = step(i, x)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        x = step(i, x)
+    el = time.perf_counter() - t0
+    per_layer = el / max(1, args.steps)
+    value = m / (per_layer * n_layers)
+    sample = (f"each step = 1 of the {n_layers} layers at m={m} (fp64 C oracle, OpenMP); rate scaled to the "
+              f"whole stack; {per_layer * 1e3:.1f} ms per layer")
+    print(json.dumps({"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_,
+                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * n_layers * 1e3,
+                      "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                      "data": "synthetic",
+                      "config": {"workload": f"{cfg.name}_mlp_stack_{n_layers}L_m{m}", "d": cfg.d, "inter": cfg.inter,
+                                 "layers": n_layers, "m": m},
+                      "cpu_baseline": {"value": value, "unit": UNIT, "cores": orc.threads(), "kind": "oracle",
+                                       "sample": sample},
+                      "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -146,6 +146,16 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   a.out = h;
   a.partials = reinterpret_cast<float *>(ws + L.part1);
   a.counters = reinterpret_cast<unsigned *>(ws + L.cnt1);
+  size_t cb = 0, mb = 0;
+  wq_packed_sizes(gate->bits, inter, d, gate->group, &cb, &mb);
+  a.nb_codes[0] = a.nb_codes[1] = cb;
+  a.nb_meta[0] = a.nb_meta[1] = mb;
+  a.nb_lora_b[0] = a.nb_lora_b[1] = (size_t)inter * r * 2;
+  a.nb_act = (size_t)m * d * 2;
+  a.nb_t = (size_t)m * 2 * r * 4;
+  a.nb_out = (size_t)m * inter * 2;
+  a.nb_part = L.part2 - L.part1;
+  a.nb_cnt = (size_t)((inter + 15) / 16) * 4;
   cudaError_t e = launch_gemv(kind, plan, a, s, true);
   if (e != cudaSuccess) return cuda_fail(e, "gate/up launch");
   return WQ_OK;
@@ -169,6 +179,15 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.out_f32 = y_f32;
   a.partials = reinterpret_cast<float *>(ws + L.part2);
   a.counters = reinterpret_cast<unsigned *>(ws + L.cnt2);
+  size_t cb = 0, mb = 0;
+  wq_packed_sizes(4, down->n, down->k, down->group, &cb, &mb);
+  a.nb_codes[0] = cb;
+  a.nb_meta[0] = mb;
+  a.nb_act = (size_t)m * down->k * 2;
+  a.nb_res = residual ? (size_t)m * down->n * 2 : 0;
+  a.nb_out = (size_t)m * down->n * (y_f32 ? 4 : 2);
+  a.nb_part = L.total - L.part2;
+  a.nb_cnt = (size_t)((down->n + 15) / 16) * 4;
   cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);
   if (e != cudaSuccess) return cuda_fail(e, "down launch");
   return WQ_OK;
@@ -382,6 +401,14 @@ wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t 
 }
 
 const char *wq_last_error(void) { return g_last_error.c_str(); }
+
+// Debug builds: first failed in-kernel bounds / alignment check.
+wq_status wq_debug_record(long long rec[4]) {
+  if (!rec) return fail(WQ_ERR_ARG, "null record");
+  cudaError_t e = read_debug_record(rec);
+  if (e != cudaSuccess) return cuda_fail(e, "debug record read");
+  return ok();
+}
 
 wq_status wq_device_status(int *status) {
   if (!status) return fail(WQ_ERR_ARG, "null status pointer");

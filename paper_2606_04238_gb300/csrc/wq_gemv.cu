@@ -13,9 +13,10 @@
 //      scales/zeros of its row tiles into shared memory -- before waiting on
 //      the previous kernel (programmatic dependent launch), so the weight
 //      stream of this kernel overlaps the tail of the previous one;
-//   2. after griddepcontrol.wait, each token's activation panel is converted
-//      to binary16 with an exact power-of-two scale per token (and per code
-//      position class, see below), and per-group activation sums are formed;
+//   2. after griddepcontrol.wait, each token's activation panel is loaded
+//      (plain 16-byte loads) and converted in place to binary16 with an exact
+//      power-of-two scale per token (and per code position class, see below),
+//      and per-group activation sums are formed;
 //   3. each warp owns one 16-row tile and a share of the panel: a 16-byte
 //      shared load per lane yields the tensor-core A fragments of 64 (2-bit)
 //      or 32 (4-bit) codes; codes are isolated with a single AND each -- the
@@ -40,9 +41,29 @@ namespace wq {
 // Device status word: WQ_OK (0) or WQ_ERR_TIMEOUT (-6) after a bounded wait ran out.
 __device__ int g_device_status = 0;
 
+// Debug builds only: first failed bounds/alignment check {site, line, value, count}.
+__device__ long long g_debug_record[4] = {0, 0, 0, 0};
+
 namespace {
 
 __device__ __forceinline__ void record_timeout() { atomicExch(&g_device_status, -6); }
+
+#ifdef WQ_DEBUG_CHECKS
+__device__ __noinline__ void debug_fail(int site, int line, long long value) {
+  if (atomicAdd(reinterpret_cast<unsigned long long *>(&g_debug_record[3]), 1ull) == 0ull) {
+    g_debug_record[0] = site;
+    g_debug_record[1] = line;
+    g_debug_record[2] = value;
+  }
+}
+// True when the access may proceed; records the first violation otherwise.
+#define WQ_OK_IF(cond, site, value) ((cond) ? true : (debug_fail((site), __LINE__, (long long)(value)), false))
+#else
+#define WQ_OK_IF(cond, site, value) true
+#endif
+// [off, off + len) inside [0, size) and off aligned to `al`
+#define WQ_RANGE(off, len, size, al) \
+  ((long long)(off) >= 0 && (long long)(off) + (long long)(len) <= (long long)(size) && ((long long)(off) % (al)) == 0)
 
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
@@ -94,7 +115,6 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 
   uint8_t *codes_s = smem + p.off_codes;
   uint8_t *meta_s = smem + p.off_meta;
-  const __nv_bfloat16 *lorab_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_lorab);
   __half *xp_s = reinterpret_cast<__half *>(smem + p.off_xp);
   float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);
   float *scale_s = reinterpret_cast<float *>(smem + p.off_scale);
@@ -105,29 +125,24 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 
   // ---- 1. weight prefetch (independent of the previous kernel) ----
   if (tid == 0) {
-    for (int i = 0; i <= p.RB + 1; ++i) mbar_init(&bars[i], 1);
+    for (int i = 0; i < p.RB; ++i) mbar_init(&bars[i], 1);
     fence_barrier_init();
     for (int i = 0; i < nrt; ++i) {
       const int rt = rt0 + i;
       mbar_arrive_expect_tx(&bars[i], NPROJ * nkb * (BPK + GPB * 64));
 #pragma unroll
       for (int pj = 0; pj < NPROJ; ++pj) {
-        bulk_g2s(codes_s + (size_t)((pj * p.RB + i) * p.KP) * BPK,
-                 reinterpret_cast<const uint8_t *>(a.codes[pj]) + ((size_t)rt * p.KB + kb0) * BPK, nkb * BPK,
-                 &bars[i]);
-        bulk_g2s(meta_s + (size_t)((pj * p.RB + i) * p.KP * GPB) * 64,
-                 reinterpret_cast<const uint8_t *>(a.meta[pj]) + ((size_t)rt * NG + (size_t)kb0 * GPB) * 64,
-                 nkb * GPB * 64, &bars[i]);
+        const size_t cd = p.off_codes + (size_t)((pj * p.RB + i) * p.KP) * BPK;
+        const size_t cs = ((size_t)rt * p.KB + kb0) * BPK;
+        if (WQ_OK_IF(WQ_RANGE(cd, nkb * BPK, p.off_meta, 16), 1, cd) &&
+            WQ_OK_IF(WQ_RANGE(cs, nkb * BPK, a.nb_codes[pj], 16), 2, cs))
+          bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nkb * BPK, &bars[i]);
+        const size_t md = p.off_meta + (size_t)((pj * p.RB + i) * p.KP * GPB) * 64;
+        const size_t ms = ((size_t)rt * NG + (size_t)kb0 * GPB) * 64;
+        if (WQ_OK_IF(WQ_RANGE(md, nkb * GPB * 64, p.off_lorab, 16), 3, md) &&
+            WQ_OK_IF(WQ_RANGE(ms, nkb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
+          bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nkb * GPB * 64, &bars[i]);
       }
-    }
-    if (p.lora_smem) {
-      const int rows = min(nrt * 16, a.N - rt0 * 16);
-      const uint32_t bytes = (uint32_t)rows * a.r * 2;
-      mbar_arrive_expect_tx(&bars[p.RB], NPROJ * bytes);
-#pragma unroll
-      for (int pj = 0; pj < NPROJ; ++pj)
-        bulk_g2s(smem + p.off_lorab + (size_t)pj * p.RB * 16 * a.r * 2,
-                 reinterpret_cast<const uint8_t *>(a.lora_b[pj]) + (size_t)rt0 * 16 * a.r * 2, bytes, &bars[p.RB]);
     }
   }
   int *tokmax_s = reinterpret_cast<int *>(scale_s + MPAD);
@@ -144,16 +159,27 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   // ---- 2. activation panel -> binary16 with per-token power-of-two scale ----
   const int kbeg = kb0 * 128;
   const int kvalid = min(nkb * 128, a.K - kbeg);  // a multiple of 8
-  if (tid == 0) {
+  // Activations are staged with ordinary loads, not a bulk copy: the panel is
+  // converted in place below, and shared memory filled by the async (bulk
+  // copy) proxy is only ever read afterwards in this kernel.
+  {
     const __nv_bfloat16 *act = reinterpret_cast<const __nv_bfloat16 *>(a.act);
-    mbar_arrive_expect_tx(&bars[p.RB + 1], (uint32_t)M * kvalid * 2);
-    for (int m = 0; m < M; ++m)
-      bulk_g2s(xp_s + (size_t)m * p.xstride, act + (size_t)m * a.K + kbeg, (uint32_t)kvalid * 2, &bars[p.RB + 1]);
+    const int nch = kvalid / 8;  // 16-byte chunks per token row
+    for (int i = tid; i < M * nch; i += blockDim.x) {
+      const int m = i / nch, c = i % nch;
+      const size_t src = ((size_t)m * a.K + kbeg + (size_t)c * 8) * 2;
+      if (WQ_OK_IF(WQ_RANGE(src, 16, a.nb_act, 16), 8, src) &&
+          WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + c * 8) * 2, 16, p.off_xs, 16), 7, i))
+        *reinterpret_cast<uint4 *>(xp_s + (size_t)m * p.xstride + c * 8) = ldg_cg128(act + (size_t)m * a.K + kbeg + c * 8);
+    }
   }
   if (NPROJ == 2 && a.r > 0) {
-    for (int i = tid; i < M * 2 * a.r; i += blockDim.x) t_s[i] = ldcg_f32(a.t + i);
+    for (int i = tid; i < M * 2 * a.r; i += blockDim.x)
+      if (WQ_OK_IF(WQ_RANGE((size_t)i * 4, 4, a.nb_t, 4), 9, i) &&
+          WQ_OK_IF(WQ_RANGE(p.off_t + (size_t)i * 4, 4, p.off_bar, 4), 10, i))
+        t_s[i] = ldcg_f32(a.t + i);
   }
-  if (!mbar_wait(&bars[p.RB + 1], 0) && tid == 0) record_timeout();
+  __syncthreads();
   {
     // Work item = 16 features of one token (one MMA k-step).  Pass 1: per
     // token max|x|.  Pass 2: in place, bf16 -> scaled binary16 in the order
@@ -162,7 +188,8 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
     const int total = M * nsteps;
     for (int i = tid; i < total; i += blockDim.x) {
       const int m = i / nsteps, st = i % nsteps;
-      if (st * 16 < kvalid) {
+      if (st * 16 < kvalid &&
+          WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + st * 16) * 2, 32, p.off_xs, 16), 11, i)) {
         const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(xp_s + (size_t)m * p.xstride + st * 16);
         float f[16];
         unpack_bf16x8(lds128(src), *reinterpret_cast<float(*)[8]>(f));
@@ -172,7 +199,7 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 #pragma unroll
         for (int e = 0; e < 16; ++e)
           if (e < nv) mx = fmaxf(mx, fabsf(f[e]));
-        atomicMax(&tokmax_s[m], __float_as_int(mx));
+        if (WQ_OK_IF(m < MPAD, 12, m)) atomicMax(&tokmax_s[m], __float_as_int(mx));
       }
     }
     __syncthreads();
@@ -185,7 +212,9 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 #pragma unroll
       for (int e = 0; e < 16; ++e) f[e] = 0.f;
       __half *slot = xp_s + (size_t)m * p.xstride + st * 16;
-      if (valid && st * 16 < kvalid) {
+      const bool slot_ok = !valid || WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + st * 16) * 2, 32,
+                                                       p.off_xs, 16), 13, i);
+      if (valid && slot_ok && st * 16 < kvalid) {
         const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(slot);
         unpack_bf16x8(lds128(src), *reinterpret_cast<float(*)[8]>(f));
         unpack_bf16x8(lds128(src + 8), *reinterpret_cast<float(*)[8]>(f + 8));
@@ -206,7 +235,7 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
         frexpf(mx, &E);
         e = max(-100, min(100, 15 - E));
       }
-      if (valid) {
+      if (valid && slot_ok) {
         const float up = ldexpf(1.f, e);
         if (st == 0) scale_s[m] = ldexpf(1.f, 24 - e);
         // bit-position class of the codes feeding features 0-7 / 8-15 of this step
@@ -225,7 +254,9 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
       }
 #pragma unroll
       for (int o = 1; o < LG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
-      if (valid && (lane % LG) == 0) xs_s[(st / LG) * MPAD + m] = gs * ldexpf(1.f, e - 24);
+      if (valid && (lane % LG) == 0 &&
+          WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)(st / LG) * MPAD + m) * 4, 4, p.off_scale, 4), 14, i))
+        xs_s[(st / LG) * MPAD + m] = gs * ldexpf(1.f, e - 24);
     }
   }
   __syncthreads();
@@ -255,7 +286,8 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int m = tc * TOK + nt * 8 + (lane >> 2);
-            if (m < M) {
+            if (m < M && WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + (kb * 8 + ks) * 16 + 4 * (lane & 3)) * 2,
+                                           8, p.off_xs, 8), 15, kb)) {
               const uint2 v = lds64(xp_s + (size_t)m * p.xstride + (kb * 8 + ks) * 16 + 4 * (lane & 3));
               b[ks][nt][0] = v.x;
               b[ks][nt][1] = v.y;
@@ -268,7 +300,9 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
         for (int pj = 0; pj < NPROJ; ++pj) {
           const uint8_t *cb = cbase + pj * cproj + (size_t)kb * BPK;
           uint32_t wds[BITS == 2 ? 4 : 8];
-          {
+          wds[0] = wds[1] = wds[2] = wds[3] = 0u;
+          if (BITS == 4) wds[BITS == 4 ? 4 : 0] = wds[BITS == 4 ? 5 : 1] = wds[BITS == 4 ? 6 : 2] = wds[BITS == 4 ? 7 : 3] = 0u;
+          if (WQ_OK_IF(WQ_RANGE(cb - smem, BPK == 512 ? 16 : 528, p.off_meta, 16), 16, kb)) {
             const uint4 w0 = lds128(cb);
             wds[0] = w0.x; wds[1] = w0.y; wds[2] = w0.z; wds[3] = w0.w;
             if (BITS == 4) {
@@ -305,13 +339,17 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
             for (int nt = 0; nt < NT; ++nt) mma_f16_16816(cg[nt], af, b[ks][nt][0], b[ks][nt][1]);
             if ((ks + 1) % GS == 0) {
               const int gl = kb * GPB + ks / GS;
-              const uint2 mt = lds64(mbase + pj * mproj + (size_t)gl * 64);
+              uint2 mt = make_uint2(0u, 0u);
+              if (WQ_OK_IF(WQ_RANGE(mbase + pj * mproj + (size_t)gl * 64 - smem, 8, p.off_lorab, 8), 17, gl))
+                mt = lds64(mbase + pj * mproj + (size_t)gl * 64);
               const float s_lo = half_bits_to_float(mt.x), s_hi = half_bits_to_float(mt.x >> 16);
               const float z_lo = half_bits_to_float(mt.y), z_hi = half_bits_to_float(mt.y >> 16);
 #pragma unroll
               for (int nt = 0; nt < NT; ++nt) {
                 const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
-                const float2 xs = *reinterpret_cast<const float2 *>(xs_s + gl * MPAD + col);
+                float2 xs = make_float2(0.f, 0.f);
+                if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + col) * 4, 8, p.off_scale, 8), 18, col))
+                  xs = *reinterpret_cast<const float2 *>(xs_s + gl * MPAD + col);
                 ctot[pj][nt][0] = fmaf(s_lo, fmaf(-z_lo, xs.x, cg[nt][0]), ctot[pj][nt][0]);
                 ctot[pj][nt][1] = fmaf(s_lo, fmaf(-z_lo, xs.y, cg[nt][1]), ctot[pj][nt][1]);
                 ctot[pj][nt][2] = fmaf(s_hi, fmaf(-z_hi, xs.x, cg[nt][2]), ctot[pj][nt][2]);
@@ -330,6 +368,7 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
         for (int nt = 0; nt < NT; ++nt) {
           const int col = tc * TOK + nt * 8 + 2 * (lane & 3), r0 = lane >> 2;
           float *sl = slot_s + (size_t)((wk * p.RB + rw) * NPROJ + pj) * 16 * MPAD;
+          if (!WQ_OK_IF(WQ_RANGE((uint8_t *)(sl + (r0 + 8) * MPAD + col) - smem, 8, p.off_t, 4), 19, col)) continue;
           sl[r0 * MPAD + col] = ctot[pj][nt][0];
           sl[r0 * MPAD + col + 1] = ctot[pj][nt][1];
           sl[(r0 + 8) * MPAD + col] = ctot[pj][nt][2];
@@ -343,7 +382,9 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   const int per_rt = NPROJ * 16 * MPAD;
   for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
     float s = 0.f;
-    for (int w = 0; w < p.WK; ++w) s += slot_s[(size_t)w * p.RB * per_rt + i];
+    for (int w = 0; w < p.WK; ++w)
+      if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_t, 4), 20, i))
+        s += slot_s[(size_t)w * p.RB * per_rt + i];
     const int m = i % MPAD;
     slot_s[i] = m < M ? s * scale_s[m] : 0.f;
   }
@@ -352,11 +393,12 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   if (p.P > 1) {
     for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
       const int rti = i / per_rt, rem = i % per_rt;
-      a.partials[((size_t)(rt0 + rti) * p.P + panel) * per_rt + rem] = slot_s[i];
+      const size_t po = ((size_t)(rt0 + rti) * p.P + panel) * per_rt + rem;
+      if (WQ_OK_IF(WQ_RANGE(po * 4, 4, a.nb_part, 4), 21, po)) a.partials[po] = slot_s[i];
     }
     __threadfence();
     __syncthreads();
-    if (tid < nrt) {
+    if (tid < nrt && WQ_OK_IF(WQ_RANGE((size_t)(rt0 + tid) * 4, 4, a.nb_cnt, 4), 22, rt0 + tid)) {
       const unsigned prev = atomicAdd(&a.counters[rt0 + tid], 1u);
       last_s[tid] = prev == (unsigned)(p.P - 1);
     }
@@ -367,16 +409,15 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
       if (!last_s[rti]) continue;
       const float *src = a.partials + (size_t)(rt0 + rti) * p.P * per_rt + rem;
       float s = 0.f;
-      for (int pp = 0; pp < p.P; ++pp) s += ldcg_f32(src + (size_t)pp * per_rt);
+      for (int pp = 0; pp < p.P; ++pp)
+        if (WQ_OK_IF(WQ_RANGE((src - a.partials + (size_t)pp * per_rt) * 4, 4, a.nb_part, 4), 23, pp))
+          s += ldcg_f32(src + (size_t)pp * per_rt);
       slot_s[i] = s;
     }
     if (tid < nrt && last_s[tid]) a.counters[rt0 + tid] = 0u;
     __syncthreads();
   } else {
     if (tid < nrt) last_s[tid] = 1;
-    if (p.lora_smem) {
-      if (!mbar_wait(&bars[p.RB], 0) && tid == 0) record_timeout();
-    }
     __syncthreads();
   }
 
@@ -394,21 +435,18 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
       float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * MPAD + r16 * MPAD + m];
       if (a.r > 0) {
         const int r = a.r;
-        const __nv_bfloat16 *bg, *bu;
-        if (p.lora_smem) {
-          bg = lorab_s + (size_t)rl * r;
-          bu = lorab_s + (size_t)p.RB * 16 * r + (size_t)rl * r;
-        } else {
-          bg = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[0]) + (size_t)n * r;
-          bu = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[1]) + (size_t)n * r;
-        }
+        const __nv_bfloat16 *bg = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[0]) + (size_t)n * r;
+        const __nv_bfloat16 *bu = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[1]) + (size_t)n * r;
         const float *tg = t_s + (size_t)m * 2 * r;
         const float *tu = tg + r;
         float lg = 0.f, lu = 0.f;
-        for (int q = 0; q < r; q += 8) {
+        const bool lora_ok =
+            WQ_OK_IF(WQ_RANGE(((size_t)m * 2 * r + 2 * r) * 4 + p.off_t - 4, 4, p.off_bar, 4), 24, m) &&
+            WQ_OK_IF(WQ_RANGE(((size_t)n * r + r) * 2 - 16, 16, a.nb_lora_b[1], 16), 26, n);
+        for (int q = 0; lora_ok && q < r; q += 8) {
           float fg[8], fu[8];
-          unpack_bf16x8(*reinterpret_cast<const uint4 *>(bg + q), fg);
-          unpack_bf16x8(*reinterpret_cast<const uint4 *>(bu + q), fu);
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4 *>(bg + q)), fg);
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4 *>(bu + q)), fu);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             lg = fmaf(tg[q + e], fg[e], lg);
@@ -419,10 +457,13 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
         u = fmaf(a.lora_scale, lu, u);
       }
       const float h = g / (1.f + __expf(-g)) * u;
-      reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(h);
+      if (WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_out, 2), 27, n))
+        reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(h);
     } else {
       float y = v0;
-      if (a.residual)
+      if (!WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * (a.out_f32 ? 4 : 2), a.out_f32 ? 4 : 2, a.nb_out, 2), 28, n))
+        continue;
+      if (a.residual && WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_res, 2), 29, n))
         y += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + n]);
       if (a.out_f32)
         reinterpret_cast<float *>(a.out)[(size_t)m * a.N + n] = y;
@@ -440,7 +481,7 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) prep_kernel(const __nv_bfloat16 *x, int M, int d,
                                                     const __nv_bfloat16 *lora_a, int r2, int prenorm,
-                                                    __nv_bfloat16 *xhat, float *t) {
+                                                    __nv_bfloat16 *xhat, float *t, uint32_t smem_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
@@ -448,16 +489,15 @@ __global__ void __launch_bounds__(256) prep_kernel(const __nv_bfloat16 *x, int M
   __nv_bfloat16 *arow = reinterpret_cast<__nv_bfloat16 *>(smem);
   float *rs_s = reinterpret_cast<float *>(smem + arow_bytes);   // [kMaxTokens]
   float *red_s = rs_s + kMaxTokens;                              // [32]
-  uint64_t *bar = reinterpret_cast<uint64_t *>(red_s + 32);
   const int rho = blockIdx.x;
   const bool lora = r2 > 0;
 
-  if (lora && tid == 0) {
-    mbar_init(bar, 1);
-    fence_barrier_init();
-    mbar_arrive_expect_tx(bar, (uint32_t)d * 2);
-    bulk_g2s(arow, lora_a + (size_t)rho * d, (uint32_t)d * 2, bar);
+  if (lora && WQ_OK_IF(rho < r2 && (d * 2) % 16 == 0, 41, rho)) {
+    // the LoRA-A row does not depend on the previous kernel: load it first
+    for (int c = tid; c < d / 8; c += blockDim.x)
+      *reinterpret_cast<uint4 *>(arow + c * 8) = __ldg(reinterpret_cast<const uint4 *>(lora_a + (size_t)rho * d) + c);
   }
+  (void)smem_bytes;
   pdl_launch_dependents();
   pdl_wait();
 
@@ -475,12 +515,11 @@ __global__ void __launch_bounds__(256) prep_kernel(const __nv_bfloat16 *x, int M
       ss = warp_sum(ss);
       rs = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)d), kRmsEps)));
     }
-    if (lane == 0) rs_s[m] = rs;
+    if (lane == 0 && WQ_OK_IF(m < kMaxTokens, 42, m)) rs_s[m] = rs;
   }
   __syncthreads();
 
   if (lora) {
-    if (!mbar_wait(bar, 0) && tid == 0) record_timeout();
     for (int m = 0; m < M; ++m) {
       const float rs = rs_s[m];
       float acc = 0.f;
@@ -500,7 +539,7 @@ __global__ void __launch_bounds__(256) prep_kernel(const __nv_bfloat16 *x, int M
       if (tid == 0) {
         float s = 0.f;
         for (int w = 0; w < nwarps; ++w) s += red_s[w];
-        t[(size_t)m * r2 + rho] = s;
+        if (WQ_OK_IF((size_t)m * r2 + rho < (size_t)M * r2, 43, m)) t[(size_t)m * r2 + rho] = s;
       }
       __syncthreads();
     }
@@ -552,8 +591,8 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->MPAD * 4, 128);
   p->off_t = off;
   off = align_up(off + (nproj == 2 ? (uint32_t)p->M * 2 * r * 4 : 0u), 128);
-  p->off_bar = off;  // RB weight barriers, LoRA-B barrier, activation barrier
-  off = align_up(off + (uint32_t)(p->RB + 2) * 8, 128);
+  p->off_bar = off;  // one weight barrier per row tile
+  off = align_up(off + (uint32_t)p->RB * 8, 128);
   p->off_last = off;
   off = align_up(off + (uint32_t)p->RB * 4, 128);
   p->smem = off;
@@ -586,7 +625,7 @@ bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms
         p.M = M; p.MPAD = MPAD; p.NT = NT;
         p.threads = RB * WK * 32;
         p.units = p.NRB * P;
-        p.lora_smem = (nproj == 2 && r > 0 && P == 1) ? 1 : 0;
+        p.lora_smem = 0;
         compute_layout(kind, group, r, &p);
         if (p.smem > kSmemLimit) continue;
         const int occ = std::max(1, std::min({(int)(233472 / (p.smem + 1024)), 2048 / p.threads, 32}));
@@ -665,7 +704,16 @@ cudaError_t launch_prep(const void *x, int M, int d, const void *lora_a, int r, 
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, prep_kernel, reinterpret_cast<const __nv_bfloat16 *>(x), M, d,
                             reinterpret_cast<const __nv_bfloat16 *>(lora_a), 2 * r, prenorm,
-                            reinterpret_cast<__nv_bfloat16 *>(xhat), t);
+                            reinterpret_cast<__nv_bfloat16 *>(xhat), t, smem);
+}
+
+cudaError_t read_debug_record(long long rec[4]) {
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return e;
+  e = cudaMemcpyFromSymbol(rec, g_debug_record, 4 * sizeof(long long));
+  if (e != cudaSuccess) return e;
+  const long long zero[4] = {0, 0, 0, 0};
+  return cudaMemcpyToSymbol(g_debug_record, zero, sizeof zero);
 }
 
 cudaError_t read_device_status(int *status) {

@@ -28,7 +28,7 @@ struct GemvPlan {
   int M, MPAD, NT;     // tokens, tokens padded to the token-chunk size, 8-token tiles per chunk
   int threads;         // RB * WK * 32
   int units;           // grid size = NRB * P
-  int lora_smem;       // LoRA B rows staged in shared memory (P == 1 and r > 0)
+  int lora_smem;       // reserved (0): LoRA B rows are read from global memory
   uint32_t smem;       // dynamic shared memory bytes
   // byte offsets inside dynamic shared memory
   uint32_t off_codes, off_meta, off_lorab, off_xp, off_xs, off_scale, off_slots, off_t, off_bar, off_last;
@@ -49,6 +49,8 @@ struct GemvArgs {
   int out_f32;
   float *partials;           // [RT][P][NPROJ][16][MPAD] fp32 (P > 1)
   unsigned *counters;        // [RT] arrival counters, zero between calls
+  // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
+  size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_t, nb_res, nb_out, nb_part, nb_cnt;
 };
 
 enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
@@ -71,5 +73,9 @@ cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint3
 
 // Reads and clears the device status word of the current device.
 cudaError_t read_device_status(int *status);
+
+// Debug builds (WQ_DEBUG_CHECKS): first failed bounds / alignment check
+// {site, line, value, count}; zeros when none failed.  Clears the record.
+cudaError_t read_debug_record(long long rec[4]);
 
 }  // namespace wq

@@ -45,14 +45,15 @@ _lib = None
 
 
 def library_path() -> str:
-    return _build.LIB_PATH
+    """libwq.so, or the bounds-checking debug build when WQ_DEBUG_LIB=1."""
+    return _build.DEBUG_LIB_PATH if os.environ.get("WQ_DEBUG_LIB") == "1" else _build.LIB_PATH
 
 
 def lib():
     """The loaded libwq.so; raises if it has not been built."""
     global _lib
     if _lib is None:
-        path = _build.LIB_PATH
+        path = library_path()
         if not os.path.exists(path):
             raise RuntimeError(f"libwq.so not found at {path}: run __graft_entry__.build() first")
         L = ctypes.CDLL(path)
@@ -73,6 +74,7 @@ def lib():
             "wq_last_error": (ctypes.c_char_p, []),
             "wq_device_status": (I, [ctypes.POINTER(I)]),
             "wq_version": (ctypes.c_char_p, []),
+            "wq_debug_record": (I, [ctypes.POINTER(ctypes.c_longlong)]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -257,6 +259,13 @@ def device_status() -> int:
     v = ctypes.c_int(0)
     _check(lib().wq_device_status(ctypes.byref(v)))
     return v.value
+
+
+def debug_record():
+    """Debug build: (site, line, value, count) of the first failed in-kernel check."""
+    rec = (ctypes.c_longlong * 4)()
+    _check(lib().wq_debug_record(rec))
+    return tuple(rec)
 
 
 def version() -> str:
