@@ -149,6 +149,37 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
                             int r, float lora_scale, unsigned flags, void *h,
                             void *ws, size_t ws_bytes, void *stream);
 
+/*
+ * wq_gateup_w2_lora without a workspace argument, for callers that cannot
+ * allocate device memory: code that runs where cudaMalloc is not allowed or
+ * not wanted (inside a host callback, between the launches of an engine whose
+ * memory is fully planned ahead, under an allocator that owns every device
+ * buffer), or a plugin that must not grow its host process's memory.  The
+ * paper has no counterpart to this call; it is a deployment convenience.
+ *
+ * Same arguments and results as wq_gateup_w2_lora minus ws / ws_bytes.  The
+ * scratch it needs (LoRA-A products, normalized input, split-K partial sums
+ * and arrival counters) lives in a fixed array of WQ_NOALLOC_SCRATCH_BYTES
+ * bytes inside the library, which every GPU that loads the library keeps
+ * until the process exits.  A call whose layer needs more scratch than that
+ * returns WQ_ERR_UNSUPPORTED and launches nothing.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, which may load the library's device code); make
+ *     that first call before any stream capture.
+ *   - Every call clears the array's arrival counters (cudaMemsetAsync on
+ *     `stream`) and then reuses the array, which keeps the previous call's
+ *     contents otherwise.  All calls share the one array: calls that can
+ *     overlap on the GPU (different streams, or different host threads
+ *     without ordering) race with each other and must be serialized by the
+ *     caller.
+ * The call allocates nothing: no cudaMalloc, cudaFree or allocating library
+ * routine.
+ */
+#define WQ_NOALLOC_SCRATCH_BYTES (4u << 20)
+wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                                    const void *lora_a, const void *lora_b_gate, const void *lora_b_up,
+                                    int r, float lora_scale, unsigned flags, void *h, void *stream);
+
 /* The uniform-W4 comparator: the same block with 4-bit gate/up and no LoRA. */
 wq_status wq_gateup_w4(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
                        unsigned flags, void *h, void *ws, size_t ws_bytes, void *stream);

@@ -6,6 +6,7 @@
 #include <cstdio>
 #include <cstring>
 #include <algorithm>
+#include <mutex>
 #include <string>
 
 #include "wq.h"
@@ -308,6 +309,64 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
                             void *h, void *ws, size_t ws_bytes, void *stream) {
   return gateup_entry(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, ws, ws_bytes,
                       stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Scratch of wq_gateup_w2_lora_noalloc: a fixed array in the library's device
+// code, so the call never allocates.  Its device address is looked up once per
+// device (host code only sees a stand-in for the symbol, not the address).
+static __device__ __align__(256) uint8_t g_noalloc_scratch[WQ_NOALLOC_SCRATCH_BYTES];
+std::mutex g_noalloc_mu;
+void *g_noalloc_base[64] = {};
+
+wq_status noalloc_scratch(void **base) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(WQ_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_base[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the built-in scratch");
+    g_noalloc_base[dev] = p;
+  }
+  *base = g_noalloc_base[dev];
+  return WQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                                    const void *lora_a, const void *lora_b_gate, const void *lora_b_up, int r,
+                                    float lora_scale, unsigned flags, void *h, void *stream) {
+  wq_status st = check_tokens(m);
+  if (st != WQ_OK) return st;
+  if ((st = check_gateup_pair(gate, up, 2)) != WQ_OK) return st;
+  if ((st = check_lora(lora_a, lora_b_gate, lora_b_up, r)) != WQ_OK) return st;
+  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (m == 0) return ok();
+  if (!x || !h) return fail(WQ_ERR_ARG, "null x or h");
+  if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
+  WsLayout L;
+  if (!ws_layout(m, gate->k, gate->n, &L)) return fail(WQ_ERR_CUDA, "cannot query the current device");
+  if (L.total > (size_t)WQ_NOALLOC_SCRATCH_BYTES)
+    return fail(WQ_ERR_UNSUPPORTED, "this layer needs %zu bytes of scratch; the built-in scratch holds %u (use wq_gateup_w2_lora)",
+                L.total, (unsigned)WQ_NOALLOC_SCRATCH_BYTES);
+  void *base = nullptr;
+  if ((st = noalloc_scratch(&base)) != WQ_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the arrival counters must start at zero
+  cudaError_t e = cudaMemsetAsync(static_cast<uint8_t *>(base) + L.cnt1, 0, L.t - L.cnt1, s);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the built-in scratch counters");
+  st = run_gateup(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, L,
+                  static_cast<uint8_t *>(base), s);
+  return st == WQ_OK ? ok() : st;
 }
 
 wq_status wq_gateup_w4(const void *x, int m, const wq_qweight *gate, const wq_qweight *up, unsigned flags, void *h,

@@ -67,6 +67,7 @@ def lib():
             "wq_workspace_bytes": (S, [I, I, I, I]),
             "wq_workspace_init": (I, [P, S, P]),
             "wq_gateup_w2_lora": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P, S, P]),
+            "wq_gateup_w2_lora_noalloc": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P]),
             "wq_gateup_w4": (I, [P, I, QP, QP, U, P, P, S, P]),
             "wq_down_w4": (I, [P, I, QP, P, P, I, P, S, P]),
             "wq_mlp_forward": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, S, P]),
@@ -172,6 +173,24 @@ def gateup_w2_lora(x, gate: QWeight, up: QWeight, lora_a=None, lora_b_gate=None,
     _check(lib().wq_gateup_w2_lora(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), _ptr(lora_a), _ptr(lora_b_gate),
                                    _ptr(lora_b_up), r, float(lora_scale), WQ_PRENORM if prenorm else 0, _ptr(h),
                                    _ptr(ws), ws.numel(), _stream()))
+    return h
+
+
+def gateup_w2_lora_noalloc(x, gate: QWeight, up: QWeight, lora_a=None, lora_b_gate=None, lora_b_up=None,
+                           lora_scale: float = 0.0, prenorm: bool = False, h=None):
+    """wq_gateup_w2_lora_noalloc: the same call with the library's built-in scratch.
+
+    For callers that cannot allocate device memory; ``h`` may be passed in so
+    that nothing is allocated on the Python side either.
+    """
+    m, d = x.shape
+    r = 0 if lora_b_gate is None else lora_b_gate.shape[1]
+    if h is None:
+        h = torch.empty((m, gate.n), dtype=torch.bfloat16, device=x.device)
+    cg, cu = gate.c(), up.c()
+    _check(lib().wq_gateup_w2_lora_noalloc(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), _ptr(lora_a),
+                                           _ptr(lora_b_gate), _ptr(lora_b_up), r, float(lora_scale),
+                                           WQ_PRENORM if prenorm else 0, _ptr(h), _stream()))
     return h
 
 
