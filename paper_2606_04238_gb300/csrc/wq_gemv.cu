@@ -124,25 +124,30 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   int *last_s = reinterpret_cast<int *>(smem + p.off_last);
 
   // ---- 1. weight prefetch (independent of the previous kernel) ----
-  if (tid == 0) {
-    for (int i = 0; i < p.RB; ++i) mbar_init(&bars[i], 1);
+  // Warp (rw, wk) owns row tile rw and blocks [kbs, kbe) of the panel; its
+  // lane 0 bulk-copies exactly that slice (both projections) on its own
+  // barrier, so each warp starts as soon as its own weights have landed.
+  const int rw = warp % p.RB, wk = warp / p.RB;
+  const int kbs = wk * nkb / p.WK, kbe = (wk + 1) * nkb / p.WK;
+  const bool has_slice = rw < nrt && kbe > kbs;
+  if (lane == 0 && has_slice) {
+    uint64_t *bar = &bars[warp];
+    mbar_init(bar, 1);
     fence_barrier_init();
-    for (int i = 0; i < nrt; ++i) {
-      const int rt = rt0 + i;
-      mbar_arrive_expect_tx(&bars[i], NPROJ * nkb * (BPK + GPB * 64));
+    const int rt = rt0 + rw, nb = kbe - kbs;
+    mbar_arrive_expect_tx(bar, NPROJ * nb * (BPK + GPB * 64));
 #pragma unroll
-      for (int pj = 0; pj < NPROJ; ++pj) {
-        const size_t cd = p.off_codes + (size_t)((pj * p.RB + i) * p.KP) * BPK;
-        const size_t cs = ((size_t)rt * p.KB + kb0) * BPK;
-        if (WQ_OK_IF(WQ_RANGE(cd, nkb * BPK, p.off_meta, 16), 1, cd) &&
-            WQ_OK_IF(WQ_RANGE(cs, nkb * BPK, a.nb_codes[pj], 16), 2, cs))
-          bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nkb * BPK, &bars[i]);
-        const size_t md = p.off_meta + (size_t)((pj * p.RB + i) * p.KP * GPB) * 64;
-        const size_t ms = ((size_t)rt * NG + (size_t)kb0 * GPB) * 64;
-        if (WQ_OK_IF(WQ_RANGE(md, nkb * GPB * 64, p.off_lorab, 16), 3, md) &&
-            WQ_OK_IF(WQ_RANGE(ms, nkb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
-          bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nkb * GPB * 64, &bars[i]);
-      }
+    for (int pj = 0; pj < NPROJ; ++pj) {
+      const size_t cd = p.off_codes + ((size_t)(pj * p.RB + rw) * p.KP + kbs) * BPK;
+      const size_t cs = ((size_t)rt * p.KB + kb0 + kbs) * BPK;
+      if (WQ_OK_IF(WQ_RANGE(cd, nb * BPK, p.off_meta, 16), 1, cd) &&
+          WQ_OK_IF(WQ_RANGE(cs, nb * BPK, a.nb_codes[pj], 16), 2, cs))
+        bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nb * BPK, bar);
+      const size_t md = p.off_meta + ((size_t)(pj * p.RB + rw) * p.KP * GPB + (size_t)kbs * GPB) * 64;
+      const size_t ms = ((size_t)rt * NG + (size_t)(kb0 + kbs) * GPB) * 64;
+      if (WQ_OK_IF(WQ_RANGE(md, nb * GPB * 64, p.off_lorab, 16), 3, md) &&
+          WQ_OK_IF(WQ_RANGE(ms, nb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
+        bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nb * GPB * 64, bar);
     }
   }
   int *tokmax_s = reinterpret_cast<int *>(scale_s + MPAD);
@@ -262,10 +267,8 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   __syncthreads();
 
   // ---- 3./4. tensor-core dot products ----
-  const int rw = warp % p.RB, wk = warp / p.RB;
   if (rw < nrt) {
-    const int kbs = wk * nkb / p.WK, kbe = (wk + 1) * nkb / p.WK;
-    const bool ok = mbar_wait(&bars[rw], 0);
+    const bool ok = !has_slice || mbar_wait(&bars[warp], 0);
     if (!ok && lane == 0) record_timeout();
     const uint8_t *cbase = codes_s + (size_t)(rw * p.KP) * BPK + lane * 16;
     const uint8_t *mbase = meta_s + (size_t)(rw * p.KP * GPB) * 64 + (lane >> 2) * 8;
@@ -311,11 +314,12 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
               wds[BITS == 4 ? 6 : 2] = w1.z; wds[BITS == 4 ? 7 : 3] = w1.w;
             }
           }
-          float cg[NT][4];
+          // two independent accumulator chains (even / odd k-steps) per group
+          float cg[NT][4], ch[NT][4];
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-            for (int q = 0; q < 4; ++q) cg[nt][q] = 0.f;
+            for (int q = 0; q < 4; ++q) cg[nt][q] = ch[nt][q] = 0.f;
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks) {
             uint32_t af[4];
@@ -336,7 +340,12 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
               af[3] = x8 & 0x00F000F0u;
             }
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) mma_f16_16816(cg[nt], af, b[ks][nt][0], b[ks][nt][1]);
+            for (int nt = 0; nt < NT; ++nt) {
+              if (ks & 1)
+                mma_f16_16816(ch[nt], af, b[ks][nt][0], b[ks][nt][1]);
+              else
+                mma_f16_16816(cg[nt], af, b[ks][nt][0], b[ks][nt][1]);
+            }
             if ((ks + 1) % GS == 0) {
               const int gl = kb * GPB + ks / GS;
               uint2 mt = make_uint2(0u, 0u);
@@ -350,12 +359,12 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
                 float2 xs = make_float2(0.f, 0.f);
                 if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + col) * 4, 8, p.off_scale, 8), 18, col))
                   xs = *reinterpret_cast<const float2 *>(xs_s + gl * MPAD + col);
-                ctot[pj][nt][0] = fmaf(s_lo, fmaf(-z_lo, xs.x, cg[nt][0]), ctot[pj][nt][0]);
-                ctot[pj][nt][1] = fmaf(s_lo, fmaf(-z_lo, xs.y, cg[nt][1]), ctot[pj][nt][1]);
-                ctot[pj][nt][2] = fmaf(s_hi, fmaf(-z_hi, xs.x, cg[nt][2]), ctot[pj][nt][2]);
-                ctot[pj][nt][3] = fmaf(s_hi, fmaf(-z_hi, xs.y, cg[nt][3]), ctot[pj][nt][3]);
+                ctot[pj][nt][0] = fmaf(s_lo, fmaf(-z_lo, xs.x, cg[nt][0] + ch[nt][0]), ctot[pj][nt][0]);
+                ctot[pj][nt][1] = fmaf(s_lo, fmaf(-z_lo, xs.y, cg[nt][1] + ch[nt][1]), ctot[pj][nt][1]);
+                ctot[pj][nt][2] = fmaf(s_hi, fmaf(-z_hi, xs.x, cg[nt][2] + ch[nt][2]), ctot[pj][nt][2]);
+                ctot[pj][nt][3] = fmaf(s_hi, fmaf(-z_hi, xs.y, cg[nt][3] + ch[nt][3]), ctot[pj][nt][3]);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) cg[nt][q] = 0.f;
+                for (int q = 0; q < 4; ++q) cg[nt][q] = ch[nt][q] = 0.f;
               }
             }
           }
@@ -591,8 +600,8 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->MPAD * 4, 128);
   p->off_t = off;
   off = align_up(off + (nproj == 2 ? (uint32_t)p->M * 2 * r * 4 : 0u), 128);
-  p->off_bar = off;  // one weight barrier per row tile
-  off = align_up(off + (uint32_t)p->RB * 8, 128);
+  p->off_bar = off;  // one weight barrier per warp
+  off = align_up(off + (uint32_t)p->RB * p->WK * 8, 128);
   p->off_last = off;
   off = align_up(off + (uint32_t)p->RB * 4, 128);
   p->smem = off;
@@ -631,12 +640,20 @@ bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms
         const int occ = std::max(1, std::min({(int)(233472 / (p.smem + 1024)), 2048 / p.threads, 32}));
         const int per_sm = (p.units + num_sms - 1) / num_sms;           // units landing on the busiest SM
         const int waves = (p.units + num_sms * occ - 1) / (num_sms * occ);
-        // throughput cost: tile-projections on the busiest SM (~26 cycles each
-        // at HBM speed); latency cost: the serial tile chain of one warp
+        // Cycle estimates: a tile-projection (16 rows x 128 features of one
+        // matrix) costs ~45 issue slots, spread over the SM's 4 schedulers;
+        // one warp's chain of tile-projections costs ~120 cycles each of MMA
+        // and shared-memory latency; each CTA wave adds a fixed prologue /
+        // epilogue latency, and a split-panel fixup an L2 round trip.
         const double tiles = (double)per_sm * RB * KP * nproj * chunks;
-        const double serial = (double)((KP + WK - 1) / WK) * nproj * chunks * waves;
-        double cost = std::max(26.0 * tiles, 60.0 * serial);
-        cost += 50.0 * per_sm + (P > 1 ? 300.0 : 0.0) + (p.smem > 113 * 1024 ? 200.0 : 0.0);
+        const double thr = tiles * 45.0 / 4.0;
+        const double lat = (double)((KP + WK - 1) / WK) * nproj * chunks * 120.0 * waves;
+        // the busiest SM's share of the weight stream at ~22 B/cycle (HBM / SMs)
+        const double mem = (double)per_sm * RB * KP * nproj * (kind_bits(kind) == 2 ? 640.0 : 1088.0) / 22.0;
+        // the weight stream (or the issue rate) bounds the bulk; the last
+        // warp's dependent chain after its slice lands is added as a tail
+        double cost = std::max(thr, mem) + lat + 800.0 * waves + (P > 1 ? 1500.0 : 0.0);
+        cost += (p.smem > 113 * 1024 ? 300.0 : 0.0);  // no room to overlap the next kernel's prologue
         if (cost < best) {
           best = cost;
           bp = p;
