@@ -12,7 +12,7 @@ What it computes (paper sections cited in ``wq_oracle.c``):
   * ``gateup``     g,u = x W^T + alpha (x A^T) B^T (Eq. 1) on the dequantized
                    gate/up weights, h = SiLU(g) * u (Sec. 3.3), fp64.
   * ``down``       y = residual + h Wd^T on the dequantized 4-bit down weights.
-  * ``prenorm``    unit-weight RMSNorm of the MLP input, rounded to bf16.
+  * ``rms_scale``  unit-weight RMSNorm scale 1/sqrt(mean(x^2)+eps) per token.
 """
 from __future__ import annotations
 
@@ -59,7 +59,7 @@ def _load():
                 "orc_tile_pack": (I, [P, P, P, I, I, I, I, P, P]),
                 "orc_tile_unpack": (I, [P, P, I, I, I, I, P, P, P]),
                 "orc_dequant": (I, [P, P, P, I, I, I, P]),
-                "orc_prenorm": (I, [P, I, I, D, P]),
+                "orc_rms_scale": (I, [P, I, I, D, P]),
                 "orc_gateup": (I, [P, I, I, I, P, P, P, P, P, P, I, P, P, P, I, D, I, D, P, P]),
                 "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
                 "orc_threads": (I, []),
@@ -171,11 +171,12 @@ def dequant(q, s, z, group: int) -> np.ndarray:
 
 
 # -------------------------------------------------------------------- forward
-def prenorm(x_bits, eps: float = RMS_EPS) -> np.ndarray:
+def rms_scale(x_bits, eps: float = RMS_EPS) -> np.ndarray:
+    """rs[t] = 1 / sqrt(mean(x[t]^2) + eps) in fp64; prenorm multiplies x by it, unrounded."""
     x = _c(x_bits, np.uint16)
     m, d = x.shape
-    out = np.empty_like(x)
-    _load().orc_prenorm(_p(x), m, d, eps, _p(out))
+    out = np.empty(m, np.float64)
+    _load().orc_rms_scale(_p(x), m, d, eps, _p(out))
     return out
 
 

@@ -22,8 +22,9 @@
  *     optionally preceded by a unit-weight RMSNorm of the MLP input.
  *
  * bf16 rounding happens only where the CUDA path stores a bf16 tensor: the
- * normalized input x_hat, the hidden activation h and the layer output y.
- * Between those points the arithmetic is fp64.
+ * hidden activation h and the layer output y.  The RMSNorm-normalized input
+ * is never stored, so it is used unrounded.  Between those points the
+ * arithmetic is fp64.
  */
 #include <math.h>
 #include <stdint.h>
@@ -284,8 +285,12 @@ int orc_dequant(const uint8_t *q, const uint16_t *s, const uint16_t *z,
 /* Forward pass.                                                       */
 /* ------------------------------------------------------------------ */
 
-/* Unit-weight RMSNorm of each token: x_hat = bf16( x / sqrt(mean(x^2) + eps) ). */
-int orc_prenorm(const uint16_t *x, int m, int d, double eps, uint16_t *xhat)
+/*
+ * Unit-weight RMSNorm scale of each token: rs[t] = 1 / sqrt(mean_c x[t,c]^2 + eps).
+ * The normalized input x[t,c] * rs[t] is used unrounded by orc_gateup (it is
+ * never stored, so it has no bf16 rounding point).
+ */
+int orc_rms_scale(const uint16_t *x, int m, int d, double eps, double *rs)
 {
     if (m < 0 || d <= 0) return ORC_ERR_ARG;
     for (int t = 0; t < m; ++t) {
@@ -294,14 +299,25 @@ int orc_prenorm(const uint16_t *x, int m, int d, double eps, uint16_t *xhat)
             double v = orc_bf16_to_f64(x[(size_t)t * d + c]);
             ss += v * v;
         }
-        double rs = 1.0 / sqrt(ss / d + eps);
-        for (int c = 0; c < d; ++c)
-            xhat[(size_t)t * d + c] = orc_f64_to_bf16(orc_bf16_to_f64(x[(size_t)t * d + c]) * rs);
+        rs[t] = 1.0 / sqrt(ss / d + eps);
     }
     return ORC_OK;
 }
 
 /* One quantized row dotted with one activation row: sum_k x[k] * s(q - z). */
+static double orc_qdot_f64(const uint8_t *qrow, const uint16_t *srow, const uint16_t *zrow,
+                           int k, int group, const double *xrow)
+{
+    double acc = 0.0;
+    for (int col = 0; col < k; ++col) {
+        const int j = col / group;
+        const double w = orc_f16_to_f64(srow[j]) * ((double)qrow[col] - orc_f16_to_f64(zrow[j]));
+        acc += xrow[col] * w;
+    }
+    return acc;
+}
+
+/* The same with a bf16 activation row. */
 static double orc_qdot(const uint8_t *qrow, const uint16_t *srow, const uint16_t *zrow,
                        int k, int group, const uint16_t *xrow)
 {
@@ -317,7 +333,7 @@ static double orc_qdot(const uint8_t *qrow, const uint16_t *srow, const uint16_t
 /*
  * Gate/up half of the gated MLP with unmerged LoRA on both projections
  * (Eq. 1 applied to gate and to up, then SiLU(gate) * up):
- *   xin      = prenorm ? RMSNorm(x) (bf16) : x
+ *   xin      = prenorm ? x * rs (RMSNorm, unrounded, rs of orc_rms_scale) : x
  *   t_g      = xin . A_g^T,  t_u = xin . A_u^T        (A = lora_a rows 0..r-1 / r..2r-1)
  *   g[m,n]   = sum_k xin[m,k] deq(Wg)[n,k] + lora_scale * sum_p t_g[m,p] B_g[n,p]
  *   u[m,n]   = likewise with Wu, A_u, B_u
@@ -335,24 +351,28 @@ int orc_gateup(const uint16_t *x, int m, int d, int inter,
 {
     if (m < 0 || d <= 0 || inter <= 0 || group <= 0 || d % group != 0 || r < 0) return ORC_ERR_ARG;
     const int ng = d / group;
-    uint16_t *xin = (uint16_t *)malloc(sizeof(uint16_t) * ((size_t)m * d + 1));
+    double *xin = (double *)malloc(sizeof(double) * ((size_t)m * d + 1));
+    double *rs = (double *)malloc(sizeof(double) * ((size_t)m + 1));
     double *t = (double *)malloc(sizeof(double) * ((size_t)m * 2 * r + 1));
-    if (!xin || !t) { free(xin); free(t); return ORC_ERR_ARG; }
-    if (prenorm) orc_prenorm(x, m, d, eps, xin);
-    else memcpy(xin, x, sizeof(uint16_t) * (size_t)m * d);
+    if (!xin || !rs || !t) { free(xin); free(rs); free(t); return ORC_ERR_ARG; }
+    for (int tk = 0; tk < m; ++tk) rs[tk] = 1.0;
+    if (prenorm) orc_rms_scale(x, m, d, eps, rs);
+    for (int tk = 0; tk < m; ++tk)
+        for (int c = 0; c < d; ++c)
+            xin[(size_t)tk * d + c] = orc_bf16_to_f64(x[(size_t)tk * d + c]) * rs[tk];
     for (int tk = 0; tk < m; ++tk)
         for (int p = 0; p < 2 * r; ++p) {
             double acc = 0.0;
             for (int c = 0; c < d; ++c)
-                acc += orc_bf16_to_f64(xin[(size_t)tk * d + c]) * orc_bf16_to_f64(lora_a[(size_t)p * d + c]);
+                acc += xin[(size_t)tk * d + c] * orc_bf16_to_f64(lora_a[(size_t)p * d + c]);
             t[(size_t)tk * 2 * r + p] = acc;
         }
 #pragma omp parallel for schedule(static)
     for (int n = 0; n < inter; ++n) {
         for (int tk = 0; tk < m; ++tk) {
-            const uint16_t *xr = xin + (size_t)tk * d;
-            double g = orc_qdot(qg + (size_t)n * d, sg + (size_t)n * ng, zg + (size_t)n * ng, d, group, xr);
-            double u = orc_qdot(qu + (size_t)n * d, su + (size_t)n * ng, zu + (size_t)n * ng, d, group, xr);
+            const double *xr = xin + (size_t)tk * d;
+            double g = orc_qdot_f64(qg + (size_t)n * d, sg + (size_t)n * ng, zg + (size_t)n * ng, d, group, xr);
+            double u = orc_qdot_f64(qu + (size_t)n * d, su + (size_t)n * ng, zu + (size_t)n * ng, d, group, xr);
             double lg = 0.0, lu = 0.0;
             for (int p = 0; p < r; ++p) {
                 lg += t[(size_t)tk * 2 * r + p] * orc_bf16_to_f64(lora_bg[(size_t)n * r + p]);
@@ -366,6 +386,7 @@ int orc_gateup(const uint16_t *x, int m, int d, int inter,
         }
     }
     free(xin);
+    free(rs);
     free(t);
     return ORC_OK;
 }

@@ -93,25 +93,51 @@ def test_lora_rank1_closed_form(orc):
     np.testing.assert_allclose(h[0], want, rtol=1e-12, atol=1e-14)
 
 
-def test_prenorm_matches_torch_rms_norm(orc):
+def test_rms_scale_matches_torch_rms_norm(orc):
     rng = np.random.default_rng(5)
     x = _rand_bf16(rng, (4, 512), 3.0)
-    got = _bf16_to_f64(orc.prenorm(x))
-    xt = torch.from_numpy(_bf16_to_f64(x))
-    want = torch.nn.functional.rms_norm(xt, (512,), eps=1e-6).numpy()
-    # the oracle rounds once to bf16: within half a bf16 ulp of the fp64 value
-    spacing = 2.0 ** (np.floor(np.log2(np.abs(want))) - 7)
-    assert np.all(np.abs(got - want) <= spacing * 0.5 * (1 + 1e-9))
+    rs = orc.rms_scale(x)
+    xf = _bf16_to_f64(x)
+    want = torch.nn.functional.rms_norm(torch.from_numpy(xf), (512,), eps=1e-6).numpy()
+    # the normalized input is used unrounded: x * rs equals torch's fp64 RMSNorm
+    np.testing.assert_allclose(xf * rs[:, None], want, rtol=1e-13, atol=0)
 
 
-def test_gateup_prenorm_equals_gateup_of_normalized(orc):
+def test_gateup_prenorm_is_scale_invariant(orc):
+    # with eps = 0, RMSNorm(2^k x) = RMSNorm(x) exactly (powers of two scale
+    # bf16 values, sums of squares and square roots without rounding), so the
+    # whole gate/up output must be bit-identical; a dropped or misplaced
+    # normalization breaks this
     rng = np.random.default_rng(6)
     d, inter = 256, 64
     g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    a = _rand_bf16(rng, (2, d), 0.1)
+    bg = _rand_bf16(rng, (inter, 1), 0.1)
+    bu = _rand_bf16(rng, (inter, 1), 0.1)
     x = _rand_bf16(rng, (2, d), 5.0)
-    h1, _ = orc.gateup(x, g, u, 64, prenorm=True)
-    h2, _ = orc.gateup(orc.prenorm(x), g, u, 64, prenorm=False)
+    x4 = torch.from_numpy(_bf16_to_f64(x) * 4.0).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    h1, _ = orc.gateup(x, g, u, 64, a, bg, bu, lora_scale=1.5, prenorm=True, eps=0.0)
+    h2, _ = orc.gateup(x4, g, u, 64, a, bg, bu, lora_scale=1.5, prenorm=True, eps=0.0)
     np.testing.assert_array_equal(h1, h2)
+    h0, _ = orc.gateup(x, g, u, 64, a, bg, bu, lora_scale=1.5, prenorm=False)
+    assert not np.allclose(h0, h1)
+
+
+def test_gateup_prenorm_matches_numpy(orc):
+    rng = np.random.default_rng(16)
+    d, inter = 256, 48
+    g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    a = _rand_bf16(rng, (2, d), 0.1)
+    bg = _rand_bf16(rng, (inter, 1), 0.1)
+    bu = _rand_bf16(rng, (inter, 1), 0.1)
+    x = _rand_bf16(rng, (3, d), 2.0)
+    h, _ = orc.gateup(x, g, u, 64, a, bg, bu, lora_scale=0.75, prenorm=True)
+    xf, af = _bf16_to_f64(x), _bf16_to_f64(a)
+    xn = xf / np.sqrt((xf * xf).mean(axis=1, keepdims=True) + 1e-6)
+    gg = xn @ _np_deq(*g, 64).T + 0.75 * (xn @ af[0])[:, None] * _bf16_to_f64(bg)[:, 0][None, :]
+    uu = xn @ _np_deq(*u, 64).T + 0.75 * (xn @ af[1])[:, None] * _bf16_to_f64(bu)[:, 0][None, :]
+    want = gg / (1 + np.exp(-gg)) * uu
+    np.testing.assert_allclose(h, want, rtol=1e-11, atol=1e-13)
 
 
 def test_down_with_residual_matches_numpy(orc):
