@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--m", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0, help="0: the config's depth")
     ap.add_argument("--no-extras", action="store_true", help="skip the comparator / per-kernel / CPU legs")
+    ap.add_argument("--eager", action="store_true",
+                    help="profiling aid: run the stack with plain stream launches (no CUDA graph), print no JSON")
     return ap.parse_args()
 
 
@@ -290,12 +292,20 @@ def run_gpu(args):
     ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
     x = synth.activations((m, cfg.d), 2024 + rank, device=dev)
     y = torch.empty_like(x)
+    if args.eager:
+        # for ncu: the same launches as one step, issued eagerly
+        for _ in range(warmup + steps):
+            wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table)
+        torch.cuda.synchronize()
+        assert wq.device_status() == 0
+        print(f"eager: {warmup + steps} stack steps of {n_layers} layers done", flush=True)
+        return
     g = capture(lambda: wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table))
     sampler = ClockSampler(local)
     ms, clocks = time_graph(g, steps, warmup, ws_, sampler)
     ms_step = ms / steps
     value = ws_ * m * steps / (ms / 1e3)
-    launches_per_step = n_layers * 3
+    launches_per_step = 2 * n_layers + 1  # first layer's input statistics, then gate/up and down per layer
 
     # end to end through the C ABI with host buffers: H2D of x, the stack, D2H of y
     xh = torch.empty((m, cfg.d), dtype=torch.bfloat16).pin_memory()

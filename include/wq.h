@@ -137,7 +137,8 @@ wq_status wq_workspace_init(void *ws, size_t ws_bytes, void *stream);
  * Fused 2-bit gate/up projection with unmerged LoRA and SiLU(gate) * up
  * (Eq. 1 on gate and up; gated MLP of Sec. 3.3; gate, activation and product
  * fused in one kernel as in the fused MLP modelling of Sec. 5):
- *     xin = (flags & WQ_PRENORM) ? bf16(RMSNorm(x)) : x
+ *     xin = (flags & WQ_PRENORM) ? x * rs : x,  rs = 1 / sqrt(mean(x^2) + 1e-6) per token
+ *           (the normalized input is never stored, so it is not rounded)
  *     g   = xin deq(Wg)^T + lora_scale * (xin A_g^T) B_g^T      (fp32 accumulate)
  *     u   = xin deq(Wu)^T + lora_scale * (xin A_u^T) B_u^T
  *     h   = bf16( g / (1 + exp(-g)) * u )
@@ -158,8 +159,8 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
  * paper has no counterpart to this call; it is a deployment convenience.
  *
  * Same arguments and results as wq_gateup_w2_lora minus ws / ws_bytes.  The
- * scratch it needs (LoRA-A products, normalized input, split-K partial sums
- * and arrival counters) lives in a fixed array of WQ_NOALLOC_SCRATCH_BYTES
+ * scratch it needs (per-16-feature RMSNorm and LoRA-A partial sums of x,
+ * split-K partial sums and arrival counters) lives in a fixed array of WQ_NOALLOC_SCRATCH_BYTES
  * bytes inside the library, which every GPU that loads the library keeps
  * until the process exits.  A call whose layer needs more scratch than that
  * returns WQ_ERR_UNSUPPORTED and launches nothing.
@@ -197,11 +198,13 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
 /*
  * A stack of gated-MLP layers for one decode step of m tokens:
  *     x_0 = x,  x_{l+1} = x_l + down_l( SiLU(gate_l(xin_l)) * up_l(xin_l) ),  y = x_L
- * with xin_l = RMSNorm(x_l) when flags has WQ_PRENORM, else x_l.  Each layer's
- * gate/up are 2-bit (with LoRA) or 4-bit (no LoRA); down is 4-bit.  x, y:
- * bf16 [m, d]; the residual stream is stored in bf16 between layers.  The
- * call launches every kernel on `stream` with programmatic dependent launch
- * and can be captured into a CUDA graph.
+ * with xin_l = RMSNorm(x_l) (unrounded, as in wq_gateup_w2_lora) when flags has
+ * WQ_PRENORM, else x_l.  Each layer's gate/up are 2-bit (with LoRA) or 4-bit
+ * (no LoRA); down is 4-bit.  x, y: bf16 [m, d]; the residual stream is stored
+ * in bf16 between layers.  The call launches 2 kernels per layer (plus one
+ * for the first layer's input statistics) on `stream` with programmatic
+ * dependent launch, each down launch also producing the next layer's RMSNorm
+ * and LoRA-A partial sums, and can be captured into a CUDA graph.
  */
 wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
                          unsigned flags, void *y, void *ws, size_t ws_bytes, void *stream);

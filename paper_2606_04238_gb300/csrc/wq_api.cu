@@ -66,16 +66,18 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
 
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
-  size_t t, xhat, xa, xb, h, cnt1, cnt2, part1, part2, total;
+  size_t cnt1, cnt2, tp, xa, xb, h, part1, part2, total;
 };
 
 size_t up256(size_t v) { return (v + 255) / 256 * 256; }
 
 size_t partial_bytes(const GemvPlan &p, int nproj) {
-  return p.P > 1 ? (size_t)p.RT * p.P * nproj * 16 * p.MPAD * 4 : 0;
+  return p.P > 1 ? (size_t)p.RT * p.P * nproj * 16 * p.M * 4 : 0;
 }
 
-// Largest split-K partial buffer any plan of this shape can need.
+// Largest split-K partial buffer any plan of this shape can need (every
+// group size and LoRA rank, including the down launch that writes the next
+// layer's tile partials).
 bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2) {
   const int sms = num_sms();
   if (sms <= 0) return false;
@@ -88,9 +90,9 @@ bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2) {
         if (plan_gemv(kGateUpW2, inter, d, m, g, r, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
         if (r == 0 && plan_gemv(kGateUpW4, inter, d, m, g, 0, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
       }
+      if (inter % g == 0 && (r == 0 || d % 8 == 0) && plan_gemv(kDownW4, d, inter, m, g, r, sms, &pl))
+        *p2 = std::max(*p2, partial_bytes(pl, 1));
     }
-    GemvPlan pl;
-    if (inter % g == 0 && plan_gemv(kDownW4, d, inter, m, g, 0, sms, &pl)) *p2 = std::max(*p2, partial_bytes(pl, 1));
   }
   return true;
 }
@@ -103,8 +105,7 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
   size_t off = 0;
   L->cnt1 = off; off = up256(off + (size_t)((inter + 15) / 16) * 4);
   L->cnt2 = off; off = up256(off + (size_t)((d + 15) / 16) * 4);
-  L->t = off;    off = up256(off + (size_t)m * 2 * kMaxRank * 4);
-  L->xhat = off; off = up256(off + (size_t)m * d * 2);
+  L->tp = off;   off = up256(off + (size_t)((d + 15) / 16) * m * (1 + 2 * kMaxRank) * 4);
   L->xa = off;   off = up256(off + (size_t)m * d * 2);
   L->xb = off;   off = up256(off + (size_t)m * d * 2);
   L->h = off;    off = up256(off + (size_t)m * inter * 2);
@@ -114,23 +115,27 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
   return true;
 }
 
-// gate/up (2-bit with LoRA, or 4-bit) for one layer.
+// gate/up (2-bit with LoRA, or 4-bit) for one layer.  tp_in: tile partials of
+// x written by the previous launch (the stack's down kernel), or null to have
+// them computed here from x when the RMSNorm or the adapter needs them.
 wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
                      const void *lora_a, const void *lora_bg, const void *lora_bu, int r, float lora_scale,
-                     unsigned flags, void *h, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+                     unsigned flags, void *h, const float *tp_in, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
   const int d = gate->k, inter = gate->n;
   const bool prenorm = (flags & WQ_PRENORM) != 0;
   GemvPlan plan;
   if (!plan_gemv(kind, inter, d, m, gate->group, r, num_sms(), &plan))
     return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits [%d x %d], m=%d, group %d", inter, d, m, gate->group);
-  float *t = reinterpret_cast<float *>(ws + L.t);
-  void *xhat = ws + L.xhat;
-  if (prenorm || r > 0) {
-    cudaError_t e = launch_prep(x, m, d, lora_a, r, prenorm ? 1 : 0, xhat, t, s, true);
-    if (e != cudaSuccess) return cuda_fail(e, "prologue launch");
+  const bool need_tp = prenorm || r > 0;
+  float *tp_ws = reinterpret_cast<float *>(ws + L.tp);
+  const float *tp = tp_in;
+  if (need_tp && !tp) {
+    cudaError_t e = launch_tile_prep(x, m, d, lora_a, 2 * r, tp_ws, s, true);
+    if (e != cudaSuccess) return cuda_fail(e, "tile-partials launch");
+    tp = tp_ws;
   }
   GemvArgs a = {};
-  a.act = prenorm ? xhat : x;
+  a.act = x;
   a.M = m;
   a.K = d;
   a.N = inter;
@@ -139,7 +144,9 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   a.codes[1] = up->codes;
   a.meta[0] = gate->meta;
   a.meta[1] = up->meta;
-  a.t = t;
+  a.tp = need_tp ? tp : nullptr;
+  a.ntp = d / 16;
+  a.prenorm = prenorm ? 1 : 0;
   a.lora_b[0] = lora_bg;
   a.lora_b[1] = lora_bu;
   a.r = r;
@@ -153,7 +160,7 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   a.nb_meta[0] = a.nb_meta[1] = mb;
   a.nb_lora_b[0] = a.nb_lora_b[1] = (size_t)inter * r * 2;
   a.nb_act = (size_t)m * d * 2;
-  a.nb_t = (size_t)m * 2 * r * 4;
+  a.nb_tp = (size_t)(d / 16) * m * (1 + 2 * r) * 4;
   a.nb_out = (size_t)m * inter * 2;
   a.nb_part = L.part2 - L.part1;
   a.nb_cnt = (size_t)((inter + 15) / 16) * 4;
@@ -162,10 +169,14 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   return WQ_OK;
 }
 
+// down for one layer; with tp_out, also the next layer's tile partials of y
+// (RMSNorm sums and, for r_next > 0, the products with its LoRA-A).
 wq_status run_down(const void *h, int m, const wq_qweight *down, const void *residual, void *y, int y_f32,
-                   const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+                   const void *lora_a_next, int r_next, float *tp_out, const WsLayout &L, uint8_t *ws,
+                   cudaStream_t s) {
+  const int rr = tp_out ? r_next : 0;
   GemvPlan plan;
-  if (!plan_gemv(kDownW4, down->n, down->k, m, down->group, 0, num_sms(), &plan))
+  if (!plan_gemv(kDownW4, down->n, down->k, m, down->group, rr, num_sms(), &plan))
     return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits [%d x %d], m=%d", down->n, down->k, m);
   GemvArgs a = {};
   a.act = h;
@@ -175,9 +186,12 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.group = down->group;
   a.codes[0] = down->codes;
   a.meta[0] = down->meta;
+  a.r = rr;
   a.residual = residual;
   a.out = y;
   a.out_f32 = y_f32;
+  a.lora_a_next = rr > 0 ? lora_a_next : nullptr;
+  a.tp_out = tp_out;
   a.partials = reinterpret_cast<float *>(ws + L.part2);
   a.counters = reinterpret_cast<unsigned *>(ws + L.cnt2);
   size_t cb = 0, mb = 0;
@@ -187,6 +201,8 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.nb_act = (size_t)m * down->k * 2;
   a.nb_res = residual ? (size_t)m * down->n * 2 : 0;
   a.nb_out = (size_t)m * down->n * (y_f32 ? 4 : 2);
+  a.nb_an = (size_t)2 * rr * down->n * 2;
+  a.nb_tp_out = tp_out ? (size_t)((down->n + 15) / 16) * m * (1 + 2 * rr) * 4 : 0;
   a.nb_part = L.total - L.part2;
   a.nb_cnt = (size_t)((down->n + 15) / 16) * 4;
   cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);
@@ -240,8 +256,8 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, gate->k, gate->n, &L)) != WQ_OK) return st;
-  st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, L, static_cast<uint8_t *>(ws),
-                  static_cast<cudaStream_t>(stream));
+  st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
+                  static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
   return st == WQ_OK ? ok() : st;
 }
 
@@ -362,9 +378,9 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
   if ((st = noalloc_scratch(&base)) != WQ_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the arrival counters must start at zero
-  cudaError_t e = cudaMemsetAsync(static_cast<uint8_t *>(base) + L.cnt1, 0, L.t - L.cnt1, s);
+  cudaError_t e = cudaMemsetAsync(static_cast<uint8_t *>(base) + L.cnt1, 0, L.tp - L.cnt1, s);
   if (e != cudaSuccess) return cuda_fail(e, "clearing the built-in scratch counters");
-  st = run_gateup(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, L,
+  st = run_gateup(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, nullptr, L,
                   static_cast<uint8_t *>(base), s);
   return st == WQ_OK ? ok() : st;
 }
@@ -386,7 +402,7 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
     return fail(WQ_ERR_ALIGN, "h, y or residual not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, down->n, down->k, &L)) != WQ_OK) return st;
-  st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
+  st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, nullptr, 0, nullptr, L, static_cast<uint8_t *>(ws),
                 static_cast<cudaStream_t>(stream));
   return st == WQ_OK ? ok() : st;
 }
@@ -429,16 +445,29 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
   if ((st = check_ws(ws, ws_bytes, m, d, inter, &L)) != WQ_OK) return st;
   uint8_t *w8 = static_cast<uint8_t *>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool prenorm = (flags & WQ_PRENORM) != 0;
+  float *tp = reinterpret_cast<float *>(w8 + L.tp);
+  // Launch chain (programmatic dependent launch throughout): the first
+  // layer's tile partials from x, then per layer gate/up -> down, each down
+  // also writing the next layer's tile partials of its output.
+  if (prenorm || layers[0].r > 0) {
+    cudaError_t e = launch_tile_prep(x, m, d, layers[0].lora_a, 2 * layers[0].r, tp, s, true);
+    if (e != cudaSuccess) return cuda_fail(e, "tile-partials launch");
+  }
   const void *cur = x;
   void *hbuf = w8 + L.h;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
     const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+    const bool need_tp = prenorm || Ly.r > 0;
     st = run_gateup(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale, flags,
-                    hbuf, L, w8, s);
+                    hbuf, need_tp ? tp : nullptr, L, w8, s);
     if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
-    st = run_down(hbuf, m, &Ly.down, cur, out, 0, L, w8, s);
+    const wq_mlp_layer *nx = l + 1 < n_layers ? &layers[l + 1] : nullptr;
+    const bool next_tp = nx && (prenorm || nx->r > 0);
+    st = run_down(hbuf, m, &Ly.down, cur, out, 0, next_tp ? nx->lora_a : nullptr, next_tp ? nx->r : 0,
+                  next_tp ? tp : nullptr, L, w8, s);
     if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     cur = out;
   }

@@ -6,32 +6,41 @@
 //     into the epilogue, so the intermediate g/u never leave the chip
 //     (Sec. 5 models the MLP operators as one fused kernel);
 //   * gate+up, 4-bit codes (the uniform-W4 comparator);
-//   * down, 4-bit codes, residual add fused into the epilogue.
+//   * down, 4-bit codes, residual add fused into the epilogue, optionally
+//     followed by the next layer's per-tile RMSNorm / LoRA-A partial sums.
 //
-// Data path of one CTA (one row block x one feature panel):
-//   1. one thread issues bulk (TMA) copies of the packed codes and binary16
-//      scales/zeros of its row tiles into shared memory -- before waiting on
-//      the previous kernel (programmatic dependent launch), so the weight
-//      stream of this kernel overlaps the tail of the previous one;
-//   2. after griddepcontrol.wait, each token's activation panel is loaded
-//      (plain 16-byte loads) and converted in place to binary16 with an exact
-//      power-of-two scale per token (and per code position class, see below),
-//      and per-group activation sums are formed;
-//   3. each warp owns one 16-row tile and a share of the panel: a 16-byte
-//      shared load per lane yields the tensor-core A fragments of 64 (2-bit)
-//      or 32 (4-bit) codes; codes are isolated with a single AND each -- the
-//      isolated bits read as a binary16 subnormal code * 4^c * 2^-24, the
-//      4^c (c = bit-position class) being cancelled by the activation's
+// The decode step is a chain of these launches joined by programmatic
+// dependent launch.  Everything a launch can do before its input exists is
+// done before griddepcontrol.wait, so that it overlaps the previous launch:
+//   1. each warp's lane 0 bulk-copies (TMA) the packed codes and binary16
+//      scales/zeros of the warp's slice into shared memory; LoRA-B rows and
+//      the next layer's LoRA-A columns are staged with plain loads;
+//   2. after the wait, every input of the previous launch is requested in one
+//      round trip: the activation panel (converted to binary16, one
+//      128-feature block per warp item, with an exact power-of-two scale per
+//      (block, token) and per code position class, below), the tile partials
+//      of the input (sum x^2 and A x per 16 features, added up for the
+//      epilogue) and the residual rows;
+//   3. each warp owns one or two 16-row tiles and a share of the panel: a
+//      16-byte shared load per lane yields the tensor-core A fragments of 64
+//      (2-bit) or 32 (4-bit) codes; codes are isolated with a single AND each
+//      -- the isolated bits read as a binary16 subnormal code * 4^c * 2^-24,
+//      the 4^c (c = bit-position class) being cancelled by the activation's
 //      class scale -- and fed to mma.sync m16n8k16 (fp32 accumulation);
-//   4. per group: acc += s * (sum_k code*x - z * sum_k x), i.e. the affine
-//      dequantization s(q - z) is applied once per group, not per weight;
+//   4. per group: acc += s * sx * sum_k code*x (block scale sx); the
+//      zero-point part -s * z * sum_k x of the affine dequantization s(q - z)
+//      is added once per output row after the loop;
 //   5. warps' partial sums are reduced in shared memory in a fixed order;
 //      with several panels the last-arriving CTA of a row tile adds the
 //      panel partials in panel order (deterministic), then the epilogue
-//      (LoRA-B expansion, SiLU(g)*u, or residual add) stores the outputs.
+//      (RMSNorm scale, LoRA-B expansion, SiLU(g)*u; or residual add and the
+//      next layer's tile partials) stores the outputs.
 #include <algorithm>
 #include <climits>
 #include <cmath>
+#include <map>
+#include <mutex>
+#include <tuple>
 
 #include "wq_internal.h"
 #include "wq_ptx.cuh"
@@ -75,12 +84,6 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4 v, float (&f)[8]) {
   f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 __device__ __forceinline__ uint32_t pack_half2(float a, float b) {
   const __half2 h = __floats2half2_rn(a, b);
   return *reinterpret_cast<const uint32_t *>(&h);
@@ -90,21 +93,28 @@ __device__ __forceinline__ float half_bits_to_float(uint32_t bits16) {
   return __half2float(__ushort_as_half(static_cast<unsigned short>(bits16 & 0xffffu)));
 }
 
+constexpr int kMaxThreads = 512;  // per CTA: up to 128 registers a thread
+
 // ---------------------------------------------------------------------------
 // The dequant-GEMV kernel.
 //   BITS  2 or 4 (code width), NPROJ 2 (gate+up) or 1 (down),
 //   GROUP 32/64/128 (quantization group), NT 1 or 2 (8-token MMA tiles per
-//   token chunk: chunks of 8 tokens for m <= 8, of 16 otherwise).
+//   token chunk: chunks of 8 tokens for m <= 8, of 16 otherwise), TPW 1 or 2
+//   (row tiles per warp: with 2, each activation fragment feeds 2 tiles x
+//   NPROJ projections).
 // ---------------------------------------------------------------------------
-template <int BITS, int NPROJ, int GROUP, int NT>
-__global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvArgs a, const GemvPlan p) {
+template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
+__global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a, const GemvPlan p) {
   extern __shared__ __align__(128) uint8_t smem[];
   constexpr int BPK = BITS == 2 ? 512 : 1024;  // code bytes per (row tile, 128-feature block)
   constexpr int GPB = 128 / GROUP;             // groups per block
   constexpr int GS = GROUP / 16;               // k-steps (16 features) per group
   constexpr int TOK = 8 * NT;                  // tokens per chunk
+  constexpr int LPG = GROUP / 4;               // conversion lanes per group (4 features a lane)
+  constexpr int CB = 16;                       // (block, token) items a warp loads before converting
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nwarps = blockDim.x >> 5;
   const int rb = blockIdx.x / p.P, panel = blockIdx.x % p.P;
   const int rt0 = rb * p.RB;
   const int nrt = min(p.RB, p.RT - rt0);
@@ -112,290 +122,374 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
   const int nkb = min(p.KP, p.KB - kb0);
   const int NG = p.KB * GPB;
   const int M = a.M, MPAD = p.MPAD;
+  const int r = a.r;
+  const int Q = 1 + 2 * r;  // values per (tile, token) of the tile partials
 
   uint8_t *codes_s = smem + p.off_codes;
   uint8_t *meta_s = smem + p.off_meta;
+  const __nv_bfloat16 *lorab_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_lorab);  // [NPROJ][RB*16][r]
+  const __nv_bfloat16 *an_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_an);        // [2r][RB*16]
   __half *xp_s = reinterpret_cast<__half *>(smem + p.off_xp);
-  float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);
-  float *scale_s = reinterpret_cast<float *>(smem + p.off_scale);
+  float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);    // [KP*GPB][MPAD] group sums of x
+  float *sc_s = reinterpret_cast<float *>(smem + p.off_sc);    // [KP][MPAD] block scales 2^(24-e)
   float *slot_s = reinterpret_cast<float *>(smem + p.off_slots);
-  float *t_s = reinterpret_cast<float *>(smem + p.off_t);
+  float *red_s = reinterpret_cast<float *>(smem + p.off_red);  // [threads] chunk sums of tile partials
+  float *rt_s = reinterpret_cast<float *>(smem + p.off_rt);    // [M][Q] tile partials summed over tiles
+  float *yv_s = reinterpret_cast<float *>(smem + p.off_yv);    // [RB*16][MPAD] residual, then stored outputs (down)
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + p.off_bar);
   int *last_s = reinterpret_cast<int *>(smem + p.off_last);
 
   // ---- 1. weight prefetch (independent of the previous kernel) ----
-  // Warp (rw, wk) owns row tile rw and blocks [kbs, kbe) of the panel; its
-  // lane 0 bulk-copies exactly that slice (both projections) on its own
-  // barrier, so each warp starts as soon as its own weights have landed.
-  const int rw = warp % p.RB, wk = warp / p.RB;
+  // Warp (rg, wk) owns row tiles rg*TPW .. rg*TPW+TPW-1 of the block and
+  // blocks [kbs, kbe) of the panel; its lane 0 bulk-copies exactly that
+  // slice (every projection) on its own barrier, so each warp starts as soon
+  // as its own weights have landed.
+  const int RG = p.RB / TPW;
+  const int rg = warp % RG, wk = warp / RG;
   const int kbs = wk * nkb / p.WK, kbe = (wk + 1) * nkb / p.WK;
-  const bool has_slice = rw < nrt && kbe > kbs;
+  const int ntw = max(0, min(TPW, nrt - rg * TPW));  // row tiles of this warp inside the matrix
+  const bool has_slice = ntw > 0 && kbe > kbs;
   if (lane == 0 && has_slice) {
     uint64_t *bar = &bars[warp];
     mbar_init(bar, 1);
     fence_barrier_init();
-    const int rt = rt0 + rw, nb = kbe - kbs;
-    mbar_arrive_expect_tx(bar, NPROJ * nb * (BPK + GPB * 64));
+    const int nb = kbe - kbs;
+    mbar_arrive_expect_tx(bar, NPROJ * ntw * nb * (BPK + GPB * 64));
+    for (int j = 0; j < ntw; ++j) {
+      const int rl = rg * TPW + j, rt = rt0 + rl;
 #pragma unroll
-    for (int pj = 0; pj < NPROJ; ++pj) {
-      const size_t cd = p.off_codes + ((size_t)(pj * p.RB + rw) * p.KP + kbs) * BPK;
-      const size_t cs = ((size_t)rt * p.KB + kb0 + kbs) * BPK;
-      if (WQ_OK_IF(WQ_RANGE(cd, nb * BPK, p.off_meta, 16), 1, cd) &&
-          WQ_OK_IF(WQ_RANGE(cs, nb * BPK, a.nb_codes[pj], 16), 2, cs))
-        bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nb * BPK, bar);
-      const size_t md = p.off_meta + ((size_t)(pj * p.RB + rw) * p.KP * GPB + (size_t)kbs * GPB) * 64;
-      const size_t ms = ((size_t)rt * NG + (size_t)(kb0 + kbs) * GPB) * 64;
-      if (WQ_OK_IF(WQ_RANGE(md, nb * GPB * 64, p.off_lorab, 16), 3, md) &&
-          WQ_OK_IF(WQ_RANGE(ms, nb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
-        bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nb * GPB * 64, bar);
+      for (int pj = 0; pj < NPROJ; ++pj) {
+        const size_t cd = p.off_codes + ((size_t)(pj * p.RB + rl) * p.KP + kbs) * BPK;
+        const size_t cs = ((size_t)rt * p.KB + kb0 + kbs) * BPK;
+        if (WQ_OK_IF(WQ_RANGE(cd, nb * BPK, p.off_meta, 16), 1, cd) &&
+            WQ_OK_IF(WQ_RANGE(cs, nb * BPK, a.nb_codes[pj], 16), 2, cs))
+          bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nb * BPK, bar);
+        const size_t md = p.off_meta + ((size_t)(pj * p.RB + rl) * p.KP * GPB + (size_t)kbs * GPB) * 64;
+        const size_t ms = ((size_t)rt * NG + (size_t)(kb0 + kbs) * GPB) * 64;
+        if (WQ_OK_IF(WQ_RANGE(md, nb * GPB * 64, p.off_lorab, 16), 3, md) &&
+            WQ_OK_IF(WQ_RANGE(ms, nb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
+          bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nb * GPB * 64, bar);
+      }
     }
   }
-  int *tokmax_s = reinterpret_cast<int *>(scale_s + MPAD);
-  for (int i = tid; i < nkb * GPB * MPAD; i += blockDim.x) xs_s[i] = 0.f;
-  for (int i = tid; i < MPAD; i += blockDim.x) {
-    scale_s[i] = 0.f;
-    tokmax_s[i] = 0;
+  // LoRA-B rows of this CTA's row tiles (gate/up with an adapter).
+  if (NPROJ == 2 && r > 0) {
+    const int rows = nrt * 16, per_row = r / 8;
+    for (int i = tid; i < NPROJ * rows * per_row; i += blockDim.x) {
+      const int pj = i / (rows * per_row), rem = i % (rows * per_row);
+      const int rl = rem / per_row, c = rem % per_row;
+      const int n = rt0 * 16 + rl;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      const size_t src = ((size_t)n * r + (size_t)c * 8) * 2;
+      if (n < a.N && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_lora_b[pj], 16), 30, n))
+        v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_b[pj]) + src));
+      const size_t dst = p.off_lorab + (((size_t)pj * p.RB * 16 + rl) * r + (size_t)c * 8) * 2;
+      if (WQ_OK_IF(WQ_RANGE(dst, 16, p.off_an, 16), 31, i)) *reinterpret_cast<uint4 *>(smem + dst) = v;
+    }
   }
+  // The next layer's LoRA-A columns for this CTA's output rows (down writing tile partials).
+  if (NPROJ == 1 && a.tp_out != nullptr && r > 0) {
+    const int per = nrt * 2;  // 16-byte chunks per LoRA-A row (16 columns a tile)
+    for (int i = tid; i < 2 * r * per; i += blockDim.x) {
+      const int j = i / per, c = i % per;
+      const int col = rt0 * 16 + c * 8;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      const size_t src = ((size_t)j * a.N + col) * 2;
+      if (col + 8 <= a.N && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_an, 16), 32, i))
+        v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_a_next) + src));
+      const size_t dst = p.off_an + ((size_t)j * p.RB * 16 + (size_t)c * 8) * 2;
+      if (WQ_OK_IF(WQ_RANGE(dst, 16, p.off_xp, 16), 33, i)) *reinterpret_cast<uint4 *>(smem + dst) = v;
+    }
+  }
+  for (int i = tid; i < nkb * GPB * MPAD; i += blockDim.x) xs_s[i] = 0.f;
+  for (int i = tid; i < nkb * MPAD; i += blockDim.x) sc_s[i] = 0.f;
   __syncthreads();  // barrier initialisation visible before any thread waits on it
 
   pdl_launch_dependents();
-  pdl_wait();  // activations (and LoRA-A products) of the previous kernel are ready
+  pdl_wait();  // activations and tile partials of the previous kernel are ready
 
-  // ---- 2. activation panel -> binary16 with per-token power-of-two scale ----
+  // ---- 2. inputs of the previous kernel, all requested in one round trip ----
+  // residual rows of this CTA (down): loaded now, added in the epilogue
+  if (NPROJ == 1 && a.residual) {
+    for (int i = tid; i < nrt * 16 * M; i += blockDim.x) {
+      const int rl = i / M, m = i - rl * M;
+      const int n = rt0 * 16 + rl;
+      float v = 0.f;
+      if (n < a.N && WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_res, 2), 29, n))
+        v = __bfloat162float(__ldcg(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + n));
+      if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 39, i))
+        yv_s[(size_t)rl * MPAD + m] = v;
+    }
+  }
+  // Activation panel -> binary16, one (block, token) item per warp at a
+  // time.  Scale 2^e puts the block's max|x| in [2^14, 2^15): binary16 then
+  // holds every scaled bf16 value exactly (bf16 has 8 significant bits), far
+  // from overflow.  Lane L holds features 4L..4L+3 of the block, i.e. k-step
+  // L/4, and writes them in the order the B fragments read them.  The tile
+  // partials of the input (gate/up) are added while the first batch of
+  // activation loads is in flight.
+  const bool use_tp = NPROJ == 2 && a.tp != nullptr;
+  const int MQ = M * Q;
+  const int nch = use_tp ? max(1, min((int)blockDim.x / MQ, a.ntp)) : 1;
+  bool tp_done = !use_tp;
   const int kbeg = kb0 * 128;
-  const int kvalid = min(nkb * 128, a.K - kbeg);  // a multiple of 8
-  // Activations are staged with ordinary loads, not a bulk copy: the panel is
-  // converted in place below, and shared memory filled by the async (bulk
-  // copy) proxy is only ever read afterwards in this kernel.
-  {
-    const __nv_bfloat16 *act = reinterpret_cast<const __nv_bfloat16 *>(a.act);
-    const int nch = kvalid / 8;  // 16-byte chunks per token row
-    for (int i = tid; i < M * nch; i += blockDim.x) {
-      const int m = i / nch, c = i % nch;
-      const size_t src = ((size_t)m * a.K + kbeg + (size_t)c * 8) * 2;
-      if (WQ_OK_IF(WQ_RANGE(src, 16, a.nb_act, 16), 8, src) &&
-          WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + c * 8) * 2, 16, p.off_xs, 16), 7, i))
-        *reinterpret_cast<uint4 *>(xp_s + (size_t)m * p.xstride + c * 8) = ldg_cg128(act + (size_t)m * a.K + kbeg + c * 8);
-    }
-  }
-  if (NPROJ == 2 && a.r > 0) {
-    for (int i = tid; i < M * 2 * a.r; i += blockDim.x)
-      if (WQ_OK_IF(WQ_RANGE((size_t)i * 4, 4, a.nb_t, 4), 9, i) &&
-          WQ_OK_IF(WQ_RANGE(p.off_t + (size_t)i * 4, 4, p.off_bar, 4), 10, i))
-        t_s[i] = ldcg_f32(a.t + i);
-  }
-  __syncthreads();
-  {
-    // Work item = 16 features of one token (one MMA k-step).  Pass 1: per
-    // token max|x|.  Pass 2: in place, bf16 -> scaled binary16 in the order
-    // the B fragments read it, plus per-group sums of x.
-    const int nsteps = nkb * 8;
-    const int total = M * nsteps;
-    for (int i = tid; i < total; i += blockDim.x) {
-      const int m = i / nsteps, st = i % nsteps;
-      if (st * 16 < kvalid &&
-          WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + st * 16) * 2, 32, p.off_xs, 16), 11, i)) {
-        const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(xp_s + (size_t)m * p.xstride + st * 16);
-        float f[16];
-        unpack_bf16x8(lds128(src), *reinterpret_cast<float(*)[8]>(f));
-        unpack_bf16x8(lds128(src + 8), *reinterpret_cast<float(*)[8]>(f + 8));
-        const int nv = min(16, kvalid - st * 16);
-        float mx = 0.f;
+  const int nitems = nkb * M;
+  for (int it0 = warp; it0 < nitems || !tp_done; it0 += nwarps * CB) {
+    uint2 v[CB];
 #pragma unroll
-        for (int e = 0; e < 16; ++e)
-          if (e < nv) mx = fmaxf(mx, fabsf(f[e]));
-        if (WQ_OK_IF(m < MPAD, 12, m)) atomicMax(&tokmax_s[m], __float_as_int(mx));
+    for (int c = 0; c < CB; ++c) {
+      const int it = it0 + c * nwarps;
+      v[c] = make_uint2(0u, 0u);
+      if (it < nitems) {
+        const int kb = it / M, m = it - kb * M;
+        const int kvalid = min(128, a.K - kbeg - kb * 128);  // a multiple of 32
+        const size_t src = ((size_t)m * a.K + kbeg + kb * 128 + 4 * lane) * 2;
+        if (4 * lane < kvalid && WQ_OK_IF(WQ_RANGE(src, 8, a.nb_act, 8), 8, src))
+          v[c] = ldg_cg64(reinterpret_cast<const uint8_t *>(a.act) + src);
       }
     }
-    __syncthreads();
-    constexpr int LG = GROUP / 16;  // lanes (work items) per group
-    for (int base = warp * 32; base < total; base += blockDim.x) {
-      const int i = base + lane;
-      const bool valid = i < total;
-      const int m = valid ? i / nsteps : 0, st = valid ? i % nsteps : 0;
-      float f[16];
+    if (!tp_done) {
+      // each thread adds up to 32 tiles of one (token, value) pair per round
+      tp_done = true;
+      float *dst = nch > 1 ? red_s : rt_s;
+      for (int w = tid; w < nch * MQ; w += blockDim.x) {
+        const int pair = w % MQ, ch = w / MQ;
+        const int m = pair / Q, q = pair % Q;
+        const int t0 = ch * a.ntp / nch, t1 = (ch + 1) * a.ntp / nch;
+        float acc = 0.f;
+        for (int tb = t0; tb < t1; tb += 32) {
+          float tv[32];
 #pragma unroll
-      for (int e = 0; e < 16; ++e) f[e] = 0.f;
-      __half *slot = xp_s + (size_t)m * p.xstride + st * 16;
-      const bool slot_ok = !valid || WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + st * 16) * 2, 32,
-                                                       p.off_xs, 16), 13, i);
-      if (valid && slot_ok && st * 16 < kvalid) {
-        const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(slot);
-        unpack_bf16x8(lds128(src), *reinterpret_cast<float(*)[8]>(f));
-        unpack_bf16x8(lds128(src + 8), *reinterpret_cast<float(*)[8]>(f + 8));
-        if (st * 16 + 8 > kvalid) {
+          for (int u = 0; u < 32; ++u) {
+            const size_t o = ((size_t)(tb + u) * M + m) * Q + q;
+            tv[u] = (tb + u < t1 && WQ_OK_IF(WQ_RANGE(o * 4, 4, a.nb_tp, 4), 34, tb + u)) ? __ldcg(a.tp + o) : 0.f;
+          }
 #pragma unroll
-          for (int e = 8; e < 16; ++e) f[e] = 0.f;
+          for (int u = 0; u < 32; ++u) acc += tv[u];
         }
+        if (WQ_OK_IF(nch > 1 ? WQ_RANGE(p.off_red + (size_t)w * 4, 4, p.off_rt, 4)
+                             : WQ_RANGE(p.off_rt + (size_t)w * 4, 4, p.off_yv, 4), 36, w))
+          dst[w] = acc;
       }
-      float gs = 0.f;
+    }
 #pragma unroll
-      for (int e = 0; e < 16; ++e) gs += f[e];
-      // scale 2^e puts max|x| in [2^14, 2^15): binary16 holds every scaled
-      // value exactly (bf16 has 8 significant bits), far from overflow.
-      const float mx = __int_as_float(valid ? tokmax_s[m] : 0);
+    for (int c = 0; c < CB; ++c) {
+      const int it = it0 + c * nwarps;
+      if (it >= nitems) break;  // warp-uniform
+      const int kb = it / M, m = it - kb * M;
+      const float f[4] = {bf16_lo(v[c].x), bf16_hi(v[c].x), bf16_lo(v[c].y), bf16_hi(v[c].y)};
+      float mx = fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3])));
+#pragma unroll
+      for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       int e = 0;
       if (mx > 0.f && mx <= 3.4e38f) {
         int E;
         frexpf(mx, &E);
         e = max(-100, min(100, 15 - E));
       }
-      if (valid && slot_ok) {
-        const float up = ldexpf(1.f, e);
-        if (st == 0) scale_s[m] = ldexpf(1.f, 24 - e);
-        // bit-position class of the codes feeding features 0-7 / 8-15 of this step
-        const int sh_lo = BITS == 2 ? 4 * (st & 1) : 0;
-        const int sh_hi = BITS == 2 ? sh_lo + 2 : 4;
-        const float mul_lo = up * ldexpf(1.f, -sh_lo), mul_hi = up * ldexpf(1.f, -sh_hi);
-        uint32_t w[8];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          w[2 * j] = pack_half2(f[2 * j] * mul_lo, f[2 * j + 1] * mul_lo);
-          w[2 * j + 1] = pack_half2(f[8 + 2 * j] * mul_hi, f[9 + 2 * j] * mul_hi);
-        }
-        uint4 *dst = reinterpret_cast<uint4 *>(slot);
-        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+      // bit-position class of the codes that meet these features: 4^c for
+      // 2-bit codes (c from the k-step parity and the feature half), 16^c for
+      // 4-bit codes (c from the feature half)
+      const int st = lane >> 2, hi = (lane >> 1) & 1;
+      const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
+      const float mul = ldexpf(1.f, e - sh);
+      const size_t xo = (size_t)m * p.xstride + (size_t)(kb * 8 + st) * 16;  // halves
+      if (WQ_OK_IF(WQ_RANGE(p.off_xp + xo * 2, 32, p.off_xs, 16), 11, it)) {
+        uint32_t *slot = reinterpret_cast<uint32_t *>(xp_s + xo);
+        const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
+        slot[u0] = pack_half2(f[0] * mul, f[1] * mul);
+        slot[u0 + 2] = pack_half2(f[2] * mul, f[3] * mul);
       }
+      // per-group sums of x (natural units) for the zero-point term
+      float gs = (f[0] + f[1]) + (f[2] + f[3]);
 #pragma unroll
-      for (int o = 1; o < LG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
-      if (valid && (lane % LG) == 0 &&
-          WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)(st / LG) * MPAD + m) * 4, 4, p.off_scale, 4), 14, i))
-        xs_s[(st / LG) * MPAD + m] = gs * ldexpf(1.f, e - 24);
+      for (int o = 1; o < LPG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
+      if ((lane % LPG) == 0) {
+        const int gl = kb * GPB + lane / LPG;
+        if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + m) * 4, 4, p.off_sc, 4), 14, it)) xs_s[gl * MPAD + m] = gs;
+      }
+      if (lane == 0 && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + m) * 4, 4, p.off_slots, 4), 12, it))
+        sc_s[kb * MPAD + m] = ldexpf(1.f, 24 - e);
     }
   }
   __syncthreads();
 
   // ---- 3./4. tensor-core dot products ----
-  if (rw < nrt) {
+  if (ntw > 0) {
     const bool ok = !has_slice || mbar_wait(&bars[warp], 0);
     if (!ok && lane == 0) record_timeout();
-    const uint8_t *cbase = codes_s + (size_t)(rw * p.KP) * BPK + lane * 16;
-    const uint8_t *mbase = meta_s + (size_t)(rw * p.KP * GPB) * 64 + (lane >> 2) * 8;
+    // tile j of this warp: codes at + j*KP*BPK, meta at + j*KP*GPB*64.  A
+    // missing tile (ragged row end, j >= ntw) multiplies whatever its shared
+    // memory holds and is never stored.
+    const uint8_t *cbase = codes_s + (size_t)(rg * TPW * p.KP) * BPK + lane * 16;
+    const uint8_t *mbase = meta_s + (size_t)(rg * TPW * p.KP * GPB) * 64 + (lane >> 2) * 8;
     const size_t cproj = (size_t)p.RB * p.KP * BPK;
     const size_t mproj = (size_t)p.RB * p.KP * GPB * 64;
     for (int tc = 0; tc * TOK < M; ++tc) {
-      float ctot[NPROJ][NT][4];
+      float ctot[NPROJ][TPW][NT][4];
 #pragma unroll
       for (int pj = 0; pj < NPROJ; ++pj)
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
+        for (int j = 0; j < TPW; ++j)
 #pragma unroll
-          for (int q = 0; q < 4; ++q) ctot[pj][nt][q] = 0.f;
+          for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) ctot[pj][j][nt][q] = 0.f;
       for (int kb = ok ? kbs : kbe; kb < kbe; ++kb) {
         uint32_t b[8][NT][2];
+        float2 scv[NT];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
+          scv[nt] = make_float2(0.f, 0.f);
+          if (WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + col) * 4, 8, p.off_slots, 8), 18, col))
+            scv[nt] = *reinterpret_cast<const float2 *>(sc_s + kb * MPAD + col);
+        }
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int m = tc * TOK + nt * 8 + (lane >> 2);
+            b[ks][nt][0] = 0u;
+            b[ks][nt][1] = 0u;
             if (m < M && WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + (kb * 8 + ks) * 16 + 4 * (lane & 3)) * 2,
                                            8, p.off_xs, 8), 15, kb)) {
               const uint2 v = lds64(xp_s + (size_t)m * p.xstride + (kb * 8 + ks) * 16 + 4 * (lane & 3));
               b[ks][nt][0] = v.x;
               b[ks][nt][1] = v.y;
-            } else {
-              b[ks][nt][0] = 0u;
-              b[ks][nt][1] = 0u;
             }
           }
+        constexpr int NW = BITS == 2 ? 4 : 8;  // code words a lane holds per (tile, block)
+        uint32_t wds[NPROJ][TPW][NW];
 #pragma unroll
-        for (int pj = 0; pj < NPROJ; ++pj) {
-          const uint8_t *cb = cbase + pj * cproj + (size_t)kb * BPK;
-          uint32_t wds[BITS == 2 ? 4 : 8];
-          wds[0] = wds[1] = wds[2] = wds[3] = 0u;
-          if (BITS == 4) wds[BITS == 4 ? 4 : 0] = wds[BITS == 4 ? 5 : 1] = wds[BITS == 4 ? 6 : 2] = wds[BITS == 4 ? 7 : 3] = 0u;
-          if (WQ_OK_IF(WQ_RANGE(cb - smem, BPK == 512 ? 16 : 528, p.off_meta, 16), 16, kb)) {
-            const uint4 w0 = lds128(cb);
-            wds[0] = w0.x; wds[1] = w0.y; wds[2] = w0.z; wds[3] = w0.w;
-            if (BITS == 4) {
-              const uint4 w1 = lds128(cb + 512);
-              wds[BITS == 4 ? 4 : 0] = w1.x; wds[BITS == 4 ? 5 : 1] = w1.y;
-              wds[BITS == 4 ? 6 : 2] = w1.z; wds[BITS == 4 ? 7 : 3] = w1.w;
-            }
-          }
-          // two independent accumulator chains (even / odd k-steps) per group
-          float cg[NT][4], ch[NT][4];
+        for (int pj = 0; pj < NPROJ; ++pj)
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
+          for (int j = 0; j < TPW; ++j) {
+            const uint8_t *cb = cbase + pj * cproj + ((size_t)j * p.KP + kb) * BPK;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) cg[nt][q] = ch[nt][q] = 0.f;
-#pragma unroll
-          for (int ks = 0; ks < 8; ++ks) {
-            uint32_t af[4];
-            if (BITS == 2) {
-              const uint32_t x = wds[(ks >> 1) & 3];
-              const uint32_t x8 = x >> 8;
-              const int s4 = (ks & 1) * 4;
-              af[0] = x & (0x00030003u << s4);   // rows g,   features 2t..2t+1
-              af[1] = x8 & (0x00030003u << s4);  // rows g+8
-              af[2] = x & (0x000C000Cu << s4);   // rows g,   features 2t+8..2t+9
-              af[3] = x8 & (0x000C000Cu << s4);  // rows g+8
-            } else {
-              const uint32_t x = wds[ks & (BITS == 2 ? 3 : 7)];
-              const uint32_t x8 = x >> 8;
-              af[0] = x & 0x000F000Fu;
-              af[1] = x8 & 0x000F000Fu;
-              af[2] = x & 0x00F000F0u;
-              af[3] = x8 & 0x00F000F0u;
-            }
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              if (ks & 1)
-                mma_f16_16816(ch[nt], af, b[ks][nt][0], b[ks][nt][1]);
-              else
-                mma_f16_16816(cg[nt], af, b[ks][nt][0], b[ks][nt][1]);
-            }
-            if ((ks + 1) % GS == 0) {
-              const int gl = kb * GPB + ks / GS;
-              uint2 mt = make_uint2(0u, 0u);
-              if (WQ_OK_IF(WQ_RANGE(mbase + pj * mproj + (size_t)gl * 64 - smem, 8, p.off_lorab, 8), 17, gl))
-                mt = lds64(mbase + pj * mproj + (size_t)gl * 64);
-              const float s_lo = half_bits_to_float(mt.x), s_hi = half_bits_to_float(mt.x >> 16);
-              const float z_lo = half_bits_to_float(mt.y), z_hi = half_bits_to_float(mt.y >> 16);
-#pragma unroll
-              for (int nt = 0; nt < NT; ++nt) {
-                const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
-                float2 xs = make_float2(0.f, 0.f);
-                if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + col) * 4, 8, p.off_scale, 8), 18, col))
-                  xs = *reinterpret_cast<const float2 *>(xs_s + gl * MPAD + col);
-                ctot[pj][nt][0] = fmaf(s_lo, fmaf(-z_lo, xs.x, cg[nt][0] + ch[nt][0]), ctot[pj][nt][0]);
-                ctot[pj][nt][1] = fmaf(s_lo, fmaf(-z_lo, xs.y, cg[nt][1] + ch[nt][1]), ctot[pj][nt][1]);
-                ctot[pj][nt][2] = fmaf(s_hi, fmaf(-z_hi, xs.x, cg[nt][2] + ch[nt][2]), ctot[pj][nt][2]);
-                ctot[pj][nt][3] = fmaf(s_hi, fmaf(-z_hi, xs.y, cg[nt][3] + ch[nt][3]), ctot[pj][nt][3]);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) cg[nt][q] = ch[nt][q] = 0.f;
+            for (int q = 0; q < NW; ++q) wds[pj][j][q] = 0u;
+            if (WQ_OK_IF(WQ_RANGE(cb - smem, BPK == 512 ? 16 : 528, p.off_meta, 16), 16, kb)) {
+              const uint4 w0 = lds128(cb);
+              wds[pj][j][0] = w0.x; wds[pj][j][1] = w0.y; wds[pj][j][2] = w0.z; wds[pj][j][3] = w0.w;
+              if (BITS == 4) {
+                const uint4 w1 = lds128(cb + 512);
+                wds[pj][j][NW - 4] = w1.x; wds[pj][j][NW - 3] = w1.y;
+                wds[pj][j][NW - 2] = w1.z; wds[pj][j][NW - 1] = w1.w;
               }
             }
           }
+        // Accumulation chains per (projection, tile): one, or two (even /
+        // odd k-steps) when a warp would otherwise run a single chain.  The
+        // first MMA of a chain in a group starts from zero.
+        constexpr int NCH = NPROJ * TPW >= 2 ? 1 : 2;
+        float acc[NCH][NPROJ][TPW][NT][4];
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+          const int ch = NCH == 2 ? (ks & 1) : 0;
+          const bool first = (ks % GS) < NCH;  // first k-step of this chain in the group
+#pragma unroll
+          for (int pj = 0; pj < NPROJ; ++pj)
+#pragma unroll
+            for (int j = 0; j < TPW; ++j) {
+              uint32_t af[4];
+              if (BITS == 2) {
+                const uint32_t x = wds[pj][j][(ks >> 1) & 3];
+                const uint32_t x8 = x >> 8;
+                const int s4 = (ks & 1) * 4;
+                af[0] = x & (0x00030003u << s4);   // rows g,   features 2t..2t+1
+                af[1] = x8 & (0x00030003u << s4);  // rows g+8
+                af[2] = x & (0x000C000Cu << s4);   // rows g,   features 2t+8..2t+9
+                af[3] = x8 & (0x000C000Cu << s4);  // rows g+8
+              } else {
+                const uint32_t x = wds[pj][j][ks & (NW - 1)];
+                const uint32_t x8 = x >> 8;
+                af[0] = x & 0x000F000Fu;
+                af[1] = x8 & 0x000F000Fu;
+                af[2] = x & 0x00F000F0u;
+                af[3] = x8 & 0x00F000F0u;
+              }
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                if (first)
+                  mma_f16_16816_zc(acc[ch][pj][j][nt], af, b[ks][nt][0], b[ks][nt][1]);
+                else
+                  mma_f16_16816(acc[ch][pj][j][nt], af, b[ks][nt][0], b[ks][nt][1]);
+              }
+            }
+          if ((ks + 1) % GS == 0) {
+            // per group: ctot += s * sx * sum_k code * x
+            const int gl = kb * GPB + ks / GS;
+#pragma unroll
+            for (int pj = 0; pj < NPROJ; ++pj)
+#pragma unroll
+              for (int j = 0; j < TPW; ++j) {
+                const uint8_t *mp = mbase + pj * mproj + ((size_t)j * p.KP * GPB + gl) * 64;
+                uint32_t sbits = 0u;
+                if (WQ_OK_IF(WQ_RANGE(mp - smem, 4, p.off_lorab, 4), 17, gl)) sbits = lds32(mp);
+                const float s_lo = half_bits_to_float(sbits), s_hi = half_bits_to_float(sbits >> 16);
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                  const float2 sc = scv[nt];
+                  float *ct = ctot[pj][j][nt];
+                  const float *g0 = acc[0][pj][j][nt];
+                  const float *g1 = acc[NCH - 1][pj][j][nt];
+                  const float a0 = NCH == 2 ? g0[0] + g1[0] : g0[0], a1 = NCH == 2 ? g0[1] + g1[1] : g0[1];
+                  const float a2 = NCH == 2 ? g0[2] + g1[2] : g0[2], a3 = NCH == 2 ? g0[3] + g1[3] : g0[3];
+                  ct[0] = fmaf(s_lo * sc.x, a0, ct[0]);
+                  ct[1] = fmaf(s_lo * sc.y, a1, ct[1]);
+                  ct[2] = fmaf(s_hi * sc.x, a2, ct[2]);
+                  ct[3] = fmaf(s_hi * sc.y, a3, ct[3]);
+                }
+              }
+          }
         }
       }
-      // per-warp partial -> shared slot [wk][rw][pj][16][MPAD]
+      // per-warp partial -> shared slot [wk][row tile][pj][16][M] (valid tokens only)
 #pragma unroll
       for (int pj = 0; pj < NPROJ; ++pj)
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const int col = tc * TOK + nt * 8 + 2 * (lane & 3), r0 = lane >> 2;
-          float *sl = slot_s + (size_t)((wk * p.RB + rw) * NPROJ + pj) * 16 * MPAD;
-          if (!WQ_OK_IF(WQ_RANGE((uint8_t *)(sl + (r0 + 8) * MPAD + col) - smem, 8, p.off_t, 4), 19, col)) continue;
-          sl[r0 * MPAD + col] = ctot[pj][nt][0];
-          sl[r0 * MPAD + col + 1] = ctot[pj][nt][1];
-          sl[(r0 + 8) * MPAD + col] = ctot[pj][nt][2];
-          sl[(r0 + 8) * MPAD + col + 1] = ctot[pj][nt][3];
+        for (int j = 0; j < TPW; ++j) {
+          if (j >= ntw) continue;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const int col = tc * TOK + nt * 8 + 2 * (lane & 3), r0 = lane >> 2;
+            float *sl = slot_s + (size_t)((wk * p.RB + rg * TPW + j) * NPROJ + pj) * 16 * M;
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+              if (col + c >= M) continue;
+              if (!WQ_OK_IF(WQ_RANGE((uint8_t *)(sl + (r0 + 8) * M + col + c) - smem, 4, p.off_red, 4), 20, col))
+                continue;
+              sl[r0 * M + col + c] = ctot[pj][j][nt][c];
+              sl[(r0 + 8) * M + col + c] = ctot[pj][j][nt][2 + c];
+            }
+          }
         }
     }
   }
   __syncthreads();
 
-  // ---- 5. reduce the k-split warps (fixed order) and undo the token scale ----
-  const int per_rt = NPROJ * 16 * MPAD;
+  // ---- 5. reduce the k-split warps (fixed order) and add the zero-point
+  // term -sum_g s_g z_g sum_{k in g} x_k of this panel's groups ----
+  const int per_rt = NPROJ * 16 * M;
   for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
     float s = 0.f;
     for (int w = 0; w < p.WK; ++w)
-      if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_t, 4), 20, i))
+      if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_red, 4), 21, i))
         s += slot_s[(size_t)w * p.RB * per_rt + i];
-    const int m = i % MPAD;
-    slot_s[i] = m < M ? s * scale_s[m] : 0.f;
+    const int rti = i / per_rt, rem = i - rti * per_rt;
+    const int pj = rem / (16 * M), r16 = (rem / M) % 16, m = rem % M;
+    // meta of (row r16, group g): 32 halves per (tile, group), s at 4e + h, z at 4e + 2 + h
+    const size_t mrow = ((size_t)(pj * p.RB + rti) * p.KP * GPB) * 64 + (size_t)(4 * (r16 & 7) + (r16 >> 3)) * 2;
+    float zt = 0.f;
+    for (int g = 0; g < nkb * GPB; ++g) {
+      const size_t mo = mrow + (size_t)g * 64;
+      if (WQ_OK_IF(WQ_RANGE(p.off_meta + mo, 6, p.off_lorab, 2), 40, g)) {
+        const uint16_t sb = *reinterpret_cast<const uint16_t *>(meta_s + mo);
+        const uint16_t zb = *reinterpret_cast<const uint16_t *>(meta_s + mo + 4);
+        zt = fmaf(half_bits_to_float(sb) * half_bits_to_float(zb), xs_s[g * MPAD + m], zt);
+      }
+    }
+    slot_s[i] = s - zt;
   }
   __syncthreads();
 
@@ -403,11 +497,11 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
     for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
       const int rti = i / per_rt, rem = i % per_rt;
       const size_t po = ((size_t)(rt0 + rti) * p.P + panel) * per_rt + rem;
-      if (WQ_OK_IF(WQ_RANGE(po * 4, 4, a.nb_part, 4), 21, po)) a.partials[po] = slot_s[i];
+      if (WQ_OK_IF(WQ_RANGE(po * 4, 4, a.nb_part, 4), 22, po)) a.partials[po] = slot_s[i];
     }
     __threadfence();
     __syncthreads();
-    if (tid < nrt && WQ_OK_IF(WQ_RANGE((size_t)(rt0 + tid) * 4, 4, a.nb_cnt, 4), 22, rt0 + tid)) {
+    if (tid < nrt && WQ_OK_IF(WQ_RANGE((size_t)(rt0 + tid) * 4, 4, a.nb_cnt, 4), 23, rt0 + tid)) {
       const unsigned prev = atomicAdd(&a.counters[rt0 + tid], 1u);
       last_s[tid] = prev == (unsigned)(p.P - 1);
     }
@@ -419,7 +513,7 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
       const float *src = a.partials + (size_t)(rt0 + rti) * p.P * per_rt + rem;
       float s = 0.f;
       for (int pp = 0; pp < p.P; ++pp)
-        if (WQ_OK_IF(WQ_RANGE((src - a.partials + (size_t)pp * per_rt) * 4, 4, a.nb_part, 4), 23, pp))
+        if (WQ_OK_IF(WQ_RANGE((src - a.partials + (size_t)pp * per_rt) * 4, 4, a.nb_part, 4), 24, pp))
           s += ldcg_f32(src + (size_t)pp * per_rt);
       slot_s[i] = s;
     }
@@ -430,7 +524,17 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
     __syncthreads();
   }
 
-  // ---- epilogue: LoRA-B + SiLU(g) * u, or residual add ----
+  // the tile partials summed over tiles: finish the chunked sums
+  if (use_tp && nch > 1) {
+    for (int pair = tid; pair < MQ; pair += blockDim.x) {
+      float s = 0.f;
+      for (int c = 0; c < nch; ++c) s += red_s[c * MQ + pair];
+      if (WQ_OK_IF(WQ_RANGE(p.off_rt + (size_t)pair * 4, 4, p.off_yv, 4), 37, pair)) rt_s[pair] = s;
+    }
+    __syncthreads();
+  }
+
+  // ---- epilogue: RMSNorm scale, LoRA-B + SiLU(g) * u; or residual add ----
   const int rows = nrt * 16;
   for (int i = tid; i < rows * M; i += blockDim.x) {
     const int m = i / rows, rl = i % rows;
@@ -438,24 +542,28 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
     if (!last_s[rti]) continue;
     const int n = (rt0 + rti) * 16 + r16;
     if (n >= a.N) continue;
-    const float v0 = slot_s[(size_t)(rti * NPROJ) * 16 * MPAD + r16 * MPAD + m];
+    const float v0 = slot_s[(size_t)(rti * NPROJ) * 16 * M + r16 * M + m];
     if (NPROJ == 2) {
       float g = v0;
-      float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * MPAD + r16 * MPAD + m];
-      if (a.r > 0) {
-        const int r = a.r;
-        const __nv_bfloat16 *bg = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[0]) + (size_t)n * r;
-        const __nv_bfloat16 *bu = reinterpret_cast<const __nv_bfloat16 *>(a.lora_b[1]) + (size_t)n * r;
-        const float *tg = t_s + (size_t)m * 2 * r;
+      float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * M + r16 * M + m];
+      // xin = x * rs (Sec. 3.3 MLP input after RMSNorm, never stored):
+      // g = rs * (x deq(Wg)^T + lora_scale * (x A_g^T) B_g^T)
+      float rs = 1.f;
+      if (use_tp && a.prenorm)
+        rs = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(rt_s[(size_t)m * Q], (float)a.K), kRmsEps)));
+      if (use_tp && r > 0) {
+        const float *tg = rt_s + (size_t)m * Q + 1;
         const float *tu = tg + r;
+        const __nv_bfloat16 *bg = lorab_s + (size_t)rl * r;
+        const __nv_bfloat16 *bu = lorab_s + ((size_t)p.RB * 16 + rl) * r;
         float lg = 0.f, lu = 0.f;
         const bool lora_ok =
-            WQ_OK_IF(WQ_RANGE(((size_t)m * 2 * r + 2 * r) * 4 + p.off_t - 4, 4, p.off_bar, 4), 24, m) &&
-            WQ_OK_IF(WQ_RANGE(((size_t)n * r + r) * 2 - 16, 16, a.nb_lora_b[1], 16), 26, n);
+            WQ_OK_IF(WQ_RANGE(p.off_rt + ((size_t)m * Q + Q) * 4 - 4, 4, p.off_yv, 4), 25, m) &&
+            WQ_OK_IF(WQ_RANGE(p.off_lorab + (((size_t)p.RB * 16 + rl) * r + r) * 2 - 16, 16, p.off_an, 16), 26, rl);
         for (int q = 0; lora_ok && q < r; q += 8) {
           float fg[8], fu[8];
-          unpack_bf16x8(__ldg(reinterpret_cast<const uint4 *>(bg + q)), fg);
-          unpack_bf16x8(__ldg(reinterpret_cast<const uint4 *>(bu + q)), fu);
+          unpack_bf16x8(lds128(bg + q), fg);
+          unpack_bf16x8(lds128(bu + q), fu);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             lg = fmaf(tg[q + e], fg[e], lg);
@@ -465,6 +573,8 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
         g = fmaf(a.lora_scale, lg, g);
         u = fmaf(a.lora_scale, lu, u);
       }
+      g *= rs;
+      u *= rs;
       const float h = g / (1.f + __expf(-g)) * u;
       if (WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_out, 2), 27, n))
         reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(h);
@@ -472,101 +582,94 @@ __global__ void __launch_bounds__(NT == 1 ? 1024 : 512) qgemv_kernel(const GemvA
       float y = v0;
       if (!WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * (a.out_f32 ? 4 : 2), a.out_f32 ? 4 : 2, a.nb_out, 2), 28, n))
         continue;
-      if (a.residual && WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_res, 2), 29, n))
-        y += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + n]);
-      if (a.out_f32)
+      if (a.residual) y += yv_s[(size_t)rl * MPAD + m];
+      if (a.out_f32) {
         reinterpret_cast<float *>(a.out)[(size_t)m * a.N + n] = y;
-      else
-        reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(y);
+      } else {
+        const __nv_bfloat16 yb = __float2bfloat16_rn(y);
+        reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = yb;
+        y = __bfloat162float(yb);
+      }
+      if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 38, rl))
+        yv_s[(size_t)rl * MPAD + m] = y;
+    }
+  }
+
+  // ---- the next layer's tile partials of the stored output (down) ----
+  // Same arithmetic and order as tile_prep_kernel: s = fma(w_c, y_c, s) over
+  // the tile's 16 features, w = y (sum of squares) or a LoRA-A row.
+  if (NPROJ == 1 && a.tp_out != nullptr) {
+    __syncthreads();
+    for (int i = tid; i < nrt * M * Q; i += blockDim.x) {
+      const int rti = i / (M * Q), rem = i % (M * Q);
+      const int m = rem / Q, q = rem % Q;
+      if (!last_s[rti]) continue;
+      const int tile = rt0 + rti;
+      float s = 0.f;
+      for (int r16 = 0; r16 < 16 && tile * 16 + r16 < a.N; ++r16) {
+        const int rl = rti * 16 + r16;
+        const float v = yv_s[(size_t)rl * MPAD + m];
+        const float w = q == 0 ? v : __bfloat162float(an_s[(size_t)(q - 1) * p.RB * 16 + rl]);
+        s = fmaf(w, v, s);
+      }
+      const size_t o = ((size_t)tile * M + m) * Q + q;
+      if (WQ_OK_IF(WQ_RANGE(o * 4, 4, a.nb_tp_out, 4), 35, o)) a.tp_out[o] = s;
     }
   }
 }
 
 // ---------------------------------------------------------------------------
-// Prologue kernel: unit-weight RMSNorm of the MLP input (rounded to bf16,
-// written by CTA 0) and the LoRA-A products t[m, rho] = xin[m] . A[rho]
-// (CTA rho).  Every CTA computes the norm scale of each token with the same
-// fixed-order reduction, so all CTAs see bit-identical xin.
+// Tile partials of an input x [M, d] (d a multiple of 16), one warp per tile
+// of 16 features: tp[tile][m][0] = sum_c x_c^2, tp[tile][m][1 + j] =
+// sum_c A[j, c] x_c, each as s = fma(w_c, x_c, s) over c in order.  The
+// gate/up kernel adds them up into the RMSNorm scale and the LoRA-A
+// products x A^T of Eq. 1.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) prep_kernel(const __nv_bfloat16 *x, int M, int d,
-                                                    const __nv_bfloat16 *lora_a, int r2, int prenorm,
-                                                    __nv_bfloat16 *xhat, float *t, uint32_t smem_bytes) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int nwarps = blockDim.x >> 5;
-  const uint32_t arow_bytes = ((uint32_t)d * 2 + 127u) & ~127u;
-  __nv_bfloat16 *arow = reinterpret_cast<__nv_bfloat16 *>(smem);
-  float *rs_s = reinterpret_cast<float *>(smem + arow_bytes);   // [kMaxTokens]
-  float *red_s = rs_s + kMaxTokens;                              // [32]
-  const int rho = blockIdx.x;
-  const bool lora = r2 > 0;
-
-  if (lora && WQ_OK_IF(rho < r2 && (d * 2) % 16 == 0, 41, rho)) {
-    // the LoRA-A row does not depend on the previous kernel: load it first
-    for (int c = tid; c < d / 8; c += blockDim.x)
-      *reinterpret_cast<uint4 *>(arow + c * 8) = __ldg(reinterpret_cast<const uint4 *>(lora_a + (size_t)rho * d) + c);
-  }
-  (void)smem_bytes;
+__global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, int M, int d,
+                                                         const __nv_bfloat16 *lora_a, int r2, float *tp,
+                                                         size_t nb_x, size_t nb_a, size_t nb_tp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ntp = d / 16;
+  const int tile = blockIdx.x * (blockDim.x >> 5) + warp;
+  const int Q = 1 + r2;
   pdl_launch_dependents();
   pdl_wait();
-
-  const int nch = d / 8;
-  for (int m = warp; m < M; m += nwarps) {
-    float rs = 1.f;
-    if (prenorm) {
-      float ss = 0.f;
-      for (int c = lane; c < nch; c += 32) {
-        float f[8];
-        unpack_bf16x8(ldg_cg128(x + (size_t)m * d + c * 8), f);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) ss = fmaf(f[e], f[e], ss);
-      }
-      ss = warp_sum(ss);
-      rs = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)d), kRmsEps)));
+  if (tile >= ntp) return;
+  const uint8_t *x8 = reinterpret_cast<const uint8_t *>(x);
+  const uint8_t *a8 = reinterpret_cast<const uint8_t *>(lora_a);
+  (void)nb_x;
+  (void)nb_a;
+  (void)nb_tp;
+  for (int m = 0; m < M; ++m) {
+    float v[16];
+    const size_t xo = ((size_t)m * d + (size_t)tile * 16) * 2;
+    uint4 x0 = make_uint4(0u, 0u, 0u, 0u), x1 = x0;
+    if (WQ_OK_IF(WQ_RANGE(xo, 32, nb_x, 16), 44, xo)) {
+      x0 = ldg_cg128(x8 + xo);
+      x1 = ldg_cg128(x8 + xo + 16);
     }
-    if (lane == 0 && WQ_OK_IF(m < kMaxTokens, 42, m)) rs_s[m] = rs;
-  }
-  __syncthreads();
-
-  if (lora) {
-    for (int m = 0; m < M; ++m) {
-      const float rs = rs_s[m];
-      float acc = 0.f;
-      for (int c = tid; c < nch; c += blockDim.x) {
-        float f[8], av[8];
-        unpack_bf16x8(ldg_cg128(x + (size_t)m * d + c * 8), f);
-        unpack_bf16x8(*reinterpret_cast<const uint4 *>(arow + c * 8), av);
+    unpack_bf16x8(x0, *reinterpret_cast<float(*)[8]>(v));
+    unpack_bf16x8(x1, *reinterpret_cast<float(*)[8]>(v + 8));
+    for (int q = lane; q < Q; q += 32) {
+      float s = 0.f;
+      if (q == 0) {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float xv = prenorm ? __bfloat162float(__float2bfloat16_rn(__fmul_rn(f[e], rs))) : f[e];
-          acc = fmaf(xv, av[e], acc);
+        for (int c = 0; c < 16; ++c) s = fmaf(v[c], v[c], s);
+      } else {
+        const size_t ao = ((size_t)(q - 1) * d + (size_t)tile * 16) * 2;
+        uint4 a0 = make_uint4(0u, 0u, 0u, 0u), a1 = a0;
+        if (WQ_OK_IF(WQ_RANGE(ao, 32, nb_a, 16), 45, ao)) {
+          a0 = __ldg(reinterpret_cast<const uint4 *>(a8 + ao));
+          a1 = __ldg(reinterpret_cast<const uint4 *>(a8 + ao + 16));
         }
-      }
-      acc = warp_sum(acc);
-      if (lane == 0) red_s[warp] = acc;
-      __syncthreads();
-      if (tid == 0) {
-        float s = 0.f;
-        for (int w = 0; w < nwarps; ++w) s += red_s[w];
-        if (WQ_OK_IF((size_t)m * r2 + rho < (size_t)M * r2, 43, m)) t[(size_t)m * r2 + rho] = s;
-      }
-      __syncthreads();
-    }
-  }
-
-  if (prenorm && blockIdx.x == 0) {
-    for (int i = tid; i < M * nch; i += blockDim.x) {
-      const int m = i / nch, c = i % nch;
-      float f[8];
-      unpack_bf16x8(ldg_cg128(x + (size_t)m * d + c * 8), f);
-      const float rs = rs_s[m];
-      uint32_t o[4];
+        float w[16];
+        unpack_bf16x8(a0, *reinterpret_cast<float(*)[8]>(w));
+        unpack_bf16x8(a1, *reinterpret_cast<float(*)[8]>(w + 8));
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const __nv_bfloat162 h2 = __floats2bfloat162_rn(__fmul_rn(f[2 * j], rs), __fmul_rn(f[2 * j + 1], rs));
-        o[j] = *reinterpret_cast<const uint32_t *>(&h2);
+        for (int c = 0; c < 16; ++c) s = fmaf(w[c], v[c], s);
       }
-      *reinterpret_cast<uint4 *>(xhat + (size_t)m * d + c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+      const size_t o = ((size_t)tile * M + m) * Q + q;
+      if (WQ_OK_IF(WQ_RANGE(o * 4, 4, nb_tp, 4), 46, o)) tp[o] = s;
     }
   }
 }
@@ -583,23 +686,30 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   const int nproj = kind_nproj(kind);
   const int BPK = kind_bits(kind) == 2 ? 512 : 1024, GPB = 128 / group;
   uint32_t off = 0;
+  p->r = r;
   p->off_codes = off;
   off = align_up(off + (uint32_t)nproj * p->RB * p->KP * BPK, 128);
   p->off_meta = off;
   off = align_up(off + (uint32_t)nproj * p->RB * p->KP * GPB * 64, 128);
-  p->off_lorab = off;
-  if (p->lora_smem) off = align_up(off + (uint32_t)nproj * p->RB * 16 * r * 2, 128);
+  p->off_lorab = off;  // gate/up: LoRA-B rows [2][RB*16][r] bf16
+  off = align_up(off + (nproj == 2 ? (uint32_t)nproj * p->RB * 16 * r * 2 : 0u), 128);
+  p->off_an = off;  // down: next layer's LoRA-A columns [2r][RB*16] bf16
+  off = align_up(off + (nproj == 1 ? (uint32_t)2 * r * p->RB * 16 * 2 : 0u), 128);
   p->xstride = p->KP * 128 + 16;  // row bytes = 256 KP + 32: conflict-free 8-byte fragment loads
   p->off_xp = off;
   off = align_up(off + (uint32_t)p->M * p->xstride * 2, 128);
   p->off_xs = off;
   off = align_up(off + (uint32_t)p->KP * GPB * p->MPAD * 4, 128);
-  p->off_scale = off;  // token scales, then token max|x| bits
-  off = align_up(off + (uint32_t)p->MPAD * 8, 128);
+  p->off_sc = off;
+  off = align_up(off + (uint32_t)p->KP * p->MPAD * 4, 128);
   p->off_slots = off;
-  off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->MPAD * 4, 128);
-  p->off_t = off;
-  off = align_up(off + (nproj == 2 ? (uint32_t)p->M * 2 * r * 4 : 0u), 128);
+  off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->M * 4, 128);
+  p->off_red = off;
+  off = align_up(off + (nproj == 2 ? (uint32_t)p->threads * 4 : 0u), 128);
+  p->off_rt = off;
+  off = align_up(off + (nproj == 2 ? (uint32_t)p->M * (1 + 2 * r) * 4 : 0u), 128);
+  p->off_yv = off;
+  off = align_up(off + (nproj == 1 ? (uint32_t)p->RB * 16 * p->MPAD * 4 : 0u), 128);
   p->off_bar = off;  // one weight barrier per warp
   off = align_up(off + (uint32_t)p->RB * p->WK * 8, 128);
   p->off_last = off;
@@ -607,53 +717,70 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   p->smem = off;
 }
 
-}  // namespace
+constexpr uint32_t kSmemLimit = 232448;       // 227 KB opt-in dynamic shared memory per CTA
+constexpr uint32_t kSmemPerSm = 233472;       // 228 KB shared memory per SM
+constexpr uint32_t kCoResident = 114 * 1024;  // shared memory per SM that leaves room for the next kernel
 
-constexpr uint32_t kSmemLimit = 232448;  // 227 KB opt-in dynamic shared memory per CTA
-
-bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *out) {
-  if (N <= 0 || K <= 0 || M <= 0 || M > kMaxTokens || num_sms <= 0) return false;
+bool search_plan(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *out) {
   const int nproj = kind_nproj(kind);
   const int RT = (N + 15) / 16, KB = (K + 127) / 128;
   const int NT = M <= 8 ? 1 : 2;
   const int tok = 8 * NT;
   const int MPAD = (M + tok - 1) / tok * tok;
   const int chunks = MPAD / tok;
+  const double blk_bytes = (kind_bits(kind) == 2 ? 512.0 : 1024.0) + 64.0 * (128 / group);
+  const double total_bytes = (double)RT * KB * nproj * blk_bytes;
+  const int max_warps = kMaxThreads / 32;
   bool found = false;
   double best = 1e300;
   GemvPlan bp{};
+  for (int TPW = 1; TPW <= (NT == 1 ? 2 : 1); ++TPW)
   for (int KP = 1; KP <= KB; ++KP) {
     const int P = (KB + KP - 1) / KP;
     if ((KB + P - 1) / P != KP) continue;  // one canonical KP per panel count
-    for (int RB = 1; RB <= std::min(RT, kMaxWarps); ++RB) {
-      for (int WK = 1; WK <= 8; WK *= 2) {
-        if (WK > KP || RB * WK > (NT == 1 ? kMaxWarps : kMaxWarps / 2)) continue;
+    for (int RB = TPW; RB <= std::min((RT + TPW - 1) / TPW * TPW, max_warps * TPW); RB += TPW) {
+      const int NRB = (RT + RB - 1) / RB;
+      if ((long long)NRB * P > 8LL * num_sms) continue;  // more than 8 CTAs an SM never pays
+      for (int WK = 1; WK <= std::min(KP, max_warps / (RB / TPW)); ++WK) {
         GemvPlan p{};
         p.RT = RT; p.KB = KB; p.RB = RB; p.KP = KP; p.WK = WK; p.P = P;
-        p.NRB = (RT + RB - 1) / RB;
-        p.M = M; p.MPAD = MPAD; p.NT = NT;
-        p.threads = RB * WK * 32;
-        p.units = p.NRB * P;
-        p.lora_smem = 0;
+        p.NRB = NRB;
+        p.M = M; p.MPAD = MPAD; p.NT = NT; p.TPW = TPW;
+        const int warps = RB / TPW * WK;
+        p.threads = warps * 32;
+        p.units = NRB * P;
         compute_layout(kind, group, r, &p);
         if (p.smem > kSmemLimit) continue;
-        const int occ = std::max(1, std::min({(int)(233472 / (p.smem + 1024)), 2048 / p.threads, 32}));
-        const int per_sm = (p.units + num_sms - 1) / num_sms;           // units landing on the busiest SM
+        const int regs = p.threads * 128;  // registers a CTA may hold (launch bound)
+        const int occ = std::max(1, std::min({(int)(kSmemPerSm / (p.smem + 1024)), 65536 / regs, 2048 / p.threads, 32}));
+        const int per_sm = (p.units + num_sms - 1) / num_sms;  // CTAs landing on the busiest SM
         const int waves = (p.units + num_sms * occ - 1) / (num_sms * occ);
-        // Cycle estimates: a tile-projection (16 rows x 128 features of one
-        // matrix) costs ~45 issue slots, spread over the SM's 4 schedulers;
-        // one warp's chain of tile-projections costs ~120 cycles each of MMA
-        // and shared-memory latency; each CTA wave adds a fixed prologue /
-        // epilogue latency, and a split-panel fixup an L2 round trip.
-        const double tiles = (double)per_sm * RB * KP * nproj * chunks;
-        const double thr = tiles * 45.0 / 4.0;
-        const double lat = (double)((KP + WK - 1) / WK) * nproj * chunks * 120.0 * waves;
-        // the busiest SM's share of the weight stream at ~22 B/cycle (HBM / SMs)
-        const double mem = (double)per_sm * RB * KP * nproj * (kind_bits(kind) == 2 ? 640.0 : 1088.0) / 22.0;
-        // the weight stream (or the issue rate) bounds the bulk; the last
-        // warp's dependent chain after its slice lands is added as a tail
-        double cost = std::max(thr, mem) + lat + 800.0 * waves + (P > 1 ? 1500.0 : 0.0);
-        cost += (p.smem > 113 * 1024 ? 300.0 : 0.0);  // no room to overlap the next kernel's prologue
+        const int res = std::min(per_sm, occ);                 // CTAs resident on that SM at once
+        const int warps_sm = res * warps;
+        // Cycle estimates (measured on GB300): mma.sync m16n8k16 with the
+        // AND-isolation of its codes issues one per ~9 cycles per scheduler
+        // (the 16-lane integer pipe is the limit); the input read after the
+        // wait costs an L2 round trip per batch of 16 converted (block,
+        // token) items a warp handles, ~60 cycles each to convert; a
+        // split-panel fixup three L2 round trips.  The weight stream runs at
+        // ~21 B/cycle per SM (HBM over the SMs), at most ~64 B/cycle into one
+        // SM.
+        const double mma_sm = (double)per_sm * RB * KP * nproj * 8.0 * NT * chunks;  // RB counts padded tiles
+        const double t_mma = mma_sm / std::min(4, warps_sm) * 9.0;
+        const double items = std::ceil((double)KP * M / warps);
+        const double conv = 2500.0 * std::ceil(items / 16.0) + items * 60.0;
+        const double epi = 400.0 + (r > 0 ? 200.0 + 8.0 * r : 0.0) + std::ceil((double)RB * 16 * M / p.threads) * 20.0;
+        const double fix = P > 1 ? 6000.0 : 0.0;
+        const double W = conv + t_mma + epi + fix;
+        const double sm_bytes = (double)per_sm * RB * KP * nproj * blk_bytes;
+        const double stream = std::max(total_bytes / (21.3 * num_sms), sm_bytes / 64.0);
+        // the next launch's CTAs can only prefetch their weights during this
+        // one if this launch leaves them half of the SM's shared memory and
+        // registers
+        const bool room = (uint32_t)res * (p.smem + 1024) <= kCoResident && res * regs <= 32768;
+        double cost = room ? std::max(stream, 2000.0 + W) : stream + W;
+        if (waves > 1) cost += (waves - 1) * (W + 2000.0);
+        cost += 0.5 * p.units;  // ties: fewer, larger CTAs
         if (cost < best) {
           best = cost;
           bp = p;
@@ -666,9 +793,38 @@ bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms
   return found;
 }
 
-template <int BITS, int NPROJ, int GROUP, int NT>
+}  // namespace
+
+bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *out) {
+  if (N <= 0 || K <= 0 || M <= 0 || M > kMaxTokens || num_sms <= 0 || r < 0 || r > kMaxRank) return false;
+  if (kind == kDownW4 && r > 0 && N % 8 != 0) return false;  // next-layer LoRA-A columns load 8 at a time
+  using Key = std::tuple<int, int, int, int, int, int, int>;
+  static std::mutex mu;
+  static std::map<Key, std::pair<bool, GemvPlan>> cache;
+  const Key key{(int)kind, N, K, M, group, r, num_sms};
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      if (it->second.first) *out = it->second.second;
+      return it->second.first;
+    }
+  }
+  GemvPlan p{};
+  const bool ok = search_plan(kind, N, K, M, group, r, num_sms, &p);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    cache[key] = {ok, p};
+  }
+  if (ok) *out = p;
+  return ok;
+}
+
+namespace {
+
+template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
 cudaError_t launch_t(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool pdl) {
-  auto kern = qgemv_kernel<BITS, NPROJ, GROUP, NT>;
+  auto kern = qgemv_kernel<BITS, NPROJ, GROUP, NT, TPW>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -684,18 +840,26 @@ cudaError_t launch_t(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool 
   return cudaLaunchKernelEx(&cfg, kern, a, p);
 }
 
+template <int BITS, int NPROJ, int GROUP>
+cudaError_t launch_v(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool pdl) {
+  if (p.NT == 2) return p.TPW == 1 ? launch_t<BITS, NPROJ, GROUP, 2, 1>(p, a, s, pdl) : cudaErrorInvalidValue;
+  return p.TPW == 2 ? launch_t<BITS, NPROJ, GROUP, 1, 2>(p, a, s, pdl) : launch_t<BITS, NPROJ, GROUP, 1, 1>(p, a, s, pdl);
+}
+
 template <int BITS, int NPROJ>
 cudaError_t launch_g(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool pdl) {
-  const bool two = p.NT == 2;
   switch (a.group) {
-    case 32: return two ? launch_t<BITS, NPROJ, 32, 2>(p, a, s, pdl) : launch_t<BITS, NPROJ, 32, 1>(p, a, s, pdl);
-    case 64: return two ? launch_t<BITS, NPROJ, 64, 2>(p, a, s, pdl) : launch_t<BITS, NPROJ, 64, 1>(p, a, s, pdl);
-    case 128: return two ? launch_t<BITS, NPROJ, 128, 2>(p, a, s, pdl) : launch_t<BITS, NPROJ, 128, 1>(p, a, s, pdl);
+    case 32: return launch_v<BITS, NPROJ, 32>(p, a, s, pdl);
+    case 64: return launch_v<BITS, NPROJ, 64>(p, a, s, pdl);
+    case 128: return launch_v<BITS, NPROJ, 128>(p, a, s, pdl);
     default: return cudaErrorInvalidValue;
   }
 }
 
+}  // namespace
+
 cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl) {
+  if (plan.r != args.r) return cudaErrorInvalidValue;  // shared-memory layout sized for another rank
   switch (kind) {
     case kGateUpW2: return launch_g<2, 2>(plan, args, stream, pdl);
     case kGateUpW4: return launch_g<4, 2>(plan, args, stream, pdl);
@@ -704,24 +868,22 @@ cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &arg
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_prep(const void *x, int M, int d, const void *lora_a, int r, int prenorm, void *xhat, float *t,
-                        cudaStream_t stream, bool pdl) {
-  const uint32_t smem = (((uint32_t)d * 2 + 127u) & ~127u) + (kMaxTokens + 32) * 4 + 16;
-  cudaError_t e = cudaFuncSetAttribute(prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
+cudaError_t launch_tile_prep(const void *x, int M, int d, const void *lora_a, int r2, float *tp, cudaStream_t stream,
+                             bool pdl) {
+  const int ntp = d / 16;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(r > 0 ? 2 * r : 1);
+  cfg.gridDim = dim3((ntp + 7) / 8);
   cfg.blockDim = dim3(256);
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, prep_kernel, reinterpret_cast<const __nv_bfloat16 *>(x), M, d,
-                            reinterpret_cast<const __nv_bfloat16 *>(lora_a), 2 * r, prenorm,
-                            reinterpret_cast<__nv_bfloat16 *>(xhat), t, smem);
+  const size_t nb_x = (size_t)M * d * 2, nb_a = (size_t)r2 * d * 2, nb_tp = (size_t)ntp * M * (1 + r2) * 4;
+  return cudaLaunchKernelEx(&cfg, tile_prep_kernel, reinterpret_cast<const __nv_bfloat16 *>(x), M, d,
+                            reinterpret_cast<const __nv_bfloat16 *>(lora_a), r2, tp, nb_x, nb_a, nb_tp);
 }
 
 cudaError_t read_debug_record(long long rec[4]) {

@@ -11,61 +11,77 @@ namespace wq {
 
 constexpr int kMaxTokens = 64;      // tokens per call on the dequant-GEMV path
 constexpr int kMaxRank = 64;        // LoRA rank limit
-constexpr int kMaxWarps = 32;       // warps per CTA
 constexpr float kRmsEps = 1e-6f;    // RMSNorm epsilon of WQ_PRENORM
 
 // How one dequant-GEMV launch splits its work.
 //   Row tiles (16 output rows) are grouped into row blocks of RB tiles; the
 //   input features (128-wide blocks) into P panels of KP blocks.  One CTA
-//   computes one (row block, panel) unit with RB*WK warps: warp (rw, wk)
-//   owns row tile rw of the block and the wk-th share of the panel's blocks.
-//   With P > 1 the panel partial sums of a row tile are added by whichever
-//   CTA finishes that row tile last (arrival counter, fixed summation order).
+//   computes one (row block, panel) unit with RB/TPW*WK warps: warp (rg, wk)
+//   owns row tiles rg*TPW .. rg*TPW+TPW-1 of the block and the wk-th share
+//   of the panel's blocks.  With P > 1 the panel partial sums of a row tile
+//   are added by whichever CTA finishes that row tile last (arrival counter,
+//   fixed summation order).
 struct GemvPlan {
   int RT, KB;          // row tiles, 128-feature blocks of the whole matrix
   int RB, KP, WK;      // row tiles per unit, blocks per panel, warps along k
   int P, NRB;          // panels, row blocks
   int M, MPAD, NT;     // tokens, tokens padded to the token-chunk size, 8-token tiles per chunk
-  int threads;         // RB * WK * 32
+  int TPW;             // row tiles per warp (1 or 2)
+  int threads;         // RB / TPW * WK * 32
   int units;           // grid size = NRB * P
-  int lora_smem;       // reserved (0): LoRA B rows are read from global memory
+  int r;               // LoRA rank the shared-memory layout was sized for
   uint32_t smem;       // dynamic shared memory bytes
   // byte offsets inside dynamic shared memory
-  uint32_t off_codes, off_meta, off_lorab, off_xp, off_xs, off_scale, off_slots, off_t, off_bar, off_last;
+  uint32_t off_codes, off_meta, off_lorab, off_an, off_xp, off_xs, off_sc, off_slots, off_red, off_rt, off_yv,
+      off_bar, off_last;
   int xstride;         // halves per token row of the converted activation panel
 };
 
+// Per-16-feature "tile partials" connect consecutive launches: for every tile
+// of 16 input features and every token, Q = 1 + 2r fp32 values
+//   [0]      sum of x^2 over the tile's features            (RMSNorm)
+//   [1 + j]  sum over the tile's features of A[j, c] * x[c]   (LoRA-A, Eq. 1)
+// laid out [tile][token][Q].  The gate/up launch adds them over all tiles.
 struct GemvArgs {
   const void *act;           // bf16 [M, K]
   int M, K, N, group;
   const uint32_t *codes[2];  // packed codes of the (one or two) matrices
   const uint16_t *meta[2];   // packed binary16 scales / zeros
-  const float *t;            // LoRA-A products [M, 2r] fp32 (gate/up with LoRA)
+  // gate/up: tile partials of the input (null when neither prenorm nor LoRA)
+  const float *tp;           // [ntp][M][1 + 2r]
+  int ntp;                   // tiles = K / 16
+  int prenorm;               // scale the products by 1/sqrt(mean(x^2) + eps)
   const void *lora_b[2];     // bf16 [N, r]
-  int r;
+  int r;                     // gate/up: LoRA rank; down: rank of lora_a_next
   float lora_scale;
-  const void *residual;      // bf16 [M, N] or null (down projection)
+  // down: residual, output and (optionally) the next layer's tile partials
+  const void *residual;      // bf16 [M, N] or null
   void *out;                 // bf16 or fp32 [M, N]
   int out_f32;
-  float *partials;           // [RT][P][NPROJ][16][MPAD] fp32 (P > 1)
+  const void *lora_a_next;   // bf16 [2r, N] (down with tp_out)
+  float *tp_out;             // [ceil(N/16)][M][1 + 2r] or null
+  float *partials;           // [RT][P][NPROJ][16][M] fp32 (P > 1)
   unsigned *counters;        // [RT] arrival counters, zero between calls
   // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
-  size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_t, nb_res, nb_out, nb_part, nb_cnt;
+  size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_tp, nb_res, nb_out, nb_an, nb_tp_out, nb_part, nb_cnt;
 };
 
 enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
 
-// Plans a launch; returns false if no configuration fits.
+// Plans a launch (memoized); returns false if no configuration fits.
+// r: LoRA rank read by the launch (gate/up: its adapter; down: the next
+// layer's LoRA-A whose tile partials it writes, 0 for none).
 bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *plan);
 
 // Launches the dequant-GEMV kernel of `kind` (programmatic dependent launch
 // when `pdl`).  Returns the CUDA error of the launch.
 cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl);
 
-// Launches the prologue kernel: RMSNorm of x (if prenorm) into xhat and the
-// LoRA-A products t = xin A^T (if r > 0).
-cudaError_t launch_prep(const void *x, int M, int d, const void *lora_a, int r, int prenorm, void *xhat,
-                        float *t, cudaStream_t stream, bool pdl);
+// Launches the tile-partials kernel of an input x [M, d] (d a multiple of
+// 16): tp[tile][m][0] = sum x^2, tp[tile][m][1 + j] = A[j] . x over the
+// tile (r2 = 2r rows of A).
+cudaError_t launch_tile_prep(const void *x, int M, int d, const void *lora_a, int r2, float *tp, cudaStream_t stream,
+                             bool pdl);
 
 // Launches the quantizer / packer (two kernels).
 cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint32_t *codes, uint16_t *meta,

@@ -55,7 +55,9 @@ GATEUP_CASES = [
     (192, 200, 64, 16),     # ragged rows (200 = 12.5 tiles) and features (192 = 1.5 blocks)
     (384, 80, 32, 0),       # group 32, no adapter
     (512, 1000, 128, 32),   # group 128, ragged rows
-    (4096, 48, 128, 8),     # few rows, many feature blocks: split panels
+    (4096, 48, 128, 8),     # few rows, many feature blocks
+    (8192, 16, 128, 8),     # one row tile, 64 feature blocks
+    (16384, 32, 64, 8),     # two row tiles, 128 feature blocks
 ]
 
 
@@ -100,7 +102,7 @@ def test_gateup_w4(wq, d, inter, group, m):
     check_bf16(h, ref, f"h(w4) d={d} I={inter} m={m}")
 
 
-DOWN_CASES = [(256, 768, 64), (200, 384, 32), (1000, 512, 128), (48, 4096, 128), (256, 192, 64)]
+DOWN_CASES = [(256, 768, 64), (200, 384, 32), (1000, 512, 128), (48, 4096, 128), (256, 192, 64), (64, 8192, 128)]
 
 
 @pytest.mark.parametrize("d,inter,group", DOWN_CASES)
@@ -122,11 +124,14 @@ def test_down_w4(wq, d, inter, group, m, residual):
 
 
 def test_split_panels_are_exercised(wq):
-    # the few-rows / many-features cases must take the multi-panel path
-    assert wq.plan_info(wq.KIND_GATEUP_W2, 48, 4096, 1, 128, 8)["panels"] > 1
-    assert wq.plan_info(wq.KIND_DOWN_W4, 48, 4096, 1, 128)["panels"] > 1
-    # the Qwen3-4B down projection (160 row tiles on 152 SMs) splits its features
-    assert wq.plan_info(wq.KIND_DOWN_W4, 2560, 9728, 1, 128)["panels"] > 1
+    # some of the parity cases above must take the multi-panel path (last-
+    # arriving CTA adds the panel partials), and some the single-panel path
+    gu = [wq.plan_info(wq.KIND_GATEUP_W2, i, d, m, g, r)["panels"]
+          for d, i, g, r in GATEUP_CASES for m in (1, 3, 8, 9, 16)]
+    dn = [wq.plan_info(wq.KIND_DOWN_W4, d, i, m, g)["panels"]
+          for d, i, g in DOWN_CASES for m in (1, 4, 8, 12, 16)]
+    assert max(gu) > 1 and min(gu) == 1
+    assert max(dn) > 1 and min(dn) == 1
 
 
 def test_deterministic_across_calls(wq):
