@@ -105,7 +105,7 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
   size_t off = 0;
   L->cnt1 = off; off = up256(off + (size_t)((inter + 15) / 16) * 4);
   L->cnt2 = off; off = up256(off + (size_t)((d + 15) / 16) * 4);
-  L->tp = off;   off = up256(off + (size_t)((d + 15) / 16) * m * (1 + 2 * kMaxRank) * 4);
+  L->tp = off;   off = up256(off + (size_t)((d + 15) / 16) * m * WQ_TP_STRIDE(kMaxRank) * 4);
   L->xa = off;   off = up256(off + (size_t)m * d * 2);
   L->xb = off;   off = up256(off + (size_t)m * d * 2);
   L->h = off;    off = up256(off + (size_t)m * inter * 2);
@@ -160,7 +160,7 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   a.nb_meta[0] = a.nb_meta[1] = mb;
   a.nb_lora_b[0] = a.nb_lora_b[1] = (size_t)inter * r * 2;
   a.nb_act = (size_t)m * d * 2;
-  a.nb_tp = (size_t)(d / 16) * m * (1 + 2 * r) * 4;
+  a.nb_tp = (size_t)(d / 16) * m * WQ_TP_STRIDE(r) * 4;
   a.nb_out = (size_t)m * inter * 2;
   a.nb_part = L.part2 - L.part1;
   a.nb_cnt = (size_t)((inter + 15) / 16) * 4;
@@ -202,7 +202,7 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.nb_res = residual ? (size_t)m * down->n * 2 : 0;
   a.nb_out = (size_t)m * down->n * (y_f32 ? 4 : 2);
   a.nb_an = (size_t)2 * rr * down->n * 2;
-  a.nb_tp_out = tp_out ? (size_t)((down->n + 15) / 16) * m * (1 + 2 * rr) * 4 : 0;
+  a.nb_tp_out = tp_out ? (size_t)((down->n + 15) / 16) * m * WQ_TP_STRIDE(rr) * 4 : 0;
   a.nb_part = L.total - L.part2;
   a.nb_cnt = (size_t)((down->n + 15) / 16) * 4;
   cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);

@@ -111,7 +111,6 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   constexpr int GS = GROUP / 16;               // k-steps (16 features) per group
   constexpr int TOK = 8 * NT;                  // tokens per chunk
   constexpr int LPG = GROUP / 4;               // conversion lanes per group (4 features a lane)
-  constexpr int CB = 16;                       // (block, token) items a warp loads before converting
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
@@ -123,7 +122,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   const int NG = p.KB * GPB;
   const int M = a.M, MPAD = p.MPAD;
   const int r = a.r;
-  const int Q = 1 + 2 * r;  // values per (tile, token) of the tile partials
+  const int Q = 1 + 2 * r;           // values per (tile, token) of the tile partials
+  const int Qp = WQ_TP_STRIDE(r);     // their stride (zero padded)
 
   uint8_t *codes_s = smem + p.off_codes;
   uint8_t *meta_s = smem + p.off_meta;
@@ -133,8 +133,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);    // [KP*GPB][MPAD] group sums of x
   float *sc_s = reinterpret_cast<float *>(smem + p.off_sc);    // [KP][MPAD] block scales 2^(24-e)
   float *slot_s = reinterpret_cast<float *>(smem + p.off_slots);
-  float *red_s = reinterpret_cast<float *>(smem + p.off_red);  // [threads] chunk sums of tile partials
-  float *rt_s = reinterpret_cast<float *>(smem + p.off_rt);    // [M][Q] tile partials summed over tiles
+  float *red_s = reinterpret_cast<float *>(smem + p.off_red);  // [4 * threads] chunk sums of tile partials
+  float *rt_s = reinterpret_cast<float *>(smem + p.off_rt);    // [M][Qp] tile partials summed over tiles
   float *yv_s = reinterpret_cast<float *>(smem + p.off_yv);    // [RB*16][MPAD] residual, then stored outputs (down)
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + p.off_bar);
   int *last_s = reinterpret_cast<int *>(smem + p.off_last);
@@ -209,108 +209,147 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   pdl_wait();  // activations and tile partials of the previous kernel are ready
 
   // ---- 2. inputs of the previous kernel, all requested in one round trip ----
-  // residual rows of this CTA (down): loaded now, added in the epilogue
-  if (NPROJ == 1 && a.residual) {
-    for (int i = tid; i < nrt * 16 * M; i += blockDim.x) {
-      const int rl = i / M, m = i - rl * M;
+  // (a) tile partials of the input (gate/up): work item = (chunk of tiles,
+  // token, 4 values); its first 8 tiles are loaded now, added below.
+  const bool use_tp = NPROJ == 2 && a.tp != nullptr;
+  const int Q4 = Qp / 4;
+  const int ntb8 = (a.ntp + 7) / 8;
+  const int nchk = use_tp ? max(1, min((4 * (int)blockDim.x) / (M * Qp), ntb8)) : 1;
+  const int tpc = (a.ntp + nchk - 1) / nchk;  // tiles per chunk
+  const int tp_items = use_tp ? nchk * M * Q4 : 0;
+  float4 tv[8];
+  auto tp_item_load = [&](int item, int tb) {
+    const int c = item / (M * Q4), rem = item - c * (M * Q4);
+    const int m = rem / Q4, j = rem - m * Q4;
+    const int t1 = min((c + 1) * tpc, a.ntp);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const size_t o = ((size_t)(tb + u) * M + m) * Qp + 4 * j;
+      tv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (tb + u < t1 && WQ_OK_IF(WQ_RANGE(o * 4, 16, a.nb_tp, 16), 34, tb + u))
+        tv[u] = __ldcg(reinterpret_cast<const float4 *>(a.tp + o));
+    }
+  };
+  if (tid < tp_items) tp_item_load(tid, (tid / (M * Q4)) * tpc);
+  // (b) residual rows of this CTA (down): the first RV per thread into
+  // registers now, parked in shared memory after the conversion below
+  constexpr int RV = 4;
+  const int nres = (NPROJ == 1 && a.residual) ? nrt * 16 * M : 0;
+  __nv_bfloat16 resv[RV];
+#pragma unroll
+  for (int k = 0; k < RV; ++k) {
+    const int i = tid + k * (int)blockDim.x;
+    resv[k] = __float2bfloat16_rn(0.f);
+    if (i < nres) {
+      const int rl = M == 1 ? i : i / M, m = M == 1 ? 0 : i - rl * M;
       const int n = rt0 * 16 + rl;
-      float v = 0.f;
       if (n < a.N && WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_res, 2), 29, n))
-        v = __bfloat162float(__ldcg(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + n));
-      if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 39, i))
-        yv_s[(size_t)rl * MPAD + m] = v;
+        resv[k] = __ldcg(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + n);
     }
   }
-  // Activation panel -> binary16, one (block, token) item per warp at a
-  // time.  Scale 2^e puts the block's max|x| in [2^14, 2^15): binary16 then
-  // holds every scaled bf16 value exactly (bf16 has 8 significant bits), far
-  // from overflow.  Lane L holds features 4L..4L+3 of the block, i.e. k-step
-  // L/4, and writes them in the order the B fragments read them.  The tile
-  // partials of the input (gate/up) are added while the first batch of
-  // activation loads is in flight.
-  const bool use_tp = NPROJ == 2 && a.tp != nullptr;
-  const int MQ = M * Q;
-  const int nch = use_tp ? max(1, min((int)blockDim.x / MQ, a.ntp)) : 1;
-  bool tp_done = !use_tp;
+  // (c) the raw bf16 activation panel, staged by asynchronous 16-byte copies
+  // in the natural order (converted in place below)
   const int kbeg = kb0 * 128;
+  {
+    const int cpr = nkb * 16;  // 16-byte chunks per token row of the panel
+    for (int i = tid; i < M * cpr; i += blockDim.x) {
+      const int m = M == 1 ? 0 : i / cpr, c = i - m * cpr;
+      const int feat = kbeg + c * 8;
+      __half *dst = xp_s + (size_t)m * p.xstride + c * 8;
+      const size_t src = ((size_t)m * a.K + feat) * 2;
+      if (!WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + c * 8) * 2, 16, p.off_xs, 16), 7, i)) continue;
+      if (feat < a.K && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_act, 16), 8, src))
+        cp_async16(dst, reinterpret_cast<const uint8_t *>(a.act) + src);
+      else
+        *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    cp_async_commit();
+  }
+  // (a) continued: add the loaded tile partials (more rounds only when a
+  // chunk has more than 8 tiles)
+  for (int item = tid; item < tp_items; item += blockDim.x) {
+    const int c = item / (M * Q4), rem = item - c * (M * Q4);
+    const int t0 = c * tpc, t1 = min(t0 + tpc, a.ntp);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int tb = t0; tb < t1; tb += 8) {
+      if (item != tid || tb != t0) tp_item_load(item, tb);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        acc.x += tv[u].x;
+        acc.y += tv[u].y;
+        acc.z += tv[u].z;
+        acc.w += tv[u].w;
+      }
+    }
+    // chunk sums: red_s[c][m][Qp] (several chunks) or directly rt_s[m][Qp]
+    float *dst = (nchk > 1 ? red_s + (size_t)c * M * Qp : rt_s) + (size_t)rem * 4;
+    if (WQ_OK_IF(nchk > 1 ? WQ_RANGE((size_t)(dst - red_s) * 4 + p.off_red, 16, p.off_rt, 16)
+                          : WQ_RANGE((size_t)(dst - rt_s) * 4 + p.off_rt, 16, p.off_yv, 16), 36, item))
+      *reinterpret_cast<float4 *>(dst) = acc;
+  }
+  cp_async_wait_all();
+  __syncthreads();
+  // Activation panel -> binary16 in place, one (block, token) item per warp.
+  // Scale 2^e puts the block's max|x| in [2^14, 2^15): binary16 then holds
+  // every scaled bf16 value exactly (bf16 has 8 significant bits), far from
+  // overflow.  Lane L holds features 4L..4L+3 of the block, i.e. k-step L/4,
+  // and writes them in the order the B fragments read them.
   const int nitems = nkb * M;
-  for (int it0 = warp; it0 < nitems || !tp_done; it0 += nwarps * CB) {
-    uint2 v[CB];
-#pragma unroll
-    for (int c = 0; c < CB; ++c) {
-      const int it = it0 + c * nwarps;
-      v[c] = make_uint2(0u, 0u);
-      if (it < nitems) {
-        const int kb = it / M, m = it - kb * M;
-        const int kvalid = min(128, a.K - kbeg - kb * 128);  // a multiple of 32
-        const size_t src = ((size_t)m * a.K + kbeg + kb * 128 + 4 * lane) * 2;
-        if (4 * lane < kvalid && WQ_OK_IF(WQ_RANGE(src, 8, a.nb_act, 8), 8, src))
-          v[c] = ldg_cg64(reinterpret_cast<const uint8_t *>(a.act) + src);
-      }
+  for (int it = warp; it < nitems; it += nwarps) {
+    const int kb = M == 1 ? it : it / M, m = M == 1 ? 0 : it - kb * M;
+    __half *blk = xp_s + (size_t)m * p.xstride + (size_t)kb * 128;
+    uint2 raw = make_uint2(0u, 0u);
+    if (WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + kb * 128 + 4 * lane) * 2, 8, p.off_xs, 8), 11, it))
+      raw = lds64(blk + 4 * lane);
+    const float f[4] = {bf16_lo(raw.x), bf16_hi(raw.x), bf16_lo(raw.y), bf16_hi(raw.y)};
+    // max |x| of the block: non-negative floats order like their bit patterns
+    const float mx = __uint_as_float(__reduce_max_sync(
+        0xffffffffu, __float_as_uint(fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3]))))));
+    int e = 0;
+    if (mx > 0.f && mx <= 3.4e38f) {
+      int E;
+      frexpf(mx, &E);
+      e = max(-100, min(100, 15 - E));
     }
-    if (!tp_done) {
-      // each thread adds up to 32 tiles of one (token, value) pair per round
-      tp_done = true;
-      float *dst = nch > 1 ? red_s : rt_s;
-      for (int w = tid; w < nch * MQ; w += blockDim.x) {
-        const int pair = w % MQ, ch = w / MQ;
-        const int m = pair / Q, q = pair % Q;
-        const int t0 = ch * a.ntp / nch, t1 = (ch + 1) * a.ntp / nch;
-        float acc = 0.f;
-        for (int tb = t0; tb < t1; tb += 32) {
-          float tv[32];
-#pragma unroll
-          for (int u = 0; u < 32; ++u) {
-            const size_t o = ((size_t)(tb + u) * M + m) * Q + q;
-            tv[u] = (tb + u < t1 && WQ_OK_IF(WQ_RANGE(o * 4, 4, a.nb_tp, 4), 34, tb + u)) ? __ldcg(a.tp + o) : 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 32; ++u) acc += tv[u];
-        }
-        if (WQ_OK_IF(nch > 1 ? WQ_RANGE(p.off_red + (size_t)w * 4, 4, p.off_rt, 4)
-                             : WQ_RANGE(p.off_rt + (size_t)w * 4, 4, p.off_yv, 4), 36, w))
-          dst[w] = acc;
-      }
+    // bit-position class of the codes that meet these features: 4^c for
+    // 2-bit codes (c from the k-step parity and the feature half), 16^c for
+    // 4-bit codes (c from the feature half)
+    const int st = lane >> 2, hi = (lane >> 1) & 1;
+    const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
+    const float mul = ldexpf(1.f, e - sh);
+    __syncwarp();  // every lane has read its raw features before the block is overwritten
+    {
+      uint32_t *slot = reinterpret_cast<uint32_t *>(blk + st * 16);
+      const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
+      slot[u0] = pack_half2(f[0] * mul, f[1] * mul);
+      slot[u0 + 2] = pack_half2(f[2] * mul, f[3] * mul);
     }
+    // per-group sums of x (natural units) for the zero-point term
+    float gs = (f[0] + f[1]) + (f[2] + f[3]);
 #pragma unroll
-    for (int c = 0; c < CB; ++c) {
-      const int it = it0 + c * nwarps;
-      if (it >= nitems) break;  // warp-uniform
-      const int kb = it / M, m = it - kb * M;
-      const float f[4] = {bf16_lo(v[c].x), bf16_hi(v[c].x), bf16_lo(v[c].y), bf16_hi(v[c].y)};
-      float mx = fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3])));
-#pragma unroll
-      for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      int e = 0;
-      if (mx > 0.f && mx <= 3.4e38f) {
-        int E;
-        frexpf(mx, &E);
-        e = max(-100, min(100, 15 - E));
-      }
-      // bit-position class of the codes that meet these features: 4^c for
-      // 2-bit codes (c from the k-step parity and the feature half), 16^c for
-      // 4-bit codes (c from the feature half)
-      const int st = lane >> 2, hi = (lane >> 1) & 1;
-      const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
-      const float mul = ldexpf(1.f, e - sh);
-      const size_t xo = (size_t)m * p.xstride + (size_t)(kb * 8 + st) * 16;  // halves
-      if (WQ_OK_IF(WQ_RANGE(p.off_xp + xo * 2, 32, p.off_xs, 16), 11, it)) {
-        uint32_t *slot = reinterpret_cast<uint32_t *>(xp_s + xo);
-        const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
-        slot[u0] = pack_half2(f[0] * mul, f[1] * mul);
-        slot[u0 + 2] = pack_half2(f[2] * mul, f[3] * mul);
-      }
-      // per-group sums of x (natural units) for the zero-point term
-      float gs = (f[0] + f[1]) + (f[2] + f[3]);
-#pragma unroll
-      for (int o = 1; o < LPG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
-      if ((lane % LPG) == 0) {
-        const int gl = kb * GPB + lane / LPG;
-        if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + m) * 4, 4, p.off_sc, 4), 14, it)) xs_s[gl * MPAD + m] = gs;
-      }
-      if (lane == 0 && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + m) * 4, 4, p.off_slots, 4), 12, it))
-        sc_s[kb * MPAD + m] = ldexpf(1.f, 24 - e);
+    for (int o = 1; o < LPG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
+    if ((lane % LPG) == 0) {
+      const int gl = kb * GPB + lane / LPG;
+      if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + m) * 4, 4, p.off_sc, 4), 14, it)) xs_s[gl * MPAD + m] = gs;
     }
+    if (lane == 0 && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + m) * 4, 4, p.off_slots, 4), 12, it))
+      sc_s[kb * MPAD + m] = ldexpf(1.f, 24 - e);
+  }
+  for (int i = tid; i < nres; i += blockDim.x) {
+    const int k = (i - tid) / (int)blockDim.x;
+    const int rl = M == 1 ? i : i / M, m = M == 1 ? 0 : i - rl * M;
+    float v = 0.f;
+    if (k < RV) {
+#pragma unroll
+      for (int kk = 0; kk < RV; ++kk)
+        if (kk == k) v = __bfloat162float(resv[kk]);
+    } else {
+      const int n = rt0 * 16 + rl;
+      if (n < a.N && WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_res, 2), 29, n))
+        v = __bfloat162float(__ldcg(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + n));
+    }
+    if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 39, i))
+      yv_s[(size_t)rl * MPAD + m] = v;
   }
   __syncthreads();
 
@@ -470,26 +509,36 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
 
   // ---- 5. reduce the k-split warps (fixed order) and add the zero-point
   // term -sum_g s_g z_g sum_{k in g} x_k of this panel's groups ----
+  // Four lanes per output: each adds every 4th group, then the quad adds up
+  // (fixed order).
   const int per_rt = NPROJ * 16 * M;
-  for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
-    float s = 0.f;
-    for (int w = 0; w < p.WK; ++w)
-      if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_red, 4), 21, i))
-        s += slot_s[(size_t)w * p.RB * per_rt + i];
-    const int rti = i / per_rt, rem = i - rti * per_rt;
-    const int pj = rem / (16 * M), r16 = (rem / M) % 16, m = rem % M;
-    // meta of (row r16, group g): 32 halves per (tile, group), s at 4e + h, z at 4e + 2 + h
-    const size_t mrow = ((size_t)(pj * p.RB + rti) * p.KP * GPB) * 64 + (size_t)(4 * (r16 & 7) + (r16 >> 3)) * 2;
-    float zt = 0.f;
-    for (int g = 0; g < nkb * GPB; ++g) {
-      const size_t mo = mrow + (size_t)g * 64;
-      if (WQ_OK_IF(WQ_RANGE(p.off_meta + mo, 6, p.off_lorab, 2), 40, g)) {
-        const uint16_t sb = *reinterpret_cast<const uint16_t *>(meta_s + mo);
-        const uint16_t zb = *reinterpret_cast<const uint16_t *>(meta_s + mo + 4);
-        zt = fmaf(half_bits_to_float(sb) * half_bits_to_float(zb), xs_s[g * MPAD + m], zt);
+  const int nel = nrt * per_rt, lim = (nel + 7) & ~7;  // equal trip counts for the quads of a warp
+  for (int i = tid >> 2; i < lim; i += blockDim.x >> 2) {
+    const int sub = tid & 3;
+    const bool live = i < nel;
+    float zt = 0.f, s = 0.f;
+    if (live) {
+      const int rti = i / per_rt, rem = i - rti * per_rt;
+      const int pj = rem / (16 * M), r16 = (rem / M) % 16, m = rem % M;
+      // meta of (row r16, group g): 32 halves per (tile, group), s at 4e + h, z at 4e + 2 + h
+      const size_t mrow = ((size_t)(pj * p.RB + rti) * p.KP * GPB) * 64 + (size_t)(4 * (r16 & 7) + (r16 >> 3)) * 2;
+      for (int g = sub; g < nkb * GPB; g += 4) {
+        const size_t mo = mrow + (size_t)g * 64;
+        if (WQ_OK_IF(WQ_RANGE(p.off_meta + mo, 6, p.off_lorab, 2), 40, g)) {
+          const uint16_t sb = *reinterpret_cast<const uint16_t *>(meta_s + mo);
+          const uint16_t zb = *reinterpret_cast<const uint16_t *>(meta_s + mo + 4);
+          zt = fmaf(half_bits_to_float(sb) * half_bits_to_float(zb), xs_s[g * MPAD + m], zt);
+        }
       }
+      if (sub == 0)
+        for (int w = 0; w < p.WK; ++w)
+          if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_red, 4), 21, i))
+            s += slot_s[(size_t)w * p.RB * per_rt + i];
     }
-    slot_s[i] = s - zt;
+    zt += __shfl_xor_sync(0xffffffffu, zt, 1);
+    zt += __shfl_xor_sync(0xffffffffu, zt, 2);
+    __syncwarp();
+    if (live && sub == 0) slot_s[i] = s - zt;
   }
   __syncthreads();
 
@@ -524,13 +573,20 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
     __syncthreads();
   }
 
-  // the tile partials summed over tiles: finish the chunked sums
-  if (use_tp && nch > 1) {
-    for (int pair = tid; pair < MQ; pair += blockDim.x) {
+  // the tile partials summed over tiles: add the chunk sums (fixed order)
+  if (use_tp && nchk > 1) {
+    for (int pair = tid; pair < M * Qp; pair += blockDim.x) {
       float s = 0.f;
-      for (int c = 0; c < nch; ++c) s += red_s[c * MQ + pair];
+      for (int c = 0; c < nchk; ++c) s += red_s[(size_t)c * M * Qp + pair];
       if (WQ_OK_IF(WQ_RANGE(p.off_rt + (size_t)pair * 4, 4, p.off_yv, 4), 37, pair)) rt_s[pair] = s;
     }
+    __syncthreads();
+  }
+
+  // RMSNorm scale of each token, rs = 1/sqrt(mean(x^2) + eps), in place of its sum of squares
+  if (use_tp && a.prenorm) {
+    for (int m = tid; m < M; m += blockDim.x)
+      rt_s[(size_t)m * Qp] = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(rt_s[(size_t)m * Qp], (float)a.K), kRmsEps)));
     __syncthreads();
   }
 
@@ -548,17 +604,15 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
       float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * M + r16 * M + m];
       // xin = x * rs (Sec. 3.3 MLP input after RMSNorm, never stored):
       // g = rs * (x deq(Wg)^T + lora_scale * (x A_g^T) B_g^T)
-      float rs = 1.f;
-      if (use_tp && a.prenorm)
-        rs = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(rt_s[(size_t)m * Q], (float)a.K), kRmsEps)));
+      const float rs = use_tp && a.prenorm ? rt_s[(size_t)m * Qp] : 1.f;
       if (use_tp && r > 0) {
-        const float *tg = rt_s + (size_t)m * Q + 1;
+        const float *tg = rt_s + (size_t)m * Qp + 1;
         const float *tu = tg + r;
         const __nv_bfloat16 *bg = lorab_s + (size_t)rl * r;
         const __nv_bfloat16 *bu = lorab_s + ((size_t)p.RB * 16 + rl) * r;
         float lg = 0.f, lu = 0.f;
         const bool lora_ok =
-            WQ_OK_IF(WQ_RANGE(p.off_rt + ((size_t)m * Q + Q) * 4 - 4, 4, p.off_yv, 4), 25, m) &&
+            WQ_OK_IF(WQ_RANGE(p.off_rt + ((size_t)m * Qp + Q) * 4 - 4, 4, p.off_yv, 4), 25, m) &&
             WQ_OK_IF(WQ_RANGE(p.off_lorab + (((size_t)p.RB * 16 + rl) * r + r) * 2 - 16, 16, p.off_an, 16), 26, rl);
         for (int q = 0; lora_ok && q < r; q += 8) {
           float fg[8], fu[8];
@@ -600,19 +654,19 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   // the tile's 16 features, w = y (sum of squares) or a LoRA-A row.
   if (NPROJ == 1 && a.tp_out != nullptr) {
     __syncthreads();
-    for (int i = tid; i < nrt * M * Q; i += blockDim.x) {
-      const int rti = i / (M * Q), rem = i % (M * Q);
-      const int m = rem / Q, q = rem % Q;
+    for (int i = tid; i < nrt * M * Qp; i += blockDim.x) {
+      const int rti = i / (M * Qp), rem = i % (M * Qp);
+      const int m = rem / Qp, q = rem % Qp;
       if (!last_s[rti]) continue;
       const int tile = rt0 + rti;
       float s = 0.f;
-      for (int r16 = 0; r16 < 16 && tile * 16 + r16 < a.N; ++r16) {
+      for (int r16 = 0; q < Q && r16 < 16 && tile * 16 + r16 < a.N; ++r16) {
         const int rl = rti * 16 + r16;
         const float v = yv_s[(size_t)rl * MPAD + m];
         const float w = q == 0 ? v : __bfloat162float(an_s[(size_t)(q - 1) * p.RB * 16 + rl]);
         s = fmaf(w, v, s);
       }
-      const size_t o = ((size_t)tile * M + m) * Q + q;
+      const size_t o = ((size_t)tile * M + m) * Qp + q;
       if (WQ_OK_IF(WQ_RANGE(o * 4, 4, a.nb_tp_out, 4), 35, o)) a.tp_out[o] = s;
     }
   }
@@ -631,7 +685,7 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ntp = d / 16;
   const int tile = blockIdx.x * (blockDim.x >> 5) + warp;
-  const int Q = 1 + r2;
+  const int Q = 1 + r2, Qp = (Q + 3) & ~3;
   pdl_launch_dependents();
   pdl_wait();
   if (tile >= ntp) return;
@@ -650,9 +704,11 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
     }
     unpack_bf16x8(x0, *reinterpret_cast<float(*)[8]>(v));
     unpack_bf16x8(x1, *reinterpret_cast<float(*)[8]>(v + 8));
-    for (int q = lane; q < Q; q += 32) {
+    for (int q = lane; q < Qp; q += 32) {
       float s = 0.f;
-      if (q == 0) {
+      if (q >= Q) {
+        s = 0.f;  // padding
+      } else if (q == 0) {
 #pragma unroll
         for (int c = 0; c < 16; ++c) s = fmaf(v[c], v[c], s);
       } else {
@@ -668,7 +724,7 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
 #pragma unroll
         for (int c = 0; c < 16; ++c) s = fmaf(w[c], v[c], s);
       }
-      const size_t o = ((size_t)tile * M + m) * Q + q;
+      const size_t o = ((size_t)tile * M + m) * Qp + q;
       if (WQ_OK_IF(WQ_RANGE(o * 4, 4, nb_tp, 4), 46, o)) tp[o] = s;
     }
   }
@@ -705,9 +761,9 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   p->off_slots = off;
   off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->M * 4, 128);
   p->off_red = off;
-  off = align_up(off + (nproj == 2 ? (uint32_t)p->threads * 4 : 0u), 128);
+  off = align_up(off + (nproj == 2 ? (uint32_t)p->threads * 16 : 0u), 128);
   p->off_rt = off;
-  off = align_up(off + (nproj == 2 ? (uint32_t)p->M * (1 + 2 * r) * 4 : 0u), 128);
+  off = align_up(off + (nproj == 2 ? (uint32_t)p->M * WQ_TP_STRIDE(r) * 4 : 0u), 128);
   p->off_yv = off;
   off = align_up(off + (nproj == 1 ? (uint32_t)p->RB * 16 * p->MPAD * 4 : 0u), 128);
   p->off_bar = off;  // one weight barrier per warp
@@ -751,35 +807,44 @@ bool search_plan(GemvKind kind, int N, int K, int M, int group, int r, int num_s
         p.units = NRB * P;
         compute_layout(kind, group, r, &p);
         if (p.smem > kSmemLimit) continue;
-        const int regs = p.threads * 128;  // registers a CTA may hold (launch bound)
+        const int regs = p.threads * ((kernel_regs(kind, group, NT, TPW) + 7) & ~7);  // registers of a CTA
         const int occ = std::max(1, std::min({(int)(kSmemPerSm / (p.smem + 1024)), 65536 / regs, 2048 / p.threads, 32}));
         const int per_sm = (p.units + num_sms - 1) / num_sms;  // CTAs landing on the busiest SM
         const int waves = (p.units + num_sms * occ - 1) / (num_sms * occ);
-        const int res = std::min(per_sm, occ);                 // CTAs resident on that SM at once
-        const int warps_sm = res * warps;
-        // Cycle estimates (measured on GB300): mma.sync m16n8k16 with the
-        // AND-isolation of its codes issues one per ~9 cycles per scheduler
-        // (the 16-lane integer pipe is the limit); the input read after the
-        // wait costs an L2 round trip per batch of 16 converted (block,
-        // token) items a warp handles, ~60 cycles each to convert; a
-        // split-panel fixup three L2 round trips.  The weight stream runs at
-        // ~21 B/cycle per SM (HBM over the SMs), at most ~64 B/cycle into one
-        // SM.
-        const double mma_sm = (double)per_sm * RB * KP * nproj * 8.0 * NT * chunks;  // RB counts padded tiles
-        const double t_mma = mma_sm / std::min(4, warps_sm) * 9.0;
+        // CTAs resident on a typical SM (a grid up to 10% larger than the SM
+        // count leaves only a few SMs with a second CTA)
+        const int res = p.units <= num_sms + num_sms / 10 ? 1 : std::min(per_sm, occ);
+        // Cycle estimates, calibrated on GB300 timings of the decode chain:
+        // after the wait, one L2 round trip for the inputs (~1500), ~250 per
+        // converted (block, token) item a warp handles, the MMA loop at ~8
+        // cycles per m16n8k16 per scheduler when each scheduler has four
+        // warps to switch between (proportionally slower with fewer), ~3000
+        // of reduction and epilogue, ~1000 per further CTA on the SM, ~5000
+        // for a split-panel fixup (three dependent round trips) plus ~100 per
+        // partial a thread adds up, ~3000 between the end of one launch and
+        // the release of the next.  The weight stream runs at ~21 B/cycle per
+        // SM (HBM over the SMs), at most ~64 B/cycle into one SM.
+        const double mma_cta = (double)RB * KP * nproj * 8.0 * NT * chunks;  // RB counts padded tiles
+        const double eff = std::min(1.0, (double)warps * std::min(occ, per_sm) / 16.0);  // CTAs of an SM run together
+        const double t_mma = per_sm * mma_cta * 8.0 / 4.0 / eff;
         const double items = std::ceil((double)KP * M / warps);
-        const double conv = 2500.0 * std::ceil(items / 16.0) + items * 60.0;
-        const double epi = 400.0 + (r > 0 ? 200.0 + 8.0 * r : 0.0) + std::ceil((double)RB * 16 * M / p.threads) * 20.0;
-        const double fix = P > 1 ? 6000.0 : 0.0;
-        const double W = conv + t_mma + epi + fix;
+        const double conv = 1500.0 + items * 250.0;
+        const double epi = 3000.0 + (r > 0 ? 8.0 * r : 0.0) + std::ceil((double)RB * 16 * M / p.threads) * 20.0;
+        // the last-arriving CTA of a row tile loads P partials per output
+        const double fix = P > 1 ? 5000.0 + std::ceil((double)RB * 16 * nproj * M / p.threads) * P * 100.0 : 0.0;
+        const double W = conv + t_mma + epi + fix + 1000.0 * (per_sm - 1);
         const double sm_bytes = (double)per_sm * RB * KP * nproj * blk_bytes;
         const double stream = std::max(total_bytes / (21.3 * num_sms), sm_bytes / 64.0);
-        // the next launch's CTAs can only prefetch their weights during this
-        // one if this launch leaves them half of the SM's shared memory and
-        // registers
-        const bool room = (uint32_t)res * (p.smem + 1024) <= kCoResident && res * regs <= 32768;
-        double cost = room ? std::max(stream, 2000.0 + W) : stream + W;
-        if (waves > 1) cost += (waves - 1) * (W + 2000.0);
+        // The chain alternates gate/up and down launches; the next launch's
+        // CTAs can prefetch their weights during this one only if both fit
+        // on an SM at once: a gate/up launch may take 5/8 of an SM's
+        // registers, a down launch 1/4 (measured: down launches of more
+        // than 8 warps a CTA delay the next gate/up launch), and each about
+        // half its shared memory.
+        const int reg_budget = kind == kDownW4 ? 16384 : 40960;
+        const bool room = (uint32_t)res * (p.smem + 1024) <= kCoResident && res * regs <= reg_budget;
+        double cost = room ? std::max(stream, 3000.0 + W) : stream + 3000.0 + W;
+        if (waves > 1) cost += (waves - 1) * (W + 3000.0);
         cost += 0.5 * p.units;  // ties: fewer, larger CTAs
         if (cost < best) {
           best = cost;
@@ -841,6 +906,13 @@ cudaError_t launch_t(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool 
 }
 
 template <int BITS, int NPROJ, int GROUP>
+const void *kernel_ptr(int NT, int TPW) {
+  if (NT == 2) return reinterpret_cast<const void *>(qgemv_kernel<BITS, NPROJ, GROUP, 2, 1>);
+  return TPW == 2 ? reinterpret_cast<const void *>(qgemv_kernel<BITS, NPROJ, GROUP, 1, 2>)
+                  : reinterpret_cast<const void *>(qgemv_kernel<BITS, NPROJ, GROUP, 1, 1>);
+}
+
+template <int BITS, int NPROJ, int GROUP>
 cudaError_t launch_v(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool pdl) {
   if (p.NT == 2) return p.TPW == 1 ? launch_t<BITS, NPROJ, GROUP, 2, 1>(p, a, s, pdl) : cudaErrorInvalidValue;
   return p.TPW == 2 ? launch_t<BITS, NPROJ, GROUP, 1, 2>(p, a, s, pdl) : launch_t<BITS, NPROJ, GROUP, 1, 1>(p, a, s, pdl);
@@ -857,6 +929,32 @@ cudaError_t launch_g(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool 
 }
 
 }  // namespace
+
+int kernel_regs(GemvKind kind, int group, int NT, int TPW) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, int, int, int>, int> cache;
+  const auto key = std::make_tuple((int)kind, group, NT, TPW);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  const int gi = group == 32 ? 0 : group == 64 ? 1 : 2;
+  const void *fn = nullptr;
+  switch (kind * 3 + gi) {
+    case 0: fn = kernel_ptr<2, 2, 32>(NT, TPW); break;
+    case 1: fn = kernel_ptr<2, 2, 64>(NT, TPW); break;
+    case 2: fn = kernel_ptr<2, 2, 128>(NT, TPW); break;
+    case 3: fn = kernel_ptr<4, 2, 32>(NT, TPW); break;
+    case 4: fn = kernel_ptr<4, 2, 64>(NT, TPW); break;
+    case 5: fn = kernel_ptr<4, 2, 128>(NT, TPW); break;
+    case 6: fn = kernel_ptr<4, 1, 32>(NT, TPW); break;
+    case 7: fn = kernel_ptr<4, 1, 64>(NT, TPW); break;
+    default: fn = kernel_ptr<4, 1, 128>(NT, TPW); break;
+  }
+  cudaFuncAttributes attr{};
+  const int regs = cudaFuncGetAttributes(&attr, fn) == cudaSuccess && attr.numRegs > 0 ? attr.numRegs : 128;
+  cache[key] = regs;
+  return regs;
+}
 
 cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl) {
   if (plan.r != args.r) return cudaErrorInvalidValue;  // shared-memory layout sized for another rank
@@ -881,7 +979,7 @@ cudaError_t launch_tile_prep(const void *x, int M, int d, const void *lora_a, in
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  const size_t nb_x = (size_t)M * d * 2, nb_a = (size_t)r2 * d * 2, nb_tp = (size_t)ntp * M * (1 + r2) * 4;
+  const size_t nb_x = (size_t)M * d * 2, nb_a = (size_t)r2 * d * 2, nb_tp = (size_t)ntp * M * ((1 + r2 + 3) & ~3) * 4;
   return cudaLaunchKernelEx(&cfg, tile_prep_kernel, reinterpret_cast<const __nv_bfloat16 *>(x), M, d,
                             reinterpret_cast<const __nv_bfloat16 *>(lora_a), r2, tp, nb_x, nb_a, nb_tp);
 }

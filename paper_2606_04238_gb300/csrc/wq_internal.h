@@ -38,17 +38,19 @@ struct GemvPlan {
 };
 
 // Per-16-feature "tile partials" connect consecutive launches: for every tile
-// of 16 input features and every token, Q = 1 + 2r fp32 values
+// of 16 input features and every token, 1 + 2r fp32 values
 //   [0]      sum of x^2 over the tile's features            (RMSNorm)
 //   [1 + j]  sum over the tile's features of A[j, c] * x[c]   (LoRA-A, Eq. 1)
-// laid out [tile][token][Q].  The gate/up launch adds them over all tiles.
+// padded with zeros to WQ_TP_STRIDE(r) (a multiple of 4) and laid out
+// [tile][token][stride].  The gate/up launch adds them over all tiles.
+#define WQ_TP_STRIDE(r) ((1 + 2 * (r) + 3) & ~3)
 struct GemvArgs {
   const void *act;           // bf16 [M, K]
   int M, K, N, group;
   const uint32_t *codes[2];  // packed codes of the (one or two) matrices
   const uint16_t *meta[2];   // packed binary16 scales / zeros
   // gate/up: tile partials of the input (null when neither prenorm nor LoRA)
-  const float *tp;           // [ntp][M][1 + 2r]
+  const float *tp;           // [ntp][M][WQ_TP_STRIDE(r)]
   int ntp;                   // tiles = K / 16
   int prenorm;               // scale the products by 1/sqrt(mean(x^2) + eps)
   const void *lora_b[2];     // bf16 [N, r]
@@ -59,7 +61,7 @@ struct GemvArgs {
   void *out;                 // bf16 or fp32 [M, N]
   int out_f32;
   const void *lora_a_next;   // bf16 [2r, N] (down with tp_out)
-  float *tp_out;             // [ceil(N/16)][M][1 + 2r] or null
+  float *tp_out;             // [ceil(N/16)][M][WQ_TP_STRIDE(r)] or null
   float *partials;           // [RT][P][NPROJ][16][M] fp32 (P > 1)
   unsigned *counters;        // [RT] arrival counters, zero between calls
   // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
@@ -73,13 +75,16 @@ enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
 // layer's LoRA-A whose tile partials it writes, 0 for none).
 bool plan_gemv(GemvKind kind, int N, int K, int M, int group, int r, int num_sms, GemvPlan *plan);
 
+// Registers per thread of the kernel instantiation a plan selects (device query, cached).
+int kernel_regs(GemvKind kind, int group, int NT, int TPW);
+
 // Launches the dequant-GEMV kernel of `kind` (programmatic dependent launch
 // when `pdl`).  Returns the CUDA error of the launch.
 cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl);
 
 // Launches the tile-partials kernel of an input x [M, d] (d a multiple of
 // 16): tp[tile][m][0] = sum x^2, tp[tile][m][1 + j] = A[j] . x over the
-// tile (r2 = 2r rows of A).
+// tile (r2 = 2r rows of A), zeros up to the stride.
 cudaError_t launch_tile_prep(const void *x, int M, int d, const void *lora_a, int r2, float *tp, cudaStream_t stream,
                              bool pdl);
 

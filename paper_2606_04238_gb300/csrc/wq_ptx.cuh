@@ -134,6 +134,14 @@ __device__ __forceinline__ uint2 ldg_cg64(const void *p) {
   return v;
 }
 
+// 16-byte asynchronous global -> shared copy (cp.async, cached in L2
+// only); complete after cp_async_wait_all().  Both addresses 16-byte aligned.
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 // fp32 load that bypasses L1 (sees other CTAs' writes after a fence).
 __device__ __forceinline__ float ldcg_f32(const float* p) {
   float v;

@@ -23,21 +23,24 @@ def f64_of_bf16(t):
     return t.detach().float().cpu().numpy().astype(np.float64)
 
 
-def check_bf16(got, ref, what, min_exact=0.97):
+def check_bf16(got, ref, what, min_exact=0.97, depth=1):
     """bf16 device output vs fp64 oracle value.
 
     Bound: max|gpu - oracle| <= 2e-3 (max|oracle| + 1), plus the half-ulp
     rounding of the bf16 store itself (|v| 2^-8 bounds half a bf16 ulp), per
     element.  Also: at least `min_exact` of the elements equal the oracle's
     own bf16 rounding bit for bit (differences only where the fp32 and fp64
-    sums straddle a rounding boundary).
+    sums straddle a rounding boundary).  `depth` > 1 compares the end of a
+    chain of `depth` layers run on their own outputs: each layer's bf16
+    rounding flips are carried into the next, so the bound is depth times the
+    one-layer bound.
     """
     g = f64_of_bf16(got)
     ref = np.asarray(ref, np.float64)
     assert g.shape == ref.shape, (g.shape, ref.shape)
     if ref.size == 0:
         return
-    tol = 2e-3 * (np.abs(ref).max() + 1.0) + np.abs(ref) * 2.0 ** -8
+    tol = depth * (2e-3 * (np.abs(ref).max() + 1.0) + np.abs(ref) * 2.0 ** -8)
     err = np.abs(g - ref)
     bad = err > tol
     assert not bad.any(), f"{what}: {bad.sum()} elements out of bound, max err {err.max():.3e} " \

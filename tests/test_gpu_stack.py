@@ -69,7 +69,7 @@ def test_stack_teacher_forced(wq, m, bits_gu):
     xb = synth.bf16_bits(x)
     for l in range(n_layers):
         y, xb = _orc_layer(cfg, ent[l], xb, prenorm=True)
-    check_bf16(prefix[-1], y, f"stack end-to-end m={m}", min_exact=0.5)
+    check_bf16(prefix[-1], y, f"stack end-to-end m={m}", min_exact=0.5, depth=n_layers)
 
 
 def test_stack_equals_layer_calls(wq):
