@@ -361,7 +361,7 @@ def run_gpu(args):
         gu_gbs, dn_gbs = gu_bytes / t_gu / 1e9, dn_bytes / t_dn / 1e9
         tr = recorded_traffic("gateup_w2_lora")
         out["roofline"] = {"bound": "hbm", "achieved": gu_gbs, "peak": peak, "unit": "GB/s", "frac": gu_gbs / peak,
-                           "traffic": tr, "kernel": "wq_gateup_w2_lora (LoRA-A prologue + fused 2-bit gate/up GEMV)",
+                           "traffic": tr, "kernel": "wq_gateup_w2_lora (first-layer tile-partials kernel + fused 2-bit gate/up GEMV)",
                            "algorithmic_bytes_per_launch": gu_bytes, "us_per_launch": t_gu * 1e6,
                            "peak_source": f"{peak_src} HBM copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"}
         out["kernels"] = {
