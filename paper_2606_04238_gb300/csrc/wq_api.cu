@@ -66,7 +66,7 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
 
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
-  size_t cnt1, cnt2, tp, xa, xb, h, part1, part2, total;
+  size_t cnt1, cnt2, tp, xa, xb, h, hq, hsc, hxs, part1, part2, total;
 };
 
 size_t up256(size_t v) { return (v + 255) / 256 * 256; }
@@ -109,6 +109,9 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
   L->xa = off;   off = up256(off + (size_t)m * d * 2);
   L->xb = off;   off = up256(off + (size_t)m * d * 2);
   L->h = off;    off = up256(off + (size_t)m * inter * 2);
+  L->hq = off;   off = up256(off + (size_t)m * ((inter + 127) / 128) * 128 * 2);
+  L->hsc = off;  off = up256(off + (size_t)((inter + 63) / 64) * m * 4);
+  L->hxs = off;  off = up256(off + (size_t)((inter + 31) / 32) * m * 4);
   L->part1 = off; off = up256(off + p1);
   L->part2 = off; off = up256(off + p2);
   L->total = off;
@@ -118,9 +121,12 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
 // gate/up (2-bit with LoRA, or 4-bit) for one layer.  tp_in: tile partials of
 // x written by the previous launch (the stack's down kernel), or null to have
 // them computed here from x when the RMSNorm or the adapter needs them.
+// With make_hq (decode chain, plans checked by chain_panel_ok), h is also
+// written as the down launch's ready binary16 panel in the workspace.
 wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
                      const void *lora_a, const void *lora_bg, const void *lora_bu, int r, float lora_scale,
-                     unsigned flags, void *h, const float *tp_in, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+                     unsigned flags, void *h, const float *tp_in, const WsLayout &L, uint8_t *ws, cudaStream_t s,
+                     bool make_hq = false) {
   const int d = gate->k, inter = gate->n;
   const bool prenorm = (flags & WQ_PRENORM) != 0;
   GemvPlan plan;
@@ -152,6 +158,15 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
   a.r = r;
   a.lora_scale = lora_scale;
   a.out = h;
+  if (make_hq) {
+    a.hq_out = reinterpret_cast<uint16_t *>(ws + L.hq);
+    a.hsc_out = reinterpret_cast<float *>(ws + L.hsc);
+    a.hxs_out = reinterpret_cast<float *>(ws + L.hxs);
+    a.hq_stride = (inter + 127) / 128 * 128;
+    a.nb_hq = L.hsc - L.hq;
+    a.nb_hsc = L.hxs - L.hsc;
+    a.nb_hxs = (size_t)((inter + 31) / 32) * m * 4;
+  }
   a.partials = reinterpret_cast<float *>(ws + L.part1);
   a.counters = reinterpret_cast<unsigned *>(ws + L.cnt1);
   size_t cb = 0, mb = 0;
@@ -171,9 +186,11 @@ wq_status run_gateup(GemvKind kind, const void *x, int m, const wq_qweight *gate
 
 // down for one layer; with tp_out, also the next layer's tile partials of y
 // (RMSNorm sums and, for r_next > 0, the products with its LoRA-A).
+// With use_hq, the input is the ready binary16 panel the gate/up launch left
+// in the workspace instead of h.
 wq_status run_down(const void *h, int m, const wq_qweight *down, const void *residual, void *y, int y_f32,
                    const void *lora_a_next, int r_next, float *tp_out, const WsLayout &L, uint8_t *ws,
-                   cudaStream_t s) {
+                   cudaStream_t s, bool use_hq = false) {
   const int rr = tp_out ? r_next : 0;
   GemvPlan plan;
   if (!plan_gemv(kDownW4, down->n, down->k, m, down->group, rr, num_sms(), &plan))
@@ -192,6 +209,15 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.out_f32 = y_f32;
   a.lora_a_next = rr > 0 ? lora_a_next : nullptr;
   a.tp_out = tp_out;
+  if (use_hq) {
+    a.pre_x = reinterpret_cast<const uint16_t *>(ws + L.hq);
+    a.pre_sc = reinterpret_cast<const float *>(ws + L.hsc);
+    a.pre_xs = reinterpret_cast<const float *>(ws + L.hxs);
+    a.pre_stride = (down->k + 127) / 128 * 128;
+    a.nb_pre_x = L.hsc - L.hq;
+    a.nb_pre_sc = L.hxs - L.hsc;
+    a.nb_pre_xs = (size_t)((down->k + 31) / 32) * m * 4;
+  }
   a.partials = reinterpret_cast<float *>(ws + L.part2);
   a.counters = reinterpret_cast<unsigned *>(ws + L.cnt2);
   size_t cb = 0, mb = 0;
@@ -208,6 +234,16 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);
   if (e != cudaSuccess) return cuda_fail(e, "down launch");
   return WQ_OK;
+}
+
+// The gate/up launch can hand the down launch a ready binary16 panel when it
+// holds whole 64-feature halves (one panel, row blocks of a multiple of 4
+// tiles) and the down kernel scales its input per half (one row tile a warp).
+bool chain_panel_ok(GemvKind kind, int m, const wq_qweight &gate, int r, const wq_qweight &down, int r_next) {
+  GemvPlan pg, pd;
+  if (!plan_gemv(kind, gate.n, gate.k, m, gate.group, r, num_sms(), &pg)) return false;
+  if (!plan_gemv(kDownW4, down.n, down.k, m, down.group, r_next, num_sms(), &pd)) return false;
+  return pg.P == 1 && pg.RB % 4 == 0 && pd.TPW == 1;
 }
 
 wq_status check_tokens(int m) {
@@ -461,13 +497,15 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
     void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
     const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
     const bool need_tp = prenorm || Ly.r > 0;
-    st = run_gateup(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale, flags,
-                    hbuf, need_tp ? tp : nullptr, L, w8, s);
-    if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     const wq_mlp_layer *nx = l + 1 < n_layers ? &layers[l + 1] : nullptr;
     const bool next_tp = nx && (prenorm || nx->r > 0);
-    st = run_down(hbuf, m, &Ly.down, cur, out, 0, next_tp ? nx->lora_a : nullptr, next_tp ? nx->r : 0,
-                  next_tp ? tp : nullptr, L, w8, s);
+    const int r_next = next_tp ? nx->r : 0;
+    const bool panel = chain_panel_ok(kind, m, Ly.gate, Ly.r, Ly.down, r_next);
+    st = run_gateup(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale, flags,
+                    hbuf, need_tp ? tp : nullptr, L, w8, s, panel);
+    if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    st = run_down(hbuf, m, &Ly.down, cur, out, 0, next_tp ? nx->lora_a : nullptr, r_next, next_tp ? tp : nullptr, L,
+                  w8, s, panel);
     if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     cur = out;
   }

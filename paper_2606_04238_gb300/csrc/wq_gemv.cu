@@ -89,6 +89,18 @@ __device__ __forceinline__ uint32_t pack_half2(float a, float b) {
   return *reinterpret_cast<const uint32_t *>(&h);
 }
 
+// 2^k for -126 <= k <= 127, built from the binary32 exponent field
+__device__ __forceinline__ float exp2i(int k) { return __int_as_float((k + 127) << 23); }
+
+// Scale exponent e of a block whose largest |x| has the bit pattern mxb:
+// 2^e puts it in [2^14, 2^15).  mx = f 2^E with f in [0.5, 1) and E = (biased
+// exponent) - 126, so e = 15 - E, clamped (subnormal mx: 100); 0 for a zero,
+// infinite or nan mx.
+__device__ __forceinline__ int block_exponent(uint32_t mxb) {
+  const int be = (int)(mxb >> 23);
+  return mxb == 0u || be >= 255 ? 0 : max(-100, min(100, 141 - be));
+}
+
 __device__ __forceinline__ float half_bits_to_float(uint32_t bits16) {
   return __half2float(__ushort_as_half(static_cast<unsigned short>(bits16 & 0xffffu)));
 }
@@ -104,13 +116,17 @@ constexpr int kMaxThreads = 512;  // per CTA: up to 128 registers a thread
 //   NPROJ projections).
 // ---------------------------------------------------------------------------
 template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
-__global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a, const GemvPlan p) {
+__global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1 ? 2 : 1) qgemv_kernel(const GemvArgs a, const GemvPlan p) {
   extern __shared__ __align__(128) uint8_t smem[];
   constexpr int BPK = BITS == 2 ? 512 : 1024;  // code bytes per (row tile, 128-feature block)
   constexpr int GPB = 128 / GROUP;             // groups per block
   constexpr int GS = GROUP / 16;               // k-steps (16 features) per group
   constexpr int TOK = 8 * NT;                  // tokens per chunk
   constexpr int LPG = GROUP / 4;               // conversion lanes per group (4 features a lane)
+  // Down with one row tile per warp runs two accumulation chains, one per
+  // 64-feature half of a block, and scales the activations per half
+  // (HALF); the other kernels scale per 128-feature block.
+  constexpr bool HALF = NPROJ * TPW < 2;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
@@ -131,7 +147,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   const __nv_bfloat16 *an_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_an);        // [2r][RB*16]
   __half *xp_s = reinterpret_cast<__half *>(smem + p.off_xp);
   float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);    // [KP*GPB][MPAD] group sums of x
-  float *sc_s = reinterpret_cast<float *>(smem + p.off_sc);    // [KP][MPAD] block scales 2^(24-e)
+  float *sc_s = reinterpret_cast<float *>(smem + p.off_sc);    // [2 KP][MPAD] half-block scales 2^(24-e)
   float *slot_s = reinterpret_cast<float *>(smem + p.off_slots);
   float *red_s = reinterpret_cast<float *>(smem + p.off_red);  // [4 * threads] chunk sums of tile partials
   float *rt_s = reinterpret_cast<float *>(smem + p.off_rt);    // [M][Qp] tile partials summed over tiles
@@ -154,6 +170,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
     mbar_init(bar, 1);
     fence_barrier_init();
     const int nb = kbe - kbs;
+    const uint64_t pol = l2_evict_first_policy();  // weights are read once a step
     mbar_arrive_expect_tx(bar, NPROJ * ntw * nb * (BPK + GPB * 64));
     for (int j = 0; j < ntw; ++j) {
       const int rl = rg * TPW + j, rt = rt0 + rl;
@@ -163,12 +180,12 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
         const size_t cs = ((size_t)rt * p.KB + kb0 + kbs) * BPK;
         if (WQ_OK_IF(WQ_RANGE(cd, nb * BPK, p.off_meta, 16), 1, cd) &&
             WQ_OK_IF(WQ_RANGE(cs, nb * BPK, a.nb_codes[pj], 16), 2, cs))
-          bulk_g2s(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nb * BPK, bar);
+          bulk_g2s_hint(smem + cd, reinterpret_cast<const uint8_t *>(a.codes[pj]) + cs, nb * BPK, bar, pol);
         const size_t md = p.off_meta + ((size_t)(pj * p.RB + rl) * p.KP * GPB + (size_t)kbs * GPB) * 64;
         const size_t ms = ((size_t)rt * NG + (size_t)(kb0 + kbs) * GPB) * 64;
         if (WQ_OK_IF(WQ_RANGE(md, nb * GPB * 64, p.off_lorab, 16), 3, md) &&
             WQ_OK_IF(WQ_RANGE(ms, nb * GPB * 64, a.nb_meta[pj], 16), 4, ms))
-          bulk_g2s(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nb * GPB * 64, bar);
+          bulk_g2s_hint(smem + md, reinterpret_cast<const uint8_t *>(a.meta[pj]) + ms, nb * GPB * 64, bar, pol);
       }
     }
   }
@@ -202,10 +219,9 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
     }
   }
   for (int i = tid; i < nkb * GPB * MPAD; i += blockDim.x) xs_s[i] = 0.f;
-  for (int i = tid; i < nkb * MPAD; i += blockDim.x) sc_s[i] = 0.f;
+  for (int i = tid; i < 2 * nkb * MPAD; i += blockDim.x) sc_s[i] = 0.f;
   __syncthreads();  // barrier initialisation visible before any thread waits on it
 
-  pdl_launch_dependents();
   pdl_wait();  // activations and tile partials of the previous kernel are ready
 
   // ---- 2. inputs of the previous kernel, all requested in one round trip ----
@@ -247,23 +263,78 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
         resv[k] = __ldcg(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + n);
     }
   }
-  // (c) the raw bf16 activation panel, staged by asynchronous 16-byte copies
-  // in the natural order (converted in place below)
+  // (c) the activation panel, staged by asynchronous 16-byte copies: the raw
+  // bf16 rows in the natural order (converted in place below), or the
+  // producer's ready binary16 panel
+  const bool pre = HALF && NPROJ == 1 && a.pre_x != nullptr;
   const int kbeg = kb0 * 128;
   {
+    const uint8_t *srcb = reinterpret_cast<const uint8_t *>(pre ? (const void *)a.pre_x : a.act);
+    const size_t row = pre ? (size_t)a.pre_stride : (size_t)a.K;
+    const size_t nb_src = pre ? a.nb_pre_x : a.nb_act;
+    (void)nb_src;
     const int cpr = nkb * 16;  // 16-byte chunks per token row of the panel
     for (int i = tid; i < M * cpr; i += blockDim.x) {
       const int m = M == 1 ? 0 : i / cpr, c = i - m * cpr;
       const int feat = kbeg + c * 8;
       __half *dst = xp_s + (size_t)m * p.xstride + c * 8;
-      const size_t src = ((size_t)m * a.K + feat) * 2;
+      const size_t src = ((size_t)m * row + feat) * 2;
       if (!WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + c * 8) * 2, 16, p.off_xs, 16), 7, i)) continue;
-      if (feat < a.K && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_act, 16), 8, src))
-        cp_async16(dst, reinterpret_cast<const uint8_t *>(a.act) + src);
+      if (feat < a.K && WQ_OK_IF(WQ_RANGE(src, 16, nb_src, 16), 8, src))
+        cp_async16(dst, srcb + src);
       else
         *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
     }
     cp_async_commit();
+  }
+  // (d) with the ready panel: its half-block scales and the group sums
+  // (from 32-feature sums, added in order)
+  // Four items a thread per round, loads first, so that they are in
+  // flight together.
+  if (pre) {
+    const int nsc = 2 * nkb * M;
+    for (int i0 = tid; i0 < nsc; i0 += 4 * blockDim.x) {
+      float v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * (int)blockDim.x, h = i / M, m = i - h * M, hb = 2 * kb0 + h;
+        v[u] = 0.f;
+        if (i < nsc && hb * 64 < a.K && WQ_OK_IF(WQ_RANGE(((size_t)hb * M + m) * 4, 4, a.nb_pre_sc, 4), 47, hb))
+          v[u] = ldcg_f32(a.pre_sc + (size_t)hb * M + m);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * (int)blockDim.x, h = i / M, m = i - h * M;
+        if (i < nsc && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)h * MPAD + m) * 4, 4, p.off_slots, 4), 48, h))
+          sc_s[h * MPAD + m] = v[u];
+      }
+    }
+    constexpr int QPG = GROUP / 32;
+    const int nxs = nkb * GPB * M;
+    for (int i0 = tid; i0 < nxs; i0 += 2 * blockDim.x) {
+      float v[2][QPG];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int i = i0 + u * (int)blockDim.x, g = i / M, m = i - g * M;
+        const int q0 = (kb0 * GPB + g) * QPG;
+#pragma unroll
+        for (int q = 0; q < QPG; ++q) {
+          v[u][q] = 0.f;
+          if (i < nxs && (q0 + q) * 32 < a.K &&
+              WQ_OK_IF(WQ_RANGE(((size_t)(q0 + q) * M + m) * 4, 4, a.nb_pre_xs, 4), 49, q0 + q))
+            v[u][q] = ldcg_f32(a.pre_xs + (size_t)(q0 + q) * M + m);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int i = i0 + u * (int)blockDim.x, g = i / M, m = i - g * M;
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < QPG; ++q) sum += v[u][q];
+        if (i < nxs && WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)g * MPAD + m) * 4, 4, p.off_sc, 4), 50, g))
+          xs_s[g * MPAD + m] = sum;
+      }
+    }
   }
   // (a) continued: add the loaded tile partials (more rounds only when a
   // chunk has more than 8 tiles)
@@ -289,51 +360,75 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   }
   cp_async_wait_all();
   __syncthreads();
+  // The next launch may start now: its weight stream then runs while this
+  // launch computes, not while its latency-bound input loads above are in
+  // flight.
+  pdl_launch_dependents();
   // Activation panel -> binary16 in place, one (block, token) item per warp.
   // Scale 2^e puts the block's max|x| in [2^14, 2^15): binary16 then holds
   // every scaled bf16 value exactly (bf16 has 8 significant bits), far from
   // overflow.  Lane L holds features 4L..4L+3 of the block, i.e. k-step L/4,
   // and writes them in the order the B fragments read them.
-  const int nitems = nkb * M;
-  for (int it = warp; it < nitems; it += nwarps) {
-    const int kb = M == 1 ? it : it / M, m = M == 1 ? 0 : it - kb * M;
-    __half *blk = xp_s + (size_t)m * p.xstride + (size_t)kb * 128;
-    uint2 raw = make_uint2(0u, 0u);
-    if (WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)m * p.xstride + kb * 128 + 4 * lane) * 2, 8, p.off_xs, 8), 11, it))
-      raw = lds64(blk + 4 * lane);
-    const float f[4] = {bf16_lo(raw.x), bf16_hi(raw.x), bf16_lo(raw.y), bf16_hi(raw.y)};
-    // max |x| of the block: non-negative floats order like their bit patterns
-    const float mx = __uint_as_float(__reduce_max_sync(
-        0xffffffffu, __float_as_uint(fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3]))))));
-    int e = 0;
-    if (mx > 0.f && mx <= 3.4e38f) {
-      int E;
-      frexpf(mx, &E);
-      e = max(-100, min(100, 15 - E));
-    }
-    // bit-position class of the codes that meet these features: 4^c for
-    // 2-bit codes (c from the k-step parity and the feature half), 16^c for
-    // 4-bit codes (c from the feature half)
-    const int st = lane >> 2, hi = (lane >> 1) & 1;
-    const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
-    const float mul = ldexpf(1.f, e - sh);
-    __syncwarp();  // every lane has read its raw features before the block is overwritten
-    {
-      uint32_t *slot = reinterpret_cast<uint32_t *>(blk + st * 16);
-      const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
-      slot[u0] = pack_half2(f[0] * mul, f[1] * mul);
-      slot[u0 + 2] = pack_half2(f[2] * mul, f[3] * mul);
-    }
-    // per-group sums of x (natural units) for the zero-point term
-    float gs = (f[0] + f[1]) + (f[2] + f[3]);
+  // Items it0 + u * nwarps (u < CU) are converted together: independent
+  // dependency chains (load, max reduction, shuffles) in flight at once.
+  constexpr int CU = 2;
+  const int nitems = pre ? 0 : nkb * M;
+  const int st = lane >> 2, hi = (lane >> 1) & 1;
+  // bit-position class of the codes that meet these features: 4^c for 2-bit
+  // codes (c from the k-step parity and the feature half), 16^c for 4-bit
+  // codes (c from the feature half)
+  const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
+  const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
+  const bool lo_half = lane < 16;      // features 0..63 of the block
+  for (int it0 = warp; it0 < nitems; it0 += CU * nwarps) {
+    float f[CU][4];
+    int kbv[CU], mv[CU], e0v[CU], e1v[CU];
 #pragma unroll
-    for (int o = 1; o < LPG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
-    if ((lane % LPG) == 0) {
-      const int gl = kb * GPB + lane / LPG;
-      if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + m) * 4, 4, p.off_sc, 4), 14, it)) xs_s[gl * MPAD + m] = gs;
+    for (int u = 0; u < CU; ++u) {
+      const int it = it0 + u * nwarps;  // warp-uniform
+      kbv[u] = M == 1 ? it : it / M;
+      mv[u] = M == 1 ? 0 : it - kbv[u] * M;
+      uint2 raw = make_uint2(0u, 0u);
+      if (it < nitems &&
+          WQ_OK_IF(WQ_RANGE(p.off_xp + ((size_t)mv[u] * p.xstride + kbv[u] * 128 + 4 * lane) * 2, 8, p.off_xs, 8), 11,
+                   it))
+        raw = lds64(xp_s + (size_t)mv[u] * p.xstride + (size_t)kbv[u] * 128 + 4 * lane);
+      f[u][0] = bf16_lo(raw.x);
+      f[u][1] = bf16_hi(raw.x);
+      f[u][2] = bf16_lo(raw.y);
+      f[u][3] = bf16_hi(raw.y);
     }
-    if (lane == 0 && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + m) * 4, 4, p.off_slots, 4), 12, it))
-      sc_s[kb * MPAD + m] = ldexpf(1.f, 24 - e);
+#pragma unroll
+    for (int u = 0; u < CU; ++u) {
+      // max |x| of the block or of each half: non-negative floats order like
+      // their bit patterns
+      const uint32_t v = __float_as_uint(fmaxf(fmaxf(fabsf(f[u][0]), fabsf(f[u][1])), fmaxf(fabsf(f[u][2]), fabsf(f[u][3]))));
+      const uint32_t mx0 = __reduce_max_sync(0xffffffffu, HALF ? (lo_half ? v : 0u) : v);
+      const uint32_t mx1 = HALF ? __reduce_max_sync(0xffffffffu, lo_half ? 0u : v) : mx0;
+      e0v[u] = block_exponent(mx0);
+      e1v[u] = block_exponent(mx1);
+    }
+    __syncwarp();  // every lane has read its raw features before the blocks are overwritten
+#pragma unroll
+    for (int u = 0; u < CU; ++u) {
+      const int it = it0 + u * nwarps;
+      if (it >= nitems) break;  // warp-uniform
+      const float mul = exp2i((lo_half ? e0v[u] : e1v[u]) - sh);
+      uint32_t *slot = reinterpret_cast<uint32_t *>(xp_s + (size_t)mv[u] * p.xstride + (size_t)kbv[u] * 128 + st * 16);
+      slot[u0] = pack_half2(f[u][0] * mul, f[u][1] * mul);
+      slot[u0 + 2] = pack_half2(f[u][2] * mul, f[u][3] * mul);
+      // per-group sums of x (natural units) for the zero-point term
+      float gs = (f[u][0] + f[u][1]) + (f[u][2] + f[u][3]);
+#pragma unroll
+      for (int o = 1; o < LPG; o <<= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
+      if ((lane % LPG) == 0) {
+        const int gl = kbv[u] * GPB + lane / LPG;
+        if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + mv[u]) * 4, 4, p.off_sc, 4), 14, it))
+          xs_s[gl * MPAD + mv[u]] = gs;
+      }
+      if (lane < 2 && WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)(2 * kbv[u] + lane) * MPAD + mv[u]) * 4, 4, p.off_slots, 4), 12, it))
+        sc_s[(2 * kbv[u] + lane) * MPAD + mv[u]] = exp2i(24 - (lane == 0 ? e0v[u] : e1v[u]));
+    }
   }
   for (int i = tid; i < nres; i += blockDim.x) {
     const int k = (i - tid) / (int)blockDim.x;
@@ -376,14 +471,18 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
             for (int q = 0; q < 4; ++q) ctot[pj][j][nt][q] = 0.f;
       for (int kb = ok ? kbs : kbe; kb < kbe; ++kb) {
         uint32_t b[8][NT][2];
-        float2 scv[NT];
+        float2 scv[2][NT];  // activation scales of the block's two halves
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
-          scv[nt] = make_float2(0.f, 0.f);
-          if (WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)kb * MPAD + col) * 4, 8, p.off_slots, 8), 18, col))
-            scv[nt] = *reinterpret_cast<const float2 *>(sc_s + kb * MPAD + col);
-        }
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
+            scv[h][nt] = make_float2(0.f, 0.f);
+            if ((HALF || h == 0) &&
+                WQ_OK_IF(WQ_RANGE(p.off_sc + ((size_t)(2 * kb + h) * MPAD + col) * 4, 8, p.off_slots, 8), 18, col))
+              scv[h][nt] = *reinterpret_cast<const float2 *>(sc_s + (2 * kb + h) * MPAD + col);
+            if (!HALF && h == 1) scv[1][nt] = scv[0][nt];
+          }
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
@@ -417,15 +516,62 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
               }
             }
           }
-        // Accumulation chains per (projection, tile): one, or two (even /
-        // odd k-steps) when a warp would otherwise run a single chain.  The
-        // first MMA of a chain in a group starts from zero.
-        constexpr int NCH = NPROJ * TPW >= 2 ? 1 : 2;
+        // Accumulation chains per (projection, tile): one, or (HALF) two, one
+        // per half of the block, issued alternately (k-steps 0,4,1,5,..).
+        // The first MMA of a chain in a group starts from zero.
+        constexpr int NCH = HALF ? 2 : 1;
+        constexpr int GH = GS < 4 ? GS : 4;  // k-steps of a group inside one chain (HALF)
         float acc[NCH][NPROJ][TPW][NT][4];
+        // per group: ctot += s * (sx * sum_k code * x' - z * sum_k x) for the
+        // chains (c0, c1) of the group, the affine dequantization s (q - z)
+        // with x' = x / sx (sx of the chain's half)
+        auto group_epi = [&](const int gl, const int c0, const int c1) {
+          float2 xs[NT];
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const int ch = NCH == 2 ? (ks & 1) : 0;
-          const bool first = (ks % GS) < NCH;  // first k-step of this chain in the group
+          for (int nt = 0; nt < NT; ++nt) {
+            const int col = tc * TOK + nt * 8 + 2 * (lane & 3);
+            xs[nt] = make_float2(0.f, 0.f);
+            if (WQ_OK_IF(WQ_RANGE(p.off_xs + ((size_t)gl * MPAD + col) * 4, 8, p.off_sc, 8), 14, gl))
+              xs[nt] = *reinterpret_cast<const float2 *>(xs_s + gl * MPAD + col);
+          }
+#pragma unroll
+          for (int pj = 0; pj < NPROJ; ++pj)
+#pragma unroll
+            for (int j = 0; j < TPW; ++j) {
+              const uint8_t *mp = mbase + pj * mproj + ((size_t)j * p.KP * GPB + gl) * 64;
+              uint2 sz = make_uint2(0u, 0u);
+              if (WQ_OK_IF(WQ_RANGE(mp - smem, 8, p.off_lorab, 8), 17, gl)) sz = lds64(mp);
+              const float s_lo = half_bits_to_float(sz.x), s_hi = half_bits_to_float(sz.x >> 16);
+              const float zs_lo = -s_lo * half_bits_to_float(sz.y), zs_hi = -s_hi * half_bits_to_float(sz.y >> 16);
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                float *ct = ctot[pj][j][nt];
+                const float2 sa = scv[c0][nt];
+                const float *ga = acc[c0][pj][j][nt];
+                ct[0] = fmaf(s_lo * sa.x, ga[0], ct[0]);
+                ct[1] = fmaf(s_lo * sa.y, ga[1], ct[1]);
+                ct[2] = fmaf(s_hi * sa.x, ga[2], ct[2]);
+                ct[3] = fmaf(s_hi * sa.y, ga[3], ct[3]);
+                if (c1 != c0) {
+                  const float2 sb = scv[c1][nt];
+                  const float *gb = acc[c1][pj][j][nt];
+                  ct[0] = fmaf(s_lo * sb.x, gb[0], ct[0]);
+                  ct[1] = fmaf(s_lo * sb.y, gb[1], ct[1]);
+                  ct[2] = fmaf(s_hi * sb.x, gb[2], ct[2]);
+                  ct[3] = fmaf(s_hi * sb.y, gb[3], ct[3]);
+                }
+                ct[0] = fmaf(zs_lo, xs[nt].x, ct[0]);
+                ct[1] = fmaf(zs_lo, xs[nt].y, ct[1]);
+                ct[2] = fmaf(zs_hi, xs[nt].x, ct[2]);
+                ct[3] = fmaf(zs_hi, xs[nt].y, ct[3]);
+              }
+            }
+        };
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int ks = NCH == 2 ? (i >> 1) + 4 * (i & 1) : i;
+          const int ch = NCH == 2 ? (i & 1) : 0;
+          const bool first = (ks % (NCH == 2 ? GH : GS)) == 0;  // first k-step of this chain in the group
 #pragma unroll
           for (int pj = 0; pj < NPROJ; ++pj)
 #pragma unroll
@@ -455,31 +601,12 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
                   mma_f16_16816(acc[ch][pj][j][nt], af, b[ks][nt][0], b[ks][nt][1]);
               }
             }
-          if ((ks + 1) % GS == 0) {
-            // per group: ctot += s * sx * sum_k code * x
-            const int gl = kb * GPB + ks / GS;
-#pragma unroll
-            for (int pj = 0; pj < NPROJ; ++pj)
-#pragma unroll
-              for (int j = 0; j < TPW; ++j) {
-                const uint8_t *mp = mbase + pj * mproj + ((size_t)j * p.KP * GPB + gl) * 64;
-                uint32_t sbits = 0u;
-                if (WQ_OK_IF(WQ_RANGE(mp - smem, 4, p.off_lorab, 4), 17, gl)) sbits = lds32(mp);
-                const float s_lo = half_bits_to_float(sbits), s_hi = half_bits_to_float(sbits >> 16);
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                  const float2 sc = scv[nt];
-                  float *ct = ctot[pj][j][nt];
-                  const float *g0 = acc[0][pj][j][nt];
-                  const float *g1 = acc[NCH - 1][pj][j][nt];
-                  const float a0 = NCH == 2 ? g0[0] + g1[0] : g0[0], a1 = NCH == 2 ? g0[1] + g1[1] : g0[1];
-                  const float a2 = NCH == 2 ? g0[2] + g1[2] : g0[2], a3 = NCH == 2 ? g0[3] + g1[3] : g0[3];
-                  ct[0] = fmaf(s_lo * sc.x, a0, ct[0]);
-                  ct[1] = fmaf(s_lo * sc.y, a1, ct[1]);
-                  ct[2] = fmaf(s_hi * sc.x, a2, ct[2]);
-                  ct[3] = fmaf(s_hi * sc.y, a3, ct[3]);
-                }
-              }
+          if (NCH == 1) {
+            if ((ks + 1) % GS == 0) group_epi(kb * GPB + ks / GS, 0, 0);
+          } else if (GS == 8) {
+            if (i == 7) group_epi(kb, 0, 1);  // a group spans both halves
+          } else if ((ks + 1) % GS == 0) {
+            group_epi(kb * GPB + ks / GS, ch, ch);
           }
         }
       }
@@ -507,40 +634,29 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
   }
   __syncthreads();
 
-  // ---- 5. reduce the k-split warps (fixed order) and add the zero-point
-  // term -sum_g s_g z_g sum_{k in g} x_k of this panel's groups ----
-  // Four lanes per output: each adds every 4th group, then the quad adds up
-  // (fixed order).
+  // ---- 5. add up the k-split warps' partial sums (fixed order) ----
   const int per_rt = NPROJ * 16 * M;
-  const int nel = nrt * per_rt, lim = (nel + 7) & ~7;  // equal trip counts for the quads of a warp
-  for (int i = tid >> 2; i < lim; i += blockDim.x >> 2) {
-    const int sub = tid & 3;
-    const bool live = i < nel;
-    float zt = 0.f, s = 0.f;
-    if (live) {
-      const int rti = i / per_rt, rem = i - rti * per_rt;
-      const int pj = rem / (16 * M), r16 = (rem / M) % 16, m = rem % M;
-      // meta of (row r16, group g): 32 halves per (tile, group), s at 4e + h, z at 4e + 2 + h
-      const size_t mrow = ((size_t)(pj * p.RB + rti) * p.KP * GPB) * 64 + (size_t)(4 * (r16 & 7) + (r16 >> 3)) * 2;
-      for (int g = sub; g < nkb * GPB; g += 4) {
-        const size_t mo = mrow + (size_t)g * 64;
-        if (WQ_OK_IF(WQ_RANGE(p.off_meta + mo, 6, p.off_lorab, 2), 40, g)) {
-          const uint16_t sb = *reinterpret_cast<const uint16_t *>(meta_s + mo);
-          const uint16_t zb = *reinterpret_cast<const uint16_t *>(meta_s + mo + 4);
-          zt = fmaf(half_bits_to_float(sb) * half_bits_to_float(zb), xs_s[g * MPAD + m], zt);
-        }
+  if (p.WK > 1) {
+    const int nel = nrt * per_rt;
+    const size_t wst = (size_t)p.RB * per_rt;  // slot stride between warps
+    for (int i = tid; i < nel; i += blockDim.x) {
+      if (!WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)(p.WK - 1) * wst + i) * 4, 4, p.off_red, 4), 21, i)) continue;
+      // four loads in flight, added in warp order
+      float s = 0.f;
+      int w = 0;
+      for (; w + 4 <= p.WK; w += 4) {
+        const float v0 = slot_s[w * wst + i], v1 = slot_s[(w + 1) * wst + i];
+        const float v2 = slot_s[(w + 2) * wst + i], v3 = slot_s[(w + 3) * wst + i];
+        s += v0;
+        s += v1;
+        s += v2;
+        s += v3;
       }
-      if (sub == 0)
-        for (int w = 0; w < p.WK; ++w)
-          if (WQ_OK_IF(WQ_RANGE(p.off_slots + ((size_t)w * p.RB * per_rt + i) * 4, 4, p.off_red, 4), 21, i))
-            s += slot_s[(size_t)w * p.RB * per_rt + i];
+      for (; w < p.WK; ++w) s += slot_s[w * wst + i];
+      slot_s[i] = s;
     }
-    zt += __shfl_xor_sync(0xffffffffu, zt, 1);
-    zt += __shfl_xor_sync(0xffffffffu, zt, 2);
-    __syncwarp();
-    if (live && sub == 0) slot_s[i] = s - zt;
+    __syncthreads();
   }
-  __syncthreads();
 
   if (p.P > 1) {
     for (int i = tid; i < nrt * per_rt; i += blockDim.x) {
@@ -575,9 +691,20 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
 
   // the tile partials summed over tiles: add the chunk sums (fixed order)
   if (use_tp && nchk > 1) {
+    const size_t cst = (size_t)M * Qp;  // stride between chunks
     for (int pair = tid; pair < M * Qp; pair += blockDim.x) {
+      // four loads in flight, added in chunk order
       float s = 0.f;
-      for (int c = 0; c < nchk; ++c) s += red_s[(size_t)c * M * Qp + pair];
+      int c = 0;
+      for (; c + 4 <= nchk; c += 4) {
+        const float v0 = red_s[c * cst + pair], v1 = red_s[(c + 1) * cst + pair];
+        const float v2 = red_s[(c + 2) * cst + pair], v3 = red_s[(c + 3) * cst + pair];
+        s += v0;
+        s += v1;
+        s += v2;
+        s += v3;
+      }
+      for (; c < nchk; ++c) s += red_s[c * cst + pair];
       if (WQ_OK_IF(WQ_RANGE(p.off_rt + (size_t)pair * 4, 4, p.off_yv, 4), 37, pair)) rt_s[pair] = s;
     }
     __syncthreads();
@@ -592,60 +719,113 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
 
   // ---- epilogue: RMSNorm scale, LoRA-B + SiLU(g) * u; or residual add ----
   const int rows = nrt * 16;
-  for (int i = tid; i < rows * M; i += blockDim.x) {
-    const int m = i / rows, rl = i % rows;
+  // gate/up output of local row rl, token m (before the bf16 store)
+  auto gateup_h = [&](int rl, int m) -> float {
     const int rti = rl >> 4, r16 = rl & 15;
-    if (!last_s[rti]) continue;
-    const int n = (rt0 + rti) * 16 + r16;
-    if (n >= a.N) continue;
-    const float v0 = slot_s[(size_t)(rti * NPROJ) * 16 * M + r16 * M + m];
-    if (NPROJ == 2) {
-      float g = v0;
-      float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * M + r16 * M + m];
-      // xin = x * rs (Sec. 3.3 MLP input after RMSNorm, never stored):
-      // g = rs * (x deq(Wg)^T + lora_scale * (x A_g^T) B_g^T)
-      const float rs = use_tp && a.prenorm ? rt_s[(size_t)m * Qp] : 1.f;
-      if (use_tp && r > 0) {
-        const float *tg = rt_s + (size_t)m * Qp + 1;
-        const float *tu = tg + r;
-        const __nv_bfloat16 *bg = lorab_s + (size_t)rl * r;
-        const __nv_bfloat16 *bu = lorab_s + ((size_t)p.RB * 16 + rl) * r;
-        float lg = 0.f, lu = 0.f;
-        const bool lora_ok =
-            WQ_OK_IF(WQ_RANGE(p.off_rt + ((size_t)m * Qp + Q) * 4 - 4, 4, p.off_yv, 4), 25, m) &&
-            WQ_OK_IF(WQ_RANGE(p.off_lorab + (((size_t)p.RB * 16 + rl) * r + r) * 2 - 16, 16, p.off_an, 16), 26, rl);
-        for (int q = 0; lora_ok && q < r; q += 8) {
-          float fg[8], fu[8];
-          unpack_bf16x8(lds128(bg + q), fg);
-          unpack_bf16x8(lds128(bu + q), fu);
+    float g = slot_s[(size_t)(rti * NPROJ) * 16 * M + r16 * M + m];
+    float u = slot_s[(size_t)(rti * NPROJ + 1) * 16 * M + r16 * M + m];
+    // xin = x * rs (Sec. 3.3 MLP input after RMSNorm, never stored):
+    // g = rs * (x deq(Wg)^T + lora_scale * (x A_g^T) B_g^T)
+    const float rs = use_tp && a.prenorm ? rt_s[(size_t)m * Qp] : 1.f;
+    if (use_tp && r > 0) {
+      const float *tg = rt_s + (size_t)m * Qp + 1;
+      const float *tu = tg + r;
+      const __nv_bfloat16 *bg = lorab_s + (size_t)rl * r;
+      const __nv_bfloat16 *bu = lorab_s + ((size_t)p.RB * 16 + rl) * r;
+      float lg = 0.f, lu = 0.f;
+      const bool lora_ok =
+          WQ_OK_IF(WQ_RANGE(p.off_rt + ((size_t)m * Qp + Q) * 4 - 4, 4, p.off_yv, 4), 25, m) &&
+          WQ_OK_IF(WQ_RANGE(p.off_lorab + (((size_t)p.RB * 16 + rl) * r + r) * 2 - 16, 16, p.off_an, 16), 26, rl);
+      for (int q = 0; lora_ok && q < r; q += 8) {
+        float fg[8], fu[8];
+        unpack_bf16x8(lds128(bg + q), fg);
+        unpack_bf16x8(lds128(bu + q), fu);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            lg = fmaf(tg[q + e], fg[e], lg);
-            lu = fmaf(tu[q + e], fu[e], lu);
-          }
+        for (int e = 0; e < 8; ++e) {
+          lg = fmaf(tg[q + e], fg[e], lg);
+          lu = fmaf(tu[q + e], fu[e], lu);
         }
-        g = fmaf(a.lora_scale, lg, g);
-        u = fmaf(a.lora_scale, lu, u);
       }
-      g *= rs;
-      u *= rs;
-      const float h = g / (1.f + __expf(-g)) * u;
-      if (WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_out, 2), 27, n))
-        reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(h);
-    } else {
-      float y = v0;
-      if (!WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * (a.out_f32 ? 4 : 2), a.out_f32 ? 4 : 2, a.nb_out, 2), 28, n))
-        continue;
-      if (a.residual) y += yv_s[(size_t)rl * MPAD + m];
-      if (a.out_f32) {
-        reinterpret_cast<float *>(a.out)[(size_t)m * a.N + n] = y;
+      g = fmaf(a.lora_scale, lg, g);
+      u = fmaf(a.lora_scale, lu, u);
+    }
+    g *= rs;
+    u *= rs;
+    return g / (1.f + __expf(-g)) * u;
+  };
+  if (NPROJ == 2 && a.hq_out != nullptr) {
+    // Decode chain (P = 1, RB a multiple of 4): h is also written as the
+    // down launch's binary16 panel.  A pair of warps per (token, 64-row
+    // half), one row a lane: each warp reduces its 32 rows (largest |h|, sum),
+    // the pair swaps maxima through shared memory behind a named barrier.
+    const int nhalf = p.RB / 4, npair = nwarps >> 1;
+    const int pair = warp >> 1, sub = warp & 1;
+    uint32_t *xch = reinterpret_cast<uint32_t *>(red_s);  // [2][npair][2], alternating by iteration
+    for (int item = pair, it = 0; item < nhalf * M; item += npair, ++it) {
+      const int m = item / nhalf, hh = item - m * nhalf;
+      const int rl = hh * 64 + sub * 32 + lane;
+      const int n = rt0 * 16 + rl;
+      float hv = 0.f;
+      if (n < a.N) {
+        const __nv_bfloat16 hb = __float2bfloat16_rn(gateup_h(rl, m));
+        if (WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_out, 2), 27, n))
+          reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = hb;
+        hv = __bfloat162float(hb);
+      }
+      const uint32_t mq = __reduce_max_sync(0xffffffffu, __float_as_uint(fabsf(hv)));
+      float sq = hv;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+      const int nq = rt0 * 16 + hh * 64 + sub * 32;  // first feature of this warp's 32
+      if (lane == 0) {
+        const int xi = ((it & 1) * npair + pair) * 2 + sub;
+        if (WQ_OK_IF(WQ_RANGE(p.off_red + (size_t)xi * 4, 4, p.off_rt, 4), 51, xi)) xch[xi] = mq;
+        if (nq < a.N && WQ_OK_IF(WQ_RANGE(((size_t)(nq >> 5) * M + m) * 4, 4, a.nb_hxs, 4), 52, nq))
+          a.hxs_out[(size_t)(nq >> 5) * M + m] = sq;
+      }
+      named_barrier_sync(1 + pair, 64);
+      const int xb = ((it & 1) * npair + pair) * 2;
+      const int e = block_exponent(max(xch[xb], xch[xb + 1]));
+      const int n0 = rt0 * 16 + hh * 64;
+      if (sub == 0 && lane == 0 && WQ_OK_IF(WQ_RANGE(((size_t)(n0 >> 6) * M + m) * 4, 4, a.nb_hsc, 4), 54, n0))
+        a.hsc_out[(size_t)(n0 >> 6) * M + m] = exp2i(24 - e);
+      if (n < a.N) {
+        // position in the B-fragment order of the 4-bit down kernel: k-step
+        // st, feature pair pr -> word 4((pr >> 1) & 1) + (pr >> 2) + 2(pr & 1);
+        // features 8..15 of a k-step scaled by 16^-1 (their code class)
+        const int st = (n >> 4) & 7, pr = (n & 15) >> 1;
+        const int w = 4 * ((pr >> 1) & 1) + (pr >> 2) + 2 * (pr & 1);
+        const size_t o = (size_t)m * a.hq_stride + (size_t)(n >> 7) * 128 + st * 16 + 2 * w + (n & 1);
+        const __half hq = __float2half_rn(hv * exp2i(e - 4 * ((n >> 3) & 1)));
+        if (WQ_OK_IF(WQ_RANGE(o * 2, 2, a.nb_hq, 2), 53, n)) a.hq_out[o] = __half_as_ushort(hq);
+      }
+    }
+  } else {
+    for (int i = tid; i < rows * M; i += blockDim.x) {
+      const int m = i / rows, rl = i % rows;
+      const int rti = rl >> 4, r16 = rl & 15;
+      if (!last_s[rti]) continue;
+      const int n = (rt0 + rti) * 16 + r16;
+      if (n >= a.N) continue;
+      if (NPROJ == 2) {
+        const float h = gateup_h(rl, m);
+        if (WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * 2, 2, a.nb_out, 2), 27, n))
+          reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = __float2bfloat16_rn(h);
       } else {
-        const __nv_bfloat16 yb = __float2bfloat16_rn(y);
-        reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = yb;
-        y = __bfloat162float(yb);
+        float y = slot_s[(size_t)(rti * NPROJ) * 16 * M + r16 * M + m];
+        if (!WQ_OK_IF(WQ_RANGE(((size_t)m * a.N + n) * (a.out_f32 ? 4 : 2), a.out_f32 ? 4 : 2, a.nb_out, 2), 28, n))
+          continue;
+        if (a.residual) y += yv_s[(size_t)rl * MPAD + m];
+        if (a.out_f32) {
+          reinterpret_cast<float *>(a.out)[(size_t)m * a.N + n] = y;
+        } else {
+          const __nv_bfloat16 yb = __float2bfloat16_rn(y);
+          reinterpret_cast<__nv_bfloat16 *>(a.out)[(size_t)m * a.N + n] = yb;
+          y = __bfloat162float(yb);
+        }
+        if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 38, rl))
+          yv_s[(size_t)rl * MPAD + m] = y;
       }
-      if (WQ_OK_IF(WQ_RANGE(p.off_yv + ((size_t)rl * MPAD + m) * 4, 4, p.off_bar, 4), 38, rl))
-        yv_s[(size_t)rl * MPAD + m] = y;
     }
   }
 
@@ -659,13 +839,18 @@ __global__ void __launch_bounds__(kMaxThreads, 1) qgemv_kernel(const GemvArgs a,
       const int m = rem / Qp, q = rem % Qp;
       if (!last_s[rti]) continue;
       const int tile = rt0 + rti;
-      float s = 0.f;
-      for (int r16 = 0; q < Q && r16 < 16 && tile * 16 + r16 < a.N; ++r16) {
+      const int nv = q < Q ? max(0, min(16, a.N - tile * 16)) : 0;  // rows of the tile inside the matrix
+      float vv[16], wv[16];
+#pragma unroll
+      for (int r16 = 0; r16 < 16; ++r16) {
         const int rl = rti * 16 + r16;
-        const float v = yv_s[(size_t)rl * MPAD + m];
-        const float w = q == 0 ? v : __bfloat162float(an_s[(size_t)(q - 1) * p.RB * 16 + rl]);
-        s = fmaf(w, v, s);
+        vv[r16] = yv_s[(size_t)rl * MPAD + m];
+        wv[r16] = q == 0 ? vv[r16] : (q < Q ? __bfloat162float(an_s[(size_t)(q - 1) * p.RB * 16 + rl]) : 0.f);
       }
+      float s = 0.f;
+#pragma unroll
+      for (int r16 = 0; r16 < 16; ++r16)
+        if (r16 < nv) s = fmaf(wv[r16], vv[r16], s);
       const size_t o = ((size_t)tile * M + m) * Qp + q;
       if (WQ_OK_IF(WQ_RANGE(o * 4, 4, a.nb_tp_out, 4), 35, o)) a.tp_out[o] = s;
     }
@@ -756,8 +941,8 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   off = align_up(off + (uint32_t)p->M * p->xstride * 2, 128);
   p->off_xs = off;
   off = align_up(off + (uint32_t)p->KP * GPB * p->MPAD * 4, 128);
-  p->off_sc = off;
-  off = align_up(off + (uint32_t)p->KP * p->MPAD * 4, 128);
+  p->off_sc = off;  // [2 KP][MPAD] half-block activation scales
+  off = align_up(off + (uint32_t)2 * p->KP * p->MPAD * 4, 128);
   p->off_slots = off;
   off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->M * 4, 128);
   p->off_red = off;
@@ -826,7 +1011,8 @@ bool search_plan(GemvKind kind, int N, int K, int M, int group, int r, int num_s
         // SM (HBM over the SMs), at most ~64 B/cycle into one SM.
         const double mma_cta = (double)RB * KP * nproj * 8.0 * NT * chunks;  // RB counts padded tiles
         const double eff = std::min(1.0, (double)warps * std::min(occ, per_sm) / 16.0);  // CTAs of an SM run together
-        const double t_mma = per_sm * mma_cta * 8.0 / 4.0 / eff;
+        const double imb = (double)((warps + 3) / 4 * 4) / warps;  // schedulers with one warp more than others
+        const double t_mma = per_sm * mma_cta * 8.0 / 4.0 * imb / eff;
         const double items = std::ceil((double)KP * M / warps);
         const double conv = 1500.0 + items * 250.0;
         const double epi = 3000.0 + (r > 0 ? 8.0 * r : 0.0) + std::ceil((double)RB * 16 * M / p.threads) * 20.0;

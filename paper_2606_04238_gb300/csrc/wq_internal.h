@@ -62,10 +62,26 @@ struct GemvArgs {
   int out_f32;
   const void *lora_a_next;   // bf16 [2r, N] (down with tp_out)
   float *tp_out;             // [ceil(N/16)][M][WQ_TP_STRIDE(r)] or null
+  // gate/up in the decode chain: the output h also as the down launch's
+  // ready-made binary16 panel (null otherwise; needs RB a multiple of 4):
+  //   hq_out  [M][hq_stride] binary16, per 16-feature k-step in the order of
+  //           the m16n8k16 B fragments, scaled by 2^e per (64 features,
+  //           token) and by 16^-1 on features 8..15 of every k-step (the
+  //           4-bit code class), e putting the largest |h| in [2^14, 2^15)
+  //   hsc_out [ceil(N/64)][M]  2^(24 - e)
+  //   hxs_out [ceil(N/32)][M]  sum of h over 32 features (zero-point term)
+  uint16_t *hq_out;
+  float *hsc_out, *hxs_out;
+  int hq_stride;
+  // down: that panel instead of converting act (null: convert act)
+  const uint16_t *pre_x;
+  const float *pre_sc, *pre_xs;
+  int pre_stride;
   float *partials;           // [RT][P][NPROJ][16][M] fp32 (P > 1)
   unsigned *counters;        // [RT] arrival counters, zero between calls
   // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
   size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_tp, nb_res, nb_out, nb_an, nb_tp_out, nb_part, nb_cnt;
+  size_t nb_hq, nb_hsc, nb_hxs, nb_pre_x, nb_pre_sc, nb_pre_xs;
 };
 
 enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
