@@ -92,6 +92,21 @@ __device__ __forceinline__ uint32_t pack_half2(float a, float b) {
 // 2^k for -126 <= k <= 127, built from the binary32 exponent field
 __device__ __forceinline__ float exp2i(int k) { return __int_as_float((k + 127) << 23); }
 
+// sum_{i < n} base[i * stride] from L2, added in index order, eight loads in
+// flight at a time (the partial sums of split work).
+__device__ __forceinline__ float sum_strided_cg(const float *base, size_t stride, int n) {
+  float s = 0.f;
+  for (int i0 = 0; i0 < n; i0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = i0 + u < n ? ldcg_f32(base + (size_t)(i0 + u) * stride) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (i0 + u < n) s += v[u];
+  }
+  return s;
+}
+
 // Scale exponent e of a block whose largest |x| has the bit pattern mxb:
 // 2^e puts it in [2^14, 2^15).  mx = f 2^E with f in [0.5, 1) and E = (biased
 // exponent) - 126, so e = 15 - E, clamped (subnormal mx: 100); 0 for a zero,
@@ -144,7 +159,7 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
   uint8_t *codes_s = smem + p.off_codes;
   uint8_t *meta_s = smem + p.off_meta;
   const __nv_bfloat16 *lorab_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_lorab);  // [NPROJ][RB*16][r]
-  const __nv_bfloat16 *an_s = reinterpret_cast<const __nv_bfloat16 *>(smem + p.off_an);        // [2r][RB*16]
+  __nv_bfloat16 *an_s = reinterpret_cast<__nv_bfloat16 *>(smem + p.off_an);                    // [RB*16][2r]
   __half *xp_s = reinterpret_cast<__half *>(smem + p.off_xp);
   float *xs_s = reinterpret_cast<float *>(smem + p.off_xs);    // [KP*GPB][MPAD] group sums of x
   float *sc_s = reinterpret_cast<float *>(smem + p.off_sc);    // [2 KP][MPAD] half-block scales 2^(24-e)
@@ -204,18 +219,25 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
       if (WQ_OK_IF(WQ_RANGE(dst, 16, p.off_an, 16), 31, i)) *reinterpret_cast<uint4 *>(smem + dst) = v;
     }
   }
-  // The next layer's LoRA-A columns for this CTA's output rows (down writing tile partials).
+  // The next layer's LoRA-A columns for this CTA's output rows (down writing
+  // tile partials), transposed to [row][2r]: the tile-partial loop reads the
+  // 2r values of a row from consecutive addresses (no bank conflicts).
   if (NPROJ == 1 && a.tp_out != nullptr && r > 0) {
     const int per = nrt * 2;  // 16-byte chunks per LoRA-A row (16 columns a tile)
     for (int i = tid; i < 2 * r * per; i += blockDim.x) {
-      const int j = i / per, c = i % per;
+      const int j = i % (2 * r), c = i / (2 * r);
       const int col = rt0 * 16 + c * 8;
       uint4 v = make_uint4(0u, 0u, 0u, 0u);
       const size_t src = ((size_t)j * a.N + col) * 2;
       if (col + 8 <= a.N && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_an, 16), 32, i))
         v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_a_next) + src));
-      const size_t dst = p.off_an + ((size_t)j * p.RB * 16 + (size_t)c * 8) * 2;
-      if (WQ_OK_IF(WQ_RANGE(dst, 16, p.off_xp, 16), 33, i)) *reinterpret_cast<uint4 *>(smem + dst) = v;
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const size_t e = (size_t)(c * 8 + t) * 2 * r + j;
+        if (WQ_OK_IF(WQ_RANGE(p.off_an + e * 2, 2, p.off_xp, 2), 33, i))
+          an_s[e] = __ushort_as_bfloat16(static_cast<unsigned short>(w[t >> 1] >> (16 * (t & 1))));
+      }
     }
   }
   for (int i = tid; i < nkb * GPB * MPAD; i += blockDim.x) xs_s[i] = 0.f;
@@ -369,9 +391,10 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
   // every scaled bf16 value exactly (bf16 has 8 significant bits), far from
   // overflow.  Lane L holds features 4L..4L+3 of the block, i.e. k-step L/4,
   // and writes them in the order the B fragments read them.
-  // Items it0 + u * nwarps (u < CU) are converted together: independent
+  // A warp converts CU consecutive (block, token) items together -- the
+  // tokens of a block, or consecutive blocks of one token: independent
   // dependency chains (load, max reduction, shuffles) in flight at once.
-  constexpr int CU = 2;
+  constexpr int CU = NPROJ == 2 ? 4 : 2;  // fewer for the down kernel (64 registers)
   const int nitems = pre ? 0 : nkb * M;
   const int st = lane >> 2, hi = (lane >> 1) & 1;
   // bit-position class of the codes that meet these features: 4^c for 2-bit
@@ -380,12 +403,12 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
   const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
   const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
   const bool lo_half = lane < 16;      // features 0..63 of the block
-  for (int it0 = warp; it0 < nitems; it0 += CU * nwarps) {
+  for (int it0 = warp * CU; it0 < nitems; it0 += CU * nwarps) {
     float f[CU][4];
     int kbv[CU], mv[CU], e0v[CU], e1v[CU];
 #pragma unroll
     for (int u = 0; u < CU; ++u) {
-      const int it = it0 + u * nwarps;  // warp-uniform
+      const int it = it0 + u;  // warp-uniform
       kbv[u] = M == 1 ? it : it / M;
       mv[u] = M == 1 ? 0 : it - kbv[u] * M;
       uint2 raw = make_uint2(0u, 0u);
@@ -411,7 +434,7 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
     __syncwarp();  // every lane has read its raw features before the blocks are overwritten
 #pragma unroll
     for (int u = 0; u < CU; ++u) {
-      const int it = it0 + u * nwarps;
+      const int it = it0 + u;
       if (it >= nitems) break;  // warp-uniform
       const float mul = exp2i((lo_half ? e0v[u] : e1v[u]) - sh);
       uint32_t *slot = reinterpret_cast<uint32_t *>(xp_s + (size_t)mv[u] * p.xstride + (size_t)kbv[u] * 128 + st * 16);
@@ -677,9 +700,8 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
       if (!last_s[rti]) continue;
       const float *src = a.partials + (size_t)(rt0 + rti) * p.P * per_rt + rem;
       float s = 0.f;
-      for (int pp = 0; pp < p.P; ++pp)
-        if (WQ_OK_IF(WQ_RANGE((src - a.partials + (size_t)pp * per_rt) * 4, 4, a.nb_part, 4), 24, pp))
-          s += ldcg_f32(src + (size_t)pp * per_rt);
+      if (WQ_OK_IF(WQ_RANGE((src - a.partials + (size_t)(p.P - 1) * per_rt) * 4, 4, a.nb_part, 4), 24, i))
+        s = sum_strided_cg(src, per_rt, p.P);
       slot_s[i] = s;
     }
     if (tid < nrt && last_s[tid]) a.counters[rt0 + tid] = 0u;
@@ -845,7 +867,7 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
       for (int r16 = 0; r16 < 16; ++r16) {
         const int rl = rti * 16 + r16;
         vv[r16] = yv_s[(size_t)rl * MPAD + m];
-        wv[r16] = q == 0 ? vv[r16] : (q < Q ? __bfloat162float(an_s[(size_t)(q - 1) * p.RB * 16 + rl]) : 0.f);
+        wv[r16] = q == 0 ? vv[r16] : (q < Q ? __bfloat162float(an_s[(size_t)rl * 2 * r + (q - 1)]) : 0.f);
       }
       float s = 0.f;
 #pragma unroll
@@ -945,8 +967,13 @@ void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   off = align_up(off + (uint32_t)2 * p->KP * p->MPAD * 4, 128);
   p->off_slots = off;
   off = align_up(off + (uint32_t)p->WK * p->RB * nproj * 16 * p->M * 4, 128);
-  p->off_red = off;
-  off = align_up(off + (nproj == 2 ? (uint32_t)p->threads * 16 : 0u), 128);
+  p->off_red = off;  // gate/up: chunk sums of the tile partials [nchk][M][Qp], or the panel epilogue's maxima
+  {
+    const int Qp = WQ_TP_STRIDE(r);
+    const int nchk = std::max(1, std::min(4 * p->threads / (p->M * Qp), p->KB));
+    const uint32_t red = (uint32_t)std::max(nchk * p->M * Qp, 4 * (p->threads / 64) + 4) * 4;
+    off = align_up(off + (nproj == 2 ? red : 0u), 128);
+  }
   p->off_rt = off;
   off = align_up(off + (nproj == 2 ? (uint32_t)p->M * WQ_TP_STRIDE(r) * 4 : 0u), 128);
   p->off_yv = off;
