@@ -66,7 +66,9 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
 
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
-  size_t cnt1, cnt2, tp, xa, xb, h, hq, hsc, hxs, part1, part2, total;
+  size_t cnt1, cnt2, tp, xa, xb, h, hq, hsc, hxs, part1, part2;
+  size_t x16, rs, ta, h16;  // dequant-GEMM path (m > kMaxTokens)
+  size_t total;
 };
 
 size_t up256(size_t v) { return (v + 255) / 256 * 256; }
@@ -100,6 +102,22 @@ bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2) {
 // The arrival counters come first: their offsets depend on (d, inter) only,
 // so a workspace zeroed once stays valid for every token count.
 bool ws_layout(int m, int d, int inter, WsLayout *L) {
+  *L = WsLayout{};
+  if (m > kMaxTokens) {
+    // dequant-GEMM path: binary16 copies of the GEMM inputs, the RMSNorm
+    // scales and the LoRA-A products, and the stack's bf16 intermediates
+    const size_t lda = (size_t)(std::max(d, inter) + 127) / 128 * 128, ldi = (size_t)(inter + 127) / 128 * 128;
+    size_t off = 0;
+    L->xa = off;  off = up256(off + (size_t)m * d * 2);
+    L->xb = off;  off = up256(off + (size_t)m * d * 2);
+    L->h = off;   off = up256(off + (size_t)m * inter * 2);
+    L->x16 = off; off = up256(off + (size_t)m * lda * 2);
+    L->rs = off;  off = up256(off + (size_t)m * 4);
+    L->ta = off;  off = up256(off + (size_t)m * 2 * kMaxRank * 2);
+    L->h16 = off; off = up256(off + (size_t)m * ldi * 2);
+    L->total = off;
+    return true;
+  }
   size_t p1, p2;
   if (!max_partials(m, d, inter, &p1, &p2)) return false;
   size_t off = 0;
@@ -236,6 +254,71 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   return WQ_OK;
 }
 
+// ---- dequant-GEMM path (m > kMaxTokens): tcgen05 tensor cores ----
+// gate/up: binary16 copy of x, RMSNorm scales and lora_scale * x A^T first,
+// then the GEMM (h in bf16, and in binary16 at h16 for the down GEMM when
+// h16 is not null).
+wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                          const void *lora_a, const void *lora_bg, const void *lora_bu, int r, float lora_scale,
+                          unsigned flags, void *h, uint16_t *h16, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+  const int d = gate->k, inter = gate->n;
+  const int lda = (d + 127) / 128 * 128;
+  uint16_t *x16 = reinterpret_cast<uint16_t *>(ws + L.x16);
+  float *rs = reinterpret_cast<float *>(ws + L.rs);
+  uint16_t *ta = reinterpret_cast<uint16_t *>(ws + L.ta);
+  cudaError_t e = launch_gemm_prep(x, m, d, lda, r > 0 ? lora_a : nullptr, r > 0 ? 2 * r : 0, lora_scale, x16, rs, ta, s);
+  if (e != cudaSuccess) return cuda_fail(e, "GEMM input launch");
+  GemmArgs a = {};
+  a.act = x16;
+  a.lda = lda;
+  a.M = m;
+  a.N = inter;
+  a.K = d;
+  a.group = gate->group;
+  a.codes[0] = gate->codes;
+  a.codes[1] = up->codes;
+  a.meta[0] = gate->meta;
+  a.meta[1] = up->meta;
+  a.ta = r > 0 ? ta : nullptr;
+  a.r = r;
+  a.lora_b[0] = lora_bg;
+  a.lora_b[1] = lora_bu;
+  a.rs = (flags & WQ_PRENORM) ? rs : nullptr;
+  a.out = h;
+  a.out_f16 = h16;
+  a.ldo16 = (inter + 127) / 128 * 128;
+  e = launch_gemm(kind, a, s);
+  if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
+  return WQ_OK;
+}
+
+// down: from the binary16 h16 (null: converted from the bf16 h first).
+wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qweight *down, const void *residual,
+                        void *y, int y_f32, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+  const int K = down->k, lda = (K + 127) / 128 * 128;
+  if (!h16) {
+    uint16_t *c = reinterpret_cast<uint16_t *>(ws + L.h16);
+    cudaError_t e = launch_to_f16(h, m, K, lda, c, s);
+    if (e != cudaSuccess) return cuda_fail(e, "GEMM input launch");
+    h16 = c;
+  }
+  GemmArgs a = {};
+  a.act = h16;
+  a.lda = lda;
+  a.M = m;
+  a.N = down->n;
+  a.K = K;
+  a.group = down->group;
+  a.codes[0] = down->codes;
+  a.meta[0] = down->meta;
+  a.residual = residual;
+  a.out = y;
+  a.out_f32 = y_f32;
+  cudaError_t e = launch_gemm(kDownW4, a, s);
+  if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
+  return WQ_OK;
+}
+
 // The gate/up launch can hand the down launch a ready binary16 panel when it
 // holds whole 64-feature halves (one panel, row blocks of a multiple of 4
 // tiles) and the down kernel scales its input per half (one row tile a warp).
@@ -248,7 +331,7 @@ bool chain_panel_ok(GemvKind kind, int m, const wq_qweight &gate, int r, const w
 
 wq_status check_tokens(int m) {
   if (m < 0) return fail(WQ_ERR_ARG, "m=%d is negative", m);
-  if (m > kMaxTokens) return fail(WQ_ERR_UNSUPPORTED, "m=%d exceeds the %d-token limit of this build", m, kMaxTokens);
+  if (m > kMaxGemmTokens) return fail(WQ_ERR_UNSUPPORTED, "m=%d exceeds the %d-token limit of this build", m, kMaxGemmTokens);
   return WQ_OK;
 }
 
@@ -292,8 +375,12 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, gate->k, gate->n, &L)) != WQ_OK) return st;
-  st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
-                  static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
+  if (m > kMaxTokens)
+    st = run_gateup_gemm(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
+                         static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
+  else
+    st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
+                    static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
   return st == WQ_OK ? ok() : st;
 }
 
@@ -339,9 +426,14 @@ wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, i
 
 size_t wq_workspace_bytes(int m, int d, int inter, int r) {
   (void)r;  // the LoRA-A product area is sized for the largest supported rank
-  if (m <= 0 || d <= 0 || inter <= 0 || m > kMaxTokens) return 0;
+  if (m <= 0 || d <= 0 || inter <= 0 || m > kMaxGemmTokens) return 0;
   size_t most = 0;  // enough for every token count up to m
-  for (int mm = 1; mm <= m; ++mm) {
+  if (m > kMaxTokens) {
+    WsLayout L;
+    if (!ws_layout(m, d, inter, &L)) return 0;  // grows with m
+    most = L.total;
+  }
+  for (int mm = 1; mm <= std::min(m, kMaxTokens); ++mm) {
     WsLayout L;
     if (!ws_layout(mm, d, inter, &L)) return 0;
     most = std::max(most, L.total);
@@ -405,6 +497,9 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
   if (m == 0) return ok();
   if (!x || !h) return fail(WQ_ERR_ARG, "null x or h");
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
+  if (m > kMaxTokens)
+    return fail(WQ_ERR_UNSUPPORTED, "m=%d: the built-in scratch serves the decode path (m <= %d; use wq_gateup_w2_lora)",
+                m, kMaxTokens);
   WsLayout L;
   if (!ws_layout(m, gate->k, gate->n, &L)) return fail(WQ_ERR_CUDA, "cannot query the current device");
   if (L.total > (size_t)WQ_NOALLOC_SCRATCH_BYTES)
@@ -438,8 +533,12 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
     return fail(WQ_ERR_ALIGN, "h, y or residual not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, down->n, down->k, &L)) != WQ_OK) return st;
-  st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, nullptr, 0, nullptr, L, static_cast<uint8_t *>(ws),
-                static_cast<cudaStream_t>(stream));
+  if (m > kMaxTokens)
+    st = run_down_gemm(h, nullptr, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
+                       static_cast<cudaStream_t>(stream));
+  else
+    st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, nullptr, 0, nullptr, L, static_cast<uint8_t *>(ws),
+                  static_cast<cudaStream_t>(stream));
   return st == WQ_OK ? ok() : st;
 }
 
@@ -481,6 +580,24 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
   if ((st = check_ws(ws, ws_bytes, m, d, inter, &L)) != WQ_OK) return st;
   uint8_t *w8 = static_cast<uint8_t *>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (m > kMaxTokens) {
+    // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up (h also in
+    // binary16), down with the residual
+    const void *cur = x;
+    for (int l = 0; l < n_layers; ++l) {
+      const wq_mlp_layer &Ly = layers[l];
+      void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
+      const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+      uint16_t *h16 = reinterpret_cast<uint16_t *>(w8 + L.h16);
+      st = run_gateup_gemm(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale,
+                           flags, w8 + L.h, h16, L, w8, s);
+      if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+      st = run_down_gemm(nullptr, h16, m, &Ly.down, cur, out, 0, L, w8, s);
+      if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+      cur = out;
+    }
+    return ok();
+  }
   const bool prenorm = (flags & WQ_PRENORM) != 0;
   float *tp = reinterpret_cast<float *>(w8 + L.tp);
   // Launch chain (programmatic dependent launch throughout): the first
@@ -540,6 +657,10 @@ wq_status wq_device_status(int *status) {
   if (!status) return fail(WQ_ERR_ARG, "null status pointer");
   cudaError_t e = read_device_status(status);
   if (e != cudaSuccess) return cuda_fail(e, "device status read");
+  int g = 0;
+  e = read_gemm_status(&g);
+  if (e != cudaSuccess) return cuda_fail(e, "device status read");
+  if (*status == 0) *status = g;
   return ok();
 }
 

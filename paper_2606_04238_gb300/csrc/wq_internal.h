@@ -10,6 +10,7 @@
 namespace wq {
 
 constexpr int kMaxTokens = 64;      // tokens per call on the dequant-GEMV path
+constexpr int kMaxGemmTokens = 16384;  // tokens per call on the dequant-GEMM path (above kMaxTokens)
 constexpr int kMaxRank = 64;        // LoRA rank limit
 constexpr float kRmsEps = 1e-6f;    // RMSNorm epsilon of WQ_PRENORM
 
@@ -85,6 +86,33 @@ struct GemvArgs {
 };
 
 enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
+
+// Batched (prefill-size) dequant-GEMM on the tcgen05 tensor cores (wq_gemm.cu).
+struct GemmArgs {
+  const uint16_t *act;       // binary16 activations [M][lda] (zero padded to whole 128-feature blocks)
+  int lda;
+  int M, N, K, group;
+  const uint32_t *codes[2];  // packed codes (gate, up) or (down)
+  const uint16_t *meta[2];
+  const uint16_t *ta;        // gate/up with LoRA: binary16 [M][2r] = lora_scale * x A^T (gate rows, up rows)
+  int r;
+  const void *lora_b[2];     // bf16 [N][r]
+  const float *rs;           // gate/up: RMSNorm scale per token, or null
+  const void *residual;      // down: bf16 [M][N] or null
+  void *out;                 // bf16 (or fp32 for down with out_f32) [M][N]
+  int out_f32;
+  uint16_t *out_f16;         // gate/up: h also as binary16 [M][ldo16] (the down GEMM's A), or null
+  int ldo16;
+};
+cudaError_t launch_gemm(GemvKind kind, const GemmArgs &args, cudaStream_t stream);
+// x16 [M][lda16] = binary16(x), rs[m] = 1/sqrt(mean(x^2) + eps), ta [M][r2] = lora_scale * x A^T (r2 > 0)
+cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void *lora_a, int r2, float lora_scale,
+                             uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t stream);
+// x16 [M][lda16] = binary16(x) (zero padded)
+cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, cudaStream_t stream);
+int gemm_stages(GemvKind kind, int group);
+// Reads and clears the GEMM kernels' device status word.
+cudaError_t read_gemm_status(int *status);
 
 // Plans a launch (memoized); returns false if no configuration fits.
 // r: LoRA rank read by the launch (gate/up: its adapter; down: the next

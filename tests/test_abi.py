@@ -67,7 +67,7 @@ def test_gateup_host_validation(wq):
                                    ctypes.c_void_p(h), ctypes.c_void_p(16), 1 << 20, None)
 
     assert call(x, -1, ok_g, ok_u) == -1                                   # negative m
-    assert call(x, 65, ok_g, ok_u) == -4                                   # beyond the token limit
+    assert call(x, 16385, ok_g, ok_u) == -4                                # beyond the token limit
     assert call(x, 1, _qw(wq, 64, 256, 64, 4), ok_u) == -2                 # wrong bit width
     assert call(x, 1, ok_g, _qw(wq, 32, 256, 64, 2)) == -2                 # gate / up differ
     assert call(x, 1, _qw(wq, 64, 200, 64, 2), _qw(wq, 64, 200, 64, 2)) == -2  # k % group
