@@ -9,19 +9,25 @@
 //     (the unmerged LoRA path of Eq. 1 enters as two more k-steps), then
 //     h = SiLU(rs D_g) * (rs D_u) with rs the RMSNorm scale of the token;
 //   * down: y = residual + h deq(Wd)^T.
-// A CTA computes a tile of 128 tokens x 128 output rows (x 2 projections for
-// gate/up) over the whole feature axis, 64 features (half a block of the
-// packed format) per pipeline stage.  Warp roles:
+// A CTA computes a tile of 128 or 256 tokens x 128 output rows (x 2
+// projections for gate/up) over the whole feature axis, 64 features (half a
+// block of the packed format) per pipeline stage; with 256 tokens the two
+// halves of 128 multiply the same dequantized B tile into accumulators of
+// their own, so each weight is dequantized once per 256 tokens.  Warp roles:
 //   warps 0..15 dequantize the stage's codes: code q of row n, group j gives
 //               the binary16 value s_nj (q - z_nj), rounded once; they write
 //               it in the tcgen05 K-major layout (8-row x 16-byte core
-//               matrices), warps 0..3 then run the epilogue from TMEM;
+//               matrices), then run the epilogue from TMEM;
 //   warp 16     loads the binary16 activation tile with the tensor-memory
-//               accelerator (TMA; zero fill outside the matrix);
+//               accelerator (TMA; one box of 64 features x 128 tokens in the
+//               128-byte swizzled layout, zero fill outside the matrix);
 //   warp 17     owns the TMEM allocation; its lane 0 issues the MMAs;
 //   warp 18     loads the packed codes and scales/zeros of the CTA's 8 row
-//               tiles (TMA, one box each per projection and stage) into their
-//               own ring, which runs a stage further ahead than the tiles.
+//               tiles (TMA, one box each per projection and block) into their
+//               own ring.
+// The activation tiles, the B tiles and the packed codes have rings of their
+// own depths: each slot is released by what last reads it (the MMAs' commit,
+// or the dequantizing warps for the codes).
 // Stages are handed over with mbarriers; every wait is bounded (a timeout
 // sets the device status word and the CTA skips the rest of its work).
 #include <algorithm>
@@ -49,6 +55,7 @@ constexpr int kMmaWarp = kDeqWarps + 1;          // TMEM owner and MMA issuer
 constexpr int kRawWarp = kDeqWarps + 2;          // packed-code ring
 constexpr int kGemmThreads = (kDeqWarps + 3) * 32;
 constexpr int kTileBytes = kBM * 64 * 2;         // one 128 x 64 binary16 operand tile (a stage)
+constexpr int kHalves = 2;                       // token halves of kBM a CTA can take (GemmArgs::mt)
 constexpr uint32_t kSboTile = 8 * 128;           // bytes between 8-row groups of a 64-feature B tile
 constexpr int kLoraK = 32;                       // LoRA rank columns a stage
 constexpr uint32_t kGemmSmemLimit = 232448;      // 227 KB opt-in
@@ -66,19 +73,25 @@ struct GemmCfg {
   static constexpr int RAW_TILE = BPK + GPB * 64;          // codes + scales/zeros of a (tile, block)
   static constexpr int RAWP = 8 * RAW_TILE;                // a projection's: [8 tiles][codes], then [8 tiles][meta]
   static constexpr int RAW = NPROJ * RAWP;                 // a block's packed weights (two stages)
-  static constexpr int TILES = kTileBytes + NB * kTileBytes;  // a stage's operand tiles
-  static constexpr int AVAIL = (int)kGemmSmemLimit - 1024;
-  // stages: as many as leave room for two blocks of packed codes, at most 4;
-  // code ring: the rest, at most 4 blocks
-  static constexpr int S = std::min(4, (AVAIL - 2 * RAW) / TILES);
-  static constexpr int R = std::min(4, (AVAIL - S * TILES) / RAW);
-  static_assert(S >= 2 && R >= 2, "GEMM pipeline does not fit");
+  static constexpr int BT = NB * kTileBytes;               // a stage's B tiles
+  static constexpr int AT = kHalves * kTileBytes;          // a stage's activation tiles (both token halves)
+  // 1 KB for the barriers, 1 KB to align the tiles on 1024 bytes
+  static constexpr int AVAIL = (int)kGemmSmemLimit - 2048;
+  // Three rings.  The activation tiles come from L2 with a long latency, so
+  // their ring is the deepest (up to 8 stages); the B tiles are made on chip
+  // and need only 3 (2 where 3 would leave fewer than 4 activation stages);
+  // the packed codes (blocks of two stages) take what is left, at most 6.
+  static constexpr int SB = (AVAIL - 3 * BT - 3 * RAW) / AT >= 4 ? 3 : 2;
+  static constexpr int SA = std::min(8, (AVAIL - SB * BT - 3 * RAW) / AT);
+  static constexpr int R = std::min(6, (AVAIL - SA * AT - SB * BT) / RAW);
+  static_assert(SA >= 2 && R >= 2, "GEMM pipeline does not fit");
   static constexpr int OFF_A = 0;
-  static constexpr int OFF_B = S * kTileBytes;
-  static constexpr int OFF_RAW = OFF_B + S * NB * kTileBytes;
-  static constexpr int OFF_BAR = OFF_RAW + R * RAW;        // 3 S + 2 R + 1 barriers
-  static constexpr int SMEM = OFF_BAR + (3 * S + 2 * R + 2) * 8 + 16;
-  static constexpr int NCOLS = NPROJ == 2 ? 256 : 128;     // TMEM columns (fp32 accumulators)
+  static constexpr int OFF_B = SA * AT;
+  static constexpr int OFF_RAW = OFF_B + SB * BT;
+  static constexpr int OFF_BAR = OFF_RAW + R * RAW;
+  static constexpr int SMEM = OFF_BAR + (2 * SA + 2 * SB + 2 * R + 2) * 8 + 16 + 1024;  // + alignment slack
+  static constexpr int NCH = NPROJ * kBN;                  // TMEM columns of a token half (fp32 accumulators)
+  static constexpr int NCOLS = kHalves * NCH;
   static_assert(SMEM <= (int)kGemmSmemLimit, "GEMM stage does not fit");
 };
 
@@ -110,7 +123,7 @@ __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, i
 }
 
 // 2-D TMA load of a box of the activations into shared memory, completing
-// on `bar` with its byte count.  x (the feature coordinate) is a multiple of 8.
+// on `bar` with its byte count.  x (the feature coordinate) is a multiple of 64.
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -122,19 +135,23 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
 template <int BITS, int NPROJ, int GROUP, bool EXACT>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a, const __grid_constant__ GemmMaps tm) {
   using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
-  constexpr int S = C::S, R = C::R, GPB = C::GPB, GS = GROUP / 16;
-  extern __shared__ __align__(1024) uint8_t smem[];
+  constexpr int SA = C::SA, SB = C::SB, R = C::R, GPB = C::GPB, GS = GROUP / 16;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // the swizzled activation tiles need 1024-byte alignment
+  uint8_t *smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
   uint64_t *raw_full = reinterpret_cast<uint64_t *>(smem + C::OFF_BAR);
   uint64_t *raw_empty = raw_full + R;
   uint64_t *a_full = raw_empty + R;
-  uint64_t *b_full = a_full + S;
-  uint64_t *empty = b_full + S;
-  uint64_t *acc_full = empty + S;
+  uint64_t *a_empty = a_full + SA;
+  uint64_t *b_full = a_empty + SA;
+  uint64_t *b_empty = b_full + SB;
+  uint64_t *acc_full = b_empty + SB;
   uint32_t *tmem_s = reinterpret_cast<uint32_t *>(acc_full + 2);
   volatile int *abort_s = reinterpret_cast<volatile int *>(tmem_s + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * kBN;
+  const int m0 = blockIdx.x * a.mt * kBM, n0 = blockIdx.y * kBN;
+  const int mth = min(a.mt, (a.M - m0 + kBM - 1) / kBM);  // token halves with tokens in them
   const int KB = (a.K + 127) / 128;
   const int nws = 2 * KB;  // weight stages (64 features each)
   const int nlora = NPROJ == 2 && a.r > 0 ? (a.r + kLoraK - 1) / kLoraK : 0;
@@ -145,10 +162,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       mbar_init(&raw_full[q], 1);
       mbar_init(&raw_empty[q], kDeqWarps);
     }
-    for (int s = 0; s < S; ++s) {
+    for (int s = 0; s < SA; ++s) {
       mbar_init(&a_full[s], 1);
+      mbar_init(&a_empty[s], 1);
+    }
+    for (int s = 0; s < SB; ++s) {
       mbar_init(&b_full[s], kDeqWarps);
-      mbar_init(&empty[s], 1);
+      mbar_init(&b_empty[s], 1);
     }
     mbar_init(acc_full, 1);
     *abort_s = 0;
@@ -163,7 +183,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   // bounded wait; a timeout (or an earlier one) makes the caller skip its work
   auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
     if (*abort_s) return false;
-    if (mbar_wait(bar, parity)) return true;
+    if (mbar_wait_sleep(bar, parity)) return true;
     *abort_s = 1;
     if (lane == 0) gemm_timeout();
     return false;
@@ -187,28 +207,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else if (warp == kProducerWarp) {
     // ---- activation tiles (TMA); the LoRA stage's by cp.async ----
     for (int it = 0; it < nit; ++it) {
-      const int s = it % S, u = it / S;
-      if (it >= S && !wait(&empty[s], (u - 1) & 1)) break;
-      uint8_t *As = smem + C::OFF_A + s * kTileBytes;
+      const int s = it % SA;
+      if (it >= SA && !wait(&a_empty[s], (it / SA - 1) & 1)) break;
+      uint8_t *As = smem + C::OFF_A + s * C::AT;
       if (it < nws) {
         if (lane == 0) {
-          // activation tile: 8 boxes of 8 features x 128 tokens, box c landing
-          // at c * 2 KB (K-major: core matrices 2 KB apart along K, 8-row
-          // groups 128 bytes apart)
-          mbar_arrive_expect_tx(&a_full[s], (uint32_t)kTileBytes);
-          for (int c = 0; c < 8; ++c) tma_load_2d(As + c * 2048, &tm.act, it * 64 + c * 8, m0, &a_full[s]);
+          // activation tiles: per token half one box of 64 features x 128
+          // tokens, a 128-byte row per token, swizzled (8-row groups 1 KB apart)
+          mbar_arrive_expect_tx(&a_full[s], (uint32_t)(mth * kTileBytes));
+          for (int h = 0; h < mth; ++h) tma_load_2d(As + h * kTileBytes, &tm.act, it * 64, m0 + h * kBM, &a_full[s]);
         }
       } else {
         // LoRA stage l: lora_scale * t, rank columns 32 l .. 32 l + 31 of gate
         // (first r columns of ta) and of up (next r), zeros past r
         const int l = it - nws;
-        for (int i = lane; i < NPROJ * kBM * 4; i += 32) {
-          const int p = i / (kBM * 4), rem = i - p * kBM * 4;
+        for (int i = lane; i < mth * NPROJ * kBM * 4; i += 32) {
+          const int h = i / (NPROJ * kBM * 4), hr = i - h * NPROJ * kBM * 4;
+          const int p = hr / (kBM * 4), rem = hr - p * kBM * 4;
           const int ml = rem >> 2, c = rem & 3;
-          const int m = m0 + ml, col = l * kLoraK + c * 8;
+          const int m = m0 + h * kBM + ml, col = l * kLoraK + c * 8;
           const bool ok = m < a.M && col < a.r;
           const uint16_t *src = ok ? a.ta + (size_t)m * 2 * a.r + p * a.r + col : a.ta;
-          cp_async16_zfill(As + p * (kBM * kLoraK * 2) + kmajor_off(ml, c * 8, 4 * 128u), src, ok ? 16u : 0u);
+          cp_async16_zfill(As + h * kTileBytes + p * (kBM * kLoraK * 2) + kmajor_off(ml, c * 8, 4 * 128u), src,
+                           ok ? 16u : 0u);
         }
         // once landed, each lane fences its generic-proxy writes against the
         // tensor cores' reads, then lane 0 arrives
@@ -226,36 +247,43 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       constexpr uint32_t idesc = umma_idesc_f16(kBM, kBN);
       constexpr uint32_t idesc2 = umma_idesc_f16(kBM, 2 * kBN);
       for (int it = 0; it < nit; ++it) {
-        const int s = it % S, u = it / S;
-        if (!wait(&a_full[s], u & 1) || !wait(&b_full[s], u & 1)) break;
+        const int sa = it % SA, sb = it % SB;
+        if (!wait(&a_full[sa], (it / SA) & 1) || !wait(&b_full[sb], (it / SB) & 1)) break;
         tc_fence_after();
-        const uint32_t as = smem_addr(smem + C::OFF_A + s * kTileBytes);
-        const uint32_t bs = smem_addr(smem + C::OFF_B + s * C::NB * kTileBytes);
-        if (it < nws && NPROJ == 2 && !EXACT) {
+        const uint32_t as0 = smem_addr(smem + C::OFF_A + sa * C::AT);
+        const uint32_t bs = smem_addr(smem + C::OFF_B + sb * C::BT);
+        // every token half multiplies the same B tile into its own accumulators
+        for (int h = 0; h < mth; ++h) {
+          const uint32_t as = as0 + h * kTileBytes, th = tmem + h * C::NCH;
+          if (it < nws && NPROJ == 2 && !EXACT) {
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            umma_f16(tmem, umma_desc_kmajor(as + ks * 4096, 2048, 128), umma_desc_kmajor(bs + ks * 256, 128, kSboTile),
-                     idesc2, (it > 0 || ks > 0) ? 1u : 0u);
-        } else if (it < nws) {
+            for (int ks = 0; ks < 4; ++ks)
+              umma_f16(th, umma_desc_kmajor_sw128(as + ks * 32, 1024), umma_desc_kmajor(bs + ks * 256, 128, kSboTile),
+                       idesc2, (it > 0 || ks > 0) ? 1u : 0u);
+          } else if (it < nws) {
 #pragma unroll
-          for (int p = 0; p < NPROJ; ++p)
+            for (int p = 0; p < NPROJ; ++p)
 #pragma unroll
-            for (int ks = 0; ks < 4; ++ks) {
-              // A (TMA layout): k-step ks = core matrices 2 ks and 2 ks + 1, 2 KB apart
-              umma_f16(tmem + p * kBN, umma_desc_kmajor(as + ks * 4096, 2048, 128),
-                       umma_desc_kmajor(bs + p * kTileBytes + ks * 256, 128, kSboTile), idesc, (it > 0 || ks > 0) ? 1u : 0u);
-              if (EXACT)  // the low parts of the same weights
-                umma_f16(tmem + p * kBN, umma_desc_kmajor(as + ks * 4096, 2048, 128),
-                         umma_desc_kmajor(bs + (NPROJ + p) * kTileBytes + ks * 256, 128, kSboTile), idesc, 1u);
-            }
-        } else {
-          constexpr uint32_t sbo = 4 * 128u;  // 32 rank columns a LoRA stage
-          for (int p = 0; p < NPROJ; ++p)
-            for (int ks = 0; ks < kLoraK / 16; ++ks)
-              umma_f16(tmem + p * kBN, umma_desc_kmajor(as + p * (kBM * kLoraK * 2) + ks * 256, 128, sbo),
-                       umma_desc_kmajor(bs + p * (kBN * kLoraK * 2) + ks * 256, 128, sbo), idesc, 1u);
+              for (int ks = 0; ks < 4; ++ks) {
+                // A (swizzled TMA layout): k-step ks at byte 32 ks of each row
+                umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
+                         umma_desc_kmajor(bs + p * kTileBytes + ks * 256, 128, kSboTile), idesc,
+                         (it > 0 || ks > 0) ? 1u : 0u);
+                if (EXACT)  // the low parts of the same weights
+                  umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
+                           umma_desc_kmajor(bs + (NPROJ + p) * kTileBytes + ks * 256, 128, kSboTile), idesc, 1u);
+              }
+          } else {
+            constexpr uint32_t sbo = 4 * 128u;  // 32 rank columns a LoRA stage
+            for (int p = 0; p < NPROJ; ++p)
+              for (int ks = 0; ks < kLoraK / 16; ++ks)
+                umma_f16(th + p * kBN, umma_desc_kmajor(as + p * (kBM * kLoraK * 2) + ks * 256, 128, sbo),
+                         umma_desc_kmajor(bs + p * (kBN * kLoraK * 2) + ks * 256, 128, sbo), idesc, 1u);
+          }
         }
-        umma_commit(&empty[s]);
+        // both slots are free once these MMAs have read them
+        umma_commit(&a_empty[sa]);
+        umma_commit(&b_empty[sb]);
       }
       umma_commit(acc_full);
     }
@@ -264,10 +292,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ---- dequantization into the B tiles ----
     const int dt = tid;  // 0 .. kDeqWarps * 32 - 1
     for (int it = 0; it < nit; ++it) {
-      const int s = it % S, u = it / S, kb = it >> 1, hb = it & 1, q = kb % R;
+      const int s = it % SB, kb = it >> 1, hb = it & 1, q = kb % R;
       if (it < nws && !wait(&raw_full[q], (kb / R) & 1)) break;
-      if (it >= S && !wait(&empty[s], (u - 1) & 1)) break;
-      uint8_t *Bs = smem + C::OFF_B + s * C::NB * kTileBytes;
+      if (it >= SB && !wait(&b_empty[s], (it / SB - 1) & 1)) break;
+      uint8_t *Bs = smem + C::OFF_B + s * C::BT;
       if (it < nws) {
         const uint8_t *raw = smem + C::OFF_RAW + q * C::RAW;
         // item = (projection, 16-row tile, lane of the packed fragment layout)
@@ -367,73 +395,77 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       }
     }
 
-    // ---- epilogue (warps 0..3: TMEM lanes 32 w .. 32 w + 31 = tokens) ----
-    if (warp < 4 && wait(acc_full, 0)) {
+    // ---- epilogue: warp w reads TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31
+    // (the tokens of each half) and columns 32 (w / 4) .. 32 (w / 4) + 31 ----
+    if (wait(acc_full, 0)) {
       tc_fence_after();
-      const int m = m0 + warp * 32 + lane;
-      const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
-      const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
-      // rows n0 + c .. n0 + c + 7 of this token: 16-byte stores when the
-      // row length allows (N a multiple of 8), element stores otherwise
-      const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
-      for (int c = 0; c < kBN; c += 8) {
-        uint32_t g[8], uu[8];
-        tmem_ld8(tl + c, g);
-        if (NPROJ == 2) tmem_ld8(tl + kBN + c, uu);
-        tmem_ld_wait();
-        const int nb = n0 + c;
-        if (m >= a.M || nb >= a.N) continue;
-        float v[8];
-        if (NPROJ == 2) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float gv = rs * __uint_as_float(g[e]), uv = rs * __uint_as_float(uu[e]);
-            v[e] = __bfloat162float(__float2bfloat16_rn(gv / (1.f + __expf(-gv)) * uv));  // h as stored
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) v[e] = __uint_as_float(g[e]);
-          if (a.residual) {
-            if (vec) {
-              const uint4 rv = *reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.residual) +
-                                                                (size_t)m * a.N + nb);
-              const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
-#pragma unroll
-              for (int e = 0; e < 8; ++e) v[e] += __uint_as_float(e & 1 ? (rw[e >> 1] & 0xffff0000u) : (rw[e >> 1] << 16));
-            } else {
-              for (int e = 0; e < 8 && nb + e < a.N; ++e)
-                v[e] += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + nb + e]);
+      const int quarter = warp & 3, c0 = (warp >> 2) * 32;
+      for (int h = 0; h < mth; ++h) {
+        const int m = m0 + h * kBM + quarter * 32 + lane;
+        const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+        const uint32_t tl = tmem + h * C::NCH + ((uint32_t)(quarter * 32) << 16);
+        // rows n0 + c .. n0 + c + 7 of this token: 16-byte stores when the
+        // row length allows (N a multiple of 8), element stores otherwise
+        const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
+        for (int c = c0; c < c0 + 32; c += 8) {
+          uint32_t g[8], uu[8];
+          tmem_ld8(tl + c, g);
+          if (NPROJ == 2) tmem_ld8(tl + kBN + c, uu);
+          tmem_ld_wait();
+          const int nb = n0 + c;
+          if (m >= a.M || nb >= a.N) continue;
+          float v[8];
+          if (NPROJ == 2) {
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float gv = rs * __uint_as_float(g[e]), uv = rs * __uint_as_float(uu[e]);
+              v[e] = __bfloat162float(__float2bfloat16_rn(gv / (1.f + __expf(-gv)) * uv));  // h as stored
             }
-          }
-        }
-        if (vec) {
-          if (NPROJ == 1 && a.out_f32) {
-            float4 *o = reinterpret_cast<float4 *>(reinterpret_cast<float *>(a.out) + (size_t)m * a.N + nb);
-            o[0] = make_float4(v[0], v[1], v[2], v[3]);
-            o[1] = make_float4(v[4], v[5], v[6], v[7]);
           } else {
-            uint32_t w[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-              w[e] = *reinterpret_cast<const uint32_t *>(&b2);
-            }
-            *reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) + (size_t)m * a.N + nb) =
-                make_uint4(w[0], w[1], w[2], w[3]);
-            if (NPROJ == 2 && a.out_f16) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) w[e] = h2bits(__floats2half2_rn(v[2 * e], v[2 * e + 1]));
-              *reinterpret_cast<uint4 *>(a.out_f16 + (size_t)m * a.ldo16 + nb) = make_uint4(w[0], w[1], w[2], w[3]);
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = __uint_as_float(g[e]);
+            if (a.residual) {
+              if (vec) {
+                const uint4 rv = *reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.residual) +
+                                                                  (size_t)m * a.N + nb);
+                const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+  #pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] += __uint_as_float(e & 1 ? (rw[e >> 1] & 0xffff0000u) : (rw[e >> 1] << 16));
+              } else {
+                for (int e = 0; e < 8 && nb + e < a.N; ++e)
+                  v[e] += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + nb + e]);
+              }
             }
           }
-        } else {
-          for (int e = 0; e < 8 && nb + e < a.N; ++e) {
-            const size_t o = (size_t)m * a.N + nb + e;
+          if (vec) {
             if (NPROJ == 1 && a.out_f32) {
-              reinterpret_cast<float *>(a.out)[o] = v[e];
+              float4 *o = reinterpret_cast<float4 *>(reinterpret_cast<float *>(a.out) + (size_t)m * a.N + nb);
+              o[0] = make_float4(v[0], v[1], v[2], v[3]);
+              o[1] = make_float4(v[4], v[5], v[6], v[7]);
             } else {
-              reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v[e]);
-              if (NPROJ == 2 && a.out_f16) a.out_f16[(size_t)m * a.ldo16 + nb + e] = __half_as_ushort(__float2half_rn(v[e]));
+              uint32_t w[4];
+  #pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+                w[e] = *reinterpret_cast<const uint32_t *>(&b2);
+              }
+              *reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) + (size_t)m * a.N + nb) =
+                  make_uint4(w[0], w[1], w[2], w[3]);
+              if (NPROJ == 2 && a.out_f16) {
+  #pragma unroll
+                for (int e = 0; e < 4; ++e) w[e] = h2bits(__floats2half2_rn(v[2 * e], v[2 * e + 1]));
+                *reinterpret_cast<uint4 *>(a.out_f16 + (size_t)m * a.ldo16 + nb) = make_uint4(w[0], w[1], w[2], w[3]);
+              }
+            }
+          } else {
+            for (int e = 0; e < 8 && nb + e < a.N; ++e) {
+              const size_t o = (size_t)m * a.N + nb + e;
+              if (NPROJ == 1 && a.out_f32) {
+                reinterpret_cast<float *>(a.out)[o] = v[e];
+              } else {
+                reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v[e]);
+                if (NPROJ == 2 && a.out_f16) a.out_f16[(size_t)m * a.ldo16 + nb + e] = __half_as_ushort(__float2half_rn(v[e]));
+              }
             }
           }
         }
@@ -447,68 +479,128 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   if (warp == kMmaWarp) tmem_dealloc(tmem, C::NCOLS);
 }
 
-// Per token of x [M, K] (bf16): the binary16 copy (the GEMM's A operand), the
-// RMSNorm scale rs = 1/sqrt(mean(x^2) + eps) and, with an adapter,
-// ta = lora_scale * x A^T as binary16 [M][2r] (gate rows, then up rows).
-// A CTA takes kPrepTok tokens, staged in shared memory, so that every LoRA-A
-// row it reads serves all of them; fixed-order reductions.
-constexpr int kPrepTok = 4;
+// Per token of x [M, K] (bf16, K a multiple of 32): the binary16 copy x16
+// [M][lda16] (the GEMM's A operand, zeros past K), the RMSNorm scale
+// rs = 1/sqrt(mean(x^2) + eps) and, with an adapter, ta = lora_scale * x A^T
+// as binary16 [M][2r] (gate rows, then up rows).
+// A CTA takes 32 tokens and 16 rows of A.  The products x A^T run on m16n8k16
+// bf16 MMAs (exact products, fp32 sums); the 8 warps take interleaved chunks
+// of 32 features and their partial sums are added in warp order.  A lane
+// loads 8 consecutive features of a row (16 bytes) and feeds features 0..3 and
+// 4..7 of them to two k-steps in the slots of k 2t, 2t+1, 2t+8, 2t+9: the same
+// permutation of k for x and A, so the sums are unchanged.  Every CTA sums x^2
+// of its tokens (row block 0 writes rs) and converts the chunks c with
+// c % gridDim.y == blockIdx.y.
+constexpr int kPrepTok = 32, kPrepRows = 16;
 
 __global__ void __launch_bounds__(256) gemm_prep_kernel(const __nv_bfloat16 *x, int M, int K, int lda16,
                                                         const __nv_bfloat16 *lora_a, int r2, float lora_scale,
                                                         uint16_t *x16, float *rs, uint16_t *ta) {
-  extern __shared__ __align__(16) __nv_bfloat16 xs[];  // [kPrepTok][K]
-  __shared__ float red[kPrepTok][8];
-  const int m0 = blockIdx.x * kPrepTok, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int nt = min(kPrepTok, M - m0);
-  float ss[kPrepTok];
+  __shared__ float part[8][kPrepTok][kPrepRows + 1];
+  __shared__ float ssp[8][kPrepTok];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, g = lane >> 2, t = lane & 3;
+  const int m0 = blockIdx.x * kPrepTok, j0 = blockIdx.y * kPrepRows;
+  const int nchunk = K / 32;
+  const bool lora = r2 > 0;
+  float acc[2][2][4];
 #pragma unroll
-  for (int t = 0; t < kPrepTok; ++t) ss[t] = 0.f;
+  for (int i = 0; i < 16; ++i) acc[i >> 3][(i >> 2) & 1][i & 3] = 0.f;
+  float ss[4] = {0.f, 0.f, 0.f, 0.f};  // tokens g, g + 8, g + 16, g + 24 of the block
+  for (int c = warp; c < nchunk; c += 8) {
+    const int k = c * 32 + 8 * t;
+    uint4 xa[4], ab[2];
 #pragma unroll
-  for (int t = 0; t < kPrepTok; ++t) {
-    if (t >= nt) break;
-    const __nv_bfloat16 *xr = x + (size_t)(m0 + t) * K;
-    for (int k = tid; k < K; k += blockDim.x) {
-      const __nv_bfloat16 bv = xr[k];
-      const float v = __bfloat162float(bv);
-      xs[t * K + k] = bv;
-      ss[t] = fmaf(v, v, ss[t]);
-      x16[(size_t)(m0 + t) * lda16 + k] = __half_as_ushort(__float2half_rn(v));
+    for (int i = 0; i < 4; ++i) {
+      const int m = m0 + g + 8 * i;
+      xa[i] = m < M ? __ldg(reinterpret_cast<const uint4 *>(x + (size_t)m * K + k)) : make_uint4(0u, 0u, 0u, 0u);
     }
-    for (int k = K + tid; k < lda16; k += blockDim.x) x16[(size_t)(m0 + t) * lda16 + k] = 0;
+#pragma unroll
+    for (int n = 0; n < 2; ++n) {
+      const int j = j0 + 8 * n + g;
+      ab[n] = lora && j < r2 ? __ldg(reinterpret_cast<const uint4 *>(lora_a + (size_t)j * K + k))
+                             : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
+        ss[i] = fmaf(lo, lo, ss[i]);
+        ss[i] = fmaf(hi, hi, ss[i]);
+      }
+    }
+    if (c % gridDim.y == blockIdx.y) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int m = m0 + g + 8 * i;
+        if (m >= M) continue;
+        const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          o[e] = h2bits(__floats2half2_rn(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u)));
+        *reinterpret_cast<uint4 *>(x16 + (size_t)m * lda16 + k) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
+    if (lora) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const auto word = [&](const uint4 &v, int q) { return q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w; };
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          // rows g, g + 8 of m-tile mt are tokens 16 mt + g (xa[2 mt]) and 16 mt + g + 8 (xa[2 mt + 1])
+          const uint32_t af[4] = {word(xa[2 * mt], 2 * h), word(xa[2 * mt + 1], 2 * h), word(xa[2 * mt], 2 * h + 1),
+                                  word(xa[2 * mt + 1], 2 * h + 1)};
+#pragma unroll
+          for (int nt = 0; nt < 2; ++nt) mma_bf16_16816(acc[mt][nt], af, word(ab[nt], 2 * h), word(ab[nt], 2 * h + 1));
+        }
+      }
+    }
   }
+  // sums of squares: the quad's lanes hold disjoint features of the same tokens
 #pragma unroll
-  for (int t = 0; t < kPrepTok; ++t) {
+  for (int i = 0; i < 4; ++i) {
+    ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 1);
+    ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 2);
+  }
+  if (t == 0)
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss[t] += __shfl_xor_sync(0xffffffffu, ss[t], o);
-    if (lane == 0) red[t][warp] = ss[t];
+    for (int i = 0; i < 4; ++i) ssp[warp][g + 8 * i] = ss[i];
+  if (lora) {
+    // accumulator (row, col) of m-tile mt, n-tile nt: rows g / g + 8, cols 2t, 2t+1
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        part[warp][16 * mt + g][8 * nt + 2 * t] = acc[mt][nt][0];
+        part[warp][16 * mt + g][8 * nt + 2 * t + 1] = acc[mt][nt][1];
+        part[warp][16 * mt + g + 8][8 * nt + 2 * t] = acc[mt][nt][2];
+        part[warp][16 * mt + g + 8][8 * nt + 2 * t + 1] = acc[mt][nt][3];
+      }
   }
   __syncthreads();
-  if (tid < nt) {
+  if (blockIdx.y == 0 && tid < kPrepTok && m0 + tid < M) {
     float tot = 0.f;
-    for (int w = 0; w < 8; ++w) tot += red[tid][w];
+    for (int w = 0; w < 8; ++w) tot += ssp[w][tid];
     rs[m0 + tid] = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)K), kRmsEps)));
   }
-  if (r2 > 0) {
-    // warp w takes LoRA-A rows w, w + 8, ...: lanes stride the features, then the warp adds up
-    for (int j = warp; j < r2; j += 8) {
-      const __nv_bfloat16 *ar = lora_a + (size_t)j * K;
-      float acc[kPrepTok];
-#pragma unroll
-      for (int t = 0; t < kPrepTok; ++t) acc[t] = 0.f;
-      for (int k = lane; k < K; k += 32) {
-        const float av = __bfloat162float(ar[k]);
-#pragma unroll
-        for (int t = 0; t < kPrepTok; ++t) acc[t] = fmaf(av, __bfloat162float(xs[t * K + k]), acc[t]);
-      }
-#pragma unroll
-      for (int t = 0; t < kPrepTok; ++t) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc[t] += __shfl_xor_sync(0xffffffffu, acc[t], o);
-        if (lane == 0 && t < nt) ta[(size_t)(m0 + t) * r2 + j] = __half_as_ushort(__float2half_rn(lora_scale * acc[t]));
-      }
+  if (lora) {
+    for (int o = tid; o < kPrepTok * kPrepRows; o += 256) {
+      const int tl = o / kPrepRows, jl = o % kPrepRows;
+      const int m = m0 + tl, j = j0 + jl;
+      if (m >= M || j >= r2) continue;
+      float v = 0.f;
+      for (int w = 0; w < 8; ++w) v += part[w][tl][jl];
+      ta[(size_t)m * r2 + j] = __half_as_ushort(__float2half_rn(lora_scale * v));
     }
   }
+  // zeros past K
+  if (blockIdx.y == 0)
+    for (int i = tid; i < kPrepTok * (lda16 - K); i += 256) {
+      const int tl = i / (lda16 - K), k = K + i % (lda16 - K);
+      if (m0 + tl < M) x16[(size_t)(m0 + tl) * lda16 + k] = 0;
+    }
 }
 
 // bf16 [M, K] -> binary16 [M, lda16] (zero padded), the down GEMM's A operand.
@@ -545,9 +637,9 @@ cudaError_t make_maps(const GemmArgs &a, int nproj, int bits, GemmMaps *m) {
   {
     const cuuint64_t dims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
     const cuuint64_t strides[1] = {(cuuint64_t)a.lda * 2};
-    const cuuint32_t box[2] = {8, (cuuint32_t)kBM};
+    const cuuint32_t box[2] = {64, (cuuint32_t)kBM};
     if (fn(&m->act, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t *>(a.act), dims, strides, box, e1,
-           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
@@ -585,8 +677,19 @@ cudaError_t launch_gemm_t(const GemmArgs &a, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   GemmMaps maps;
   if ((e = make_maps(a, NPROJ, BITS, &maps)) != cudaSuccess) return e;
-  const dim3 grid((a.M + kBM - 1) / kBM, (a.N + kBN - 1) / kBN);
-  kern<<<grid, kGemmThreads, C::SMEM, s>>>(a, maps);
+  // two token halves a CTA (the B tile dequantized once for 256 tokens) when
+  // that still gives every SM a CTA; one otherwise
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  }
+  const int nt = (a.N + kBN - 1) / kBN;
+  GemmArgs ka = a;
+  ka.mt = (a.M + 2 * kBM - 1) / (2 * kBM) * nt >= sms ? 2 : 1;
+  const dim3 grid((a.M + ka.mt * kBM - 1) / (ka.mt * kBM), nt);
+  kern<<<grid, kGemmThreads, C::SMEM, s>>>(ka, maps);
   return cudaGetLastError();
 }
 
@@ -613,12 +716,9 @@ cudaError_t launch_gemm(GemvKind kind, const GemmArgs &a, cudaStream_t s) {
 cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void *lora_a, int r2, float lora_scale,
                              uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  const size_t smem = (size_t)kPrepTok * K * 2;
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  gemm_prep_kernel<<<(M + kPrepTok - 1) / kPrepTok, 256, smem, s>>>(
+  if (K % 32 != 0 || lda16 < K) return cudaErrorInvalidValue;
+  const dim3 grid((M + kPrepTok - 1) / kPrepTok, r2 > 0 ? (r2 + kPrepRows - 1) / kPrepRows : 1);
+  gemm_prep_kernel<<<grid, 256, 0, s>>>(
       reinterpret_cast<const __nv_bfloat16 *>(x), M, K, lda16, reinterpret_cast<const __nv_bfloat16 *>(lora_a), r2,
       lora_scale, x16, rs, ta);
   return cudaGetLastError();
@@ -644,15 +744,15 @@ cudaError_t read_gemm_status(int *status) {
 
 int gemm_stages(GemvKind kind, int group) {
   switch (kind * 3 + (group == 32 ? 0 : group == 64 ? 1 : 2)) {
-    case 0: return GemmCfg<2, 2, 32, false>::S;
-    case 1: return GemmCfg<2, 2, 64, false>::S;
-    case 2: return GemmCfg<2, 2, 128, false>::S;
-    case 3: return GemmCfg<4, 2, 32, false>::S;
-    case 4: return GemmCfg<4, 2, 64, false>::S;
-    case 5: return GemmCfg<4, 2, 128, false>::S;
-    case 6: return GemmCfg<4, 1, 32, false>::S;
-    case 7: return GemmCfg<4, 1, 64, false>::S;
-    default: return GemmCfg<4, 1, 128, false>::S;
+    case 0: return GemmCfg<2, 2, 32, false>::SA;
+    case 1: return GemmCfg<2, 2, 64, false>::SA;
+    case 2: return GemmCfg<2, 2, 128, false>::SA;
+    case 3: return GemmCfg<4, 2, 32, false>::SA;
+    case 4: return GemmCfg<4, 2, 64, false>::SA;
+    case 5: return GemmCfg<4, 2, 128, false>::SA;
+    case 6: return GemmCfg<4, 1, 32, false>::SA;
+    case 7: return GemmCfg<4, 1, 64, false>::SA;
+    default: return GemmCfg<4, 1, 128, false>::SA;
   }
 }
 

@@ -103,6 +103,7 @@ struct GemmArgs {
   int out_f32;
   uint16_t *out_f16;         // gate/up: h also as binary16 [M][ldo16] (the down GEMM's A), or null
   int ldo16;
+  int mt;                    // token halves of 128 per CTA (1 or 2; set by launch_gemm)
 };
 cudaError_t launch_gemm(GemvKind kind, const GemmArgs &args, cudaStream_t stream);
 // x16 [M][lda16] = binary16(x), rs[m] = 1/sqrt(mean(x^2) + eps), ta [M][r2] = lora_scale * x A^T (r2 > 0)
@@ -110,7 +111,7 @@ cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void 
                              uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t stream);
 // x16 [M][lda16] = binary16(x) (zero padded)
 cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, cudaStream_t stream);
-int gemm_stages(GemvKind kind, int group);
+int gemm_stages(GemvKind kind, int group);  // depth of the activation-tile ring
 // Reads and clears the GEMM kernels' device status word.
 cudaError_t read_gemm_status(int *status);
 

@@ -136,3 +136,34 @@ def test_gemm_stack_matches_oracle(wq, m):
     torch.cuda.synchronize()
     assert wq.device_status() == 0
     assert torch.equal(y, cur), "the stack call differs from its layers called one by one"
+
+
+@pytest.mark.parametrize("m", [257, 300, 512])
+def test_gemm_two_token_halves(wq, m):
+    """Enough 256-token x 128-row tiles for every SM: each CTA takes two token
+    halves of 128 that share the dequantized B tile (the last CTA of m = 300
+    holds one half).  Gate/up with the adapter and the RMSNorm, then down with
+    a residual, in bf16 and fp32."""
+    d, inter, group, r = 256, 9728, 64, 16
+    qg, qu = _q((inter, d), group, 2, 71), _q((inter, d), group, 2, 72)
+    a, bg, bu = synth.lora(d, inter, r, 73)
+    x = synth.activations((m, d), 74 + m)
+    h = wq.gateup_w2_lora(x.cuda(), upload_packed(*qg, group, 2), upload_packed(*qu, group, 2), prenorm=True,
+                          lora_a=a.cuda(), lora_b_gate=bg.cuda(), lora_b_up=bu.cuda(), lora_scale=2.0)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.gateup(synth.bf16_bits(x), qg, qu, group, synth.bf16_bits(a), synth.bf16_bits(bg),
+                        synth.bf16_bits(bu), lora_scale=2.0, prenorm=True)
+    check_bf16(h, ref, f"GEMM h (two halves) m={m}", min_exact=MIN_EXACT)
+    # down: 9728 output rows from 256 features
+    qd = _q((inter, d), group, 4, 75)
+    hd = (synth.activations((m, d), 76 + m) * 0.5).to(torch.bfloat16)
+    res = synth.activations((m, inter), 77 + m)
+    dn = upload_packed(*qd, group, 4)
+    y = wq.down_w4(hd.cuda(), dn, residual=res.cuda())
+    y32 = wq.down_w4(hd.cuda(), dn, residual=res.cuda(), out_f32=True)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.down(synth.bf16_bits(hd), qd, group, synth.bf16_bits(res))
+    check_bf16(y, ref, f"GEMM y (two halves) m={m}", min_exact=MIN_EXACT)
+    check_f32(y32, ref, f"GEMM y(f32) (two halves) m={m}")
