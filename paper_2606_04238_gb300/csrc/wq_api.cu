@@ -115,6 +115,13 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
     L->rs = off;  off = up256(off + (size_t)m * 4);
     L->ta = off;  off = up256(off + (size_t)m * 2 * kMaxRank * 2);
     L->h16 = off; off = up256(off + (size_t)m * ldi * 2);
+    // stream-K scratch shared by the gate/up and down launches (one at a time)
+    const int sms = num_sms();
+    if (sms <= 0) return false;
+    const size_t cnt = std::max(gemm_counters(m, inter), gemm_counters(m, d));
+    const size_t part = std::max(gemm_scratch_floats(m, inter, d, 2, sms), gemm_scratch_floats(m, d, inter, 1, sms));
+    L->cnt1 = off;  off = up256(off + cnt * 4);
+    L->part1 = off; off = up256(off + part * 4);
     L->total = off;
     return true;
   }
@@ -287,6 +294,8 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
   a.out = h;
   a.out_f16 = h16;
   a.ldo16 = (inter + 127) / 128 * 128;
+  a.sk_part = reinterpret_cast<float *>(ws + L.part1);
+  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.cnt1);
   e = launch_gemm(kind, a, s);
   if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
   return WQ_OK;
@@ -314,6 +323,8 @@ wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qwei
   a.residual = residual;
   a.out = y;
   a.out_f32 = y_f32;
+  a.sk_part = reinterpret_cast<float *>(ws + L.part1);
+  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.cnt1);
   cudaError_t e = launch_gemm(kDownW4, a, s);
   if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   return WQ_OK;

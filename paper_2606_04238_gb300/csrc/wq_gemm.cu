@@ -132,23 +132,314 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
       : "memory");
 }
 
-template <int BITS, int NPROJ, int GROUP, bool EXACT>
-__global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a, const __grid_constant__ GemmMaps tm) {
-  using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
-  constexpr int SA = C::SA, SB = C::SB, R = C::R, GPB = C::GPB, GS = GROUP / 16;
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  // the swizzled activation tiles need 1024-byte alignment
-  uint8_t *smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
-  uint64_t *raw_full = reinterpret_cast<uint64_t *>(smem + C::OFF_BAR);
-  uint64_t *raw_empty = raw_full + R;
-  uint64_t *a_full = raw_empty + R;
-  uint64_t *a_empty = a_full + SA;
-  uint64_t *b_full = a_empty + SA;
-  uint64_t *b_empty = b_full + SB;
-  uint64_t *acc_full = b_empty + SB;
-  uint32_t *tmem_s = reinterpret_cast<uint32_t *>(acc_full + 2);
-  volatile int *abort_s = reinterpret_cast<volatile int *>(tmem_s + 1);
+// The epilogue of one part of a tile (the 16 dequantizing warps, after the
+// part's accumulators are complete; `have`: no timeout so far).  Warp w reads
+// TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the tokens of each half) and
+// columns 32 (w / 4) .. 32 (w / 4) + 31.  A whole tile is finished from TMEM;
+// a part of a split tile is written to its scratch slot, and the CTA that adds
+// the tile's last part to its counter sums the parts in k order (their CTAs
+// are consecutive) and finishes the tile.  Kept out of line so that the
+// dequantization loop keeps its registers.
+// ---------------------------------------------------------------------------
+// Pieces shared by the two kernels below.
+// ---------------------------------------------------------------------------
 
+// Dequantizes the stage hb (features 64 hb .. 64 hb + 63) of a block of
+// packed codes `raw` into the B tiles `Bs`; thread dt of the 16 dequantizing
+// warps takes the items (projection, 16-row tile, lane of the fragment layout)
+// dt, dt + 512, ...
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+__device__ __forceinline__ void gemm_deq_stage(const uint8_t *raw, uint8_t *Bs, int hb, int dt) {
+  using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  constexpr int GPB = C::GPB, GS = GROUP / 16;
+  for (int item = dt; item < NPROJ * 8 * 32; item += kDeqWarps * 32) {
+    const int p = item >> 8, j = (item >> 5) & 7, L = item & 31;
+    const int g = L >> 2, t = L & 3;
+    uint8_t *Bp = Bs + p * kTileBytes;
+    // the lane's code words of this half block: 2-bit, words 2 hb, 2 hb + 1
+    // of its 16 bytes; 4-bit, the 16 bytes of half hb
+    uint32_t wds[BITS == 2 ? 2 : 4];
+    const uint8_t *cb = raw + p * C::RAWP + j * C::BPK;               // codes of tile j
+    const uint8_t *mb = raw + p * C::RAWP + 8 * C::BPK + j * GPB * 64;  // its scales/zeros
+    if (BITS == 2) {
+      const uint2 w0 = lds64(cb + L * 16 + hb * 8);
+      wds[0] = w0.x;
+      wds[1] = w0.y;
+    } else {
+      const uint4 w0 = lds128(cb + hb * 512 + L * 16);
+      wds[0] = w0.x;
+      wds[1] = w0.y;
+      wds[2] = w0.z;
+      wds[3] = w0.w;
+    }
+    // this stage: k-steps 4 hb .. 4 hb + 3 of the block
+#pragma unroll
+    for (int gl = 0; gl < (GS >= 4 ? 1 : 4 / GS); ++gl) {
+      const int gi = (4 * hb) / GS + gl;
+      // scales and zeros of rows g and g + 8 in group gi (zero for tiles outside the matrix)
+      const uint2 sz = lds64(mb + gi * 64 + g * 8);
+      // scales of rows g ("lo" row) and g + 8 ("hi" row); EXACT splits each
+      // into a head with the 4 lowest mantissa bits cleared and the tail
+      const uint32_t sg = sz.x & 0xffffu, sg8 = sz.x >> 16;
+      const __half2 s_lo = __half2half2(__ushort_as_half((unsigned short)(EXACT ? (sg & 0xfff0u) : sg)));
+      const __half2 s_hi = __half2half2(__ushort_as_half((unsigned short)(EXACT ? (sg8 & 0xfff0u) : sg8)));
+      const __half2 t_lo = __half2half2(
+          __hsub(__ushort_as_half((unsigned short)sg), __ushort_as_half((unsigned short)(sg & 0xfff0u))));
+      const __half2 t_hi = __half2half2(
+          __hsub(__ushort_as_half((unsigned short)sg8), __ushort_as_half((unsigned short)(sg8 & 0xfff0u))));
+      // 1024 + z: the code read as 1024 + q minus this is q - z exactly
+      const __half2 z_lo =
+          __half2half2(__hadd(__ushort_as_half((unsigned short)(sz.y & 0xffffu)), __float2half(1024.f)));
+      const __half2 z_hi = __half2half2(__hadd(__ushort_as_half((unsigned short)(sz.y >> 16)), __float2half(1024.f)));
+#pragma unroll
+      for (int kk = 0; kk < (GS >= 4 ? 4 : GS); ++kk) {
+        const int ks = (GS >= 4 ? 4 * hb : gi * GS) + kk;
+        uint32_t q[4];  // (row g, k 2t..2t+1), (row g+8, ...), (row g, k 2t+8..), (row g+8, k 2t+8..)
+        const int kl = ks - 4 * hb;  // k-step within the half block
+        if (BITS == 2) {
+          const uint32_t x = wds[(kl >> 1) & 1];
+          const int s4 = (kl & 1) * 4;
+          q[0] = (x >> s4) & 0x00030003u;
+          q[1] = (x >> (s4 + 8)) & 0x00030003u;
+          q[2] = (x >> (s4 + 2)) & 0x00030003u;
+          q[3] = (x >> (s4 + 10)) & 0x00030003u;
+        } else {
+          const uint32_t x = wds[kl & 3];
+          q[0] = x & 0x000F000Fu;
+          q[1] = (x >> 8) & 0x000F000Fu;
+          q[2] = (x >> 4) & 0x000F000Fu;
+          q[3] = (x >> 12) & 0x000F000Fu;
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __half2 v = bits2h(q[e] | 0x64006400u);  // 1024 + q, exact
+          const bool hi_row = (e & 1) != 0;
+          const __half2 qz = __hsub2(v, hi_row ? z_hi : z_lo);  // q - z, exact
+          const __half2 w = __hmul2(qz, hi_row ? s_hi : s_lo);
+          const int row = j * 16 + g + (hi_row ? 8 : 0);
+          const int k = kl * 16 + 2 * t + ((e & 2) ? 8 : 0);  // within the stage
+          *reinterpret_cast<uint32_t *>(Bp + kmajor_off(row, k, kSboTile)) = h2bits(w);
+          if (EXACT)
+            *reinterpret_cast<uint32_t *>(Bp + NPROJ * kTileBytes + kmajor_off(row, k, kSboTile)) =
+                h2bits(__hmul2(qz, hi_row ? t_hi : t_lo));
+        }
+      }
+    }
+  }
+}
+
+// LoRA stage l, B side: rows n0 .. n0 + 127 of B_p (bf16 [N][r]), rank
+// columns 32 l .. 32 l + 31 -> binary16, zeros past r.
+template <int NPROJ>
+__device__ __forceinline__ void gemm_lora_b_stage(const GemmArgs &a, uint8_t *Bs, int n0, int l, int dt) {
+  constexpr uint32_t sbo = 4 * 128u;
+  for (int i = dt; i < NPROJ * kBN * 4; i += kDeqWarps * 32) {
+    const int p = i / (kBN * 4), rem = i - p * kBN * 4;
+    const int nl = rem >> 2, c = rem & 3;
+    const int n = n0 + nl, col = l * kLoraK + c * 8;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (n < a.N && col < a.r)
+      v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_b[p]) +
+                                                ((size_t)n * a.r + col) * 2));
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
+      o[e] = h2bits(__floats2half2_rn(lo, hi));
+    }
+    *reinterpret_cast<uint4 *>(Bs + p * (kBN * kLoraK * 2) + kmajor_off(nl, c * 8, sbo)) =
+        make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// LoRA stage l, A side (one warp): lora_scale * t, rank columns 32 l .. 32 l
+// + 31 of gate (first r columns of ta) and of up (next r) for the mth token
+// halves from m0, zeros past r; lane 0 arrives on `full` once all landed.
+template <int NPROJ>
+__device__ __forceinline__ void gemm_lora_a_stage(const GemmArgs &a, uint8_t *As, int m0, int mth, int l, int lane,
+                                                  uint64_t *full) {
+  for (int i = lane; i < mth * NPROJ * kBM * 4; i += 32) {
+    const int h = i / (NPROJ * kBM * 4), hr = i - h * NPROJ * kBM * 4;
+    const int p = hr / (kBM * 4), rem = hr - p * kBM * 4;
+    const int ml = rem >> 2, c = rem & 3;
+    const int m = m0 + h * kBM + ml, col = l * kLoraK + c * 8;
+    const bool in = m < a.M && col < a.r;
+    const uint16_t *src = in ? a.ta + (size_t)m * 2 * a.r + p * a.r + col : a.ta;
+    cp_async16_zfill(As + h * kTileBytes + p * (kBM * kLoraK * 2) + kmajor_off(ml, c * 8, 4 * 128u), src,
+                     in ? 16u : 0u);
+  }
+  // once landed, each lane fences its generic-proxy writes against the tensor
+  // cores' reads, then lane 0 arrives
+  cp_async_wait_all();
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(full);
+}
+
+// The MMAs of one stage (one thread): every token half multiplies the same B
+// tile into its own accumulators; `first` starts the accumulators.
+template <int NPROJ, bool EXACT>
+__device__ __forceinline__ void gemm_issue_stage(uint32_t tmem, uint32_t as0, uint32_t bs, int mth, bool wstage,
+                                                 bool first) {
+  constexpr int NCH = NPROJ * kBN;
+  // gate/up: one MMA of N = 256 a k-step (the gate tile and the up tile are
+  // adjacent, 256 rows), so the activation tile is read once
+  constexpr uint32_t idesc = umma_idesc_f16(kBM, kBN);
+  constexpr uint32_t idesc2 = umma_idesc_f16(kBM, 2 * kBN);
+  for (int h = 0; h < mth; ++h) {
+    const uint32_t as = as0 + h * kTileBytes, th = tmem + h * NCH;
+    if (wstage && NPROJ == 2 && !EXACT) {
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks)
+        umma_f16(th, umma_desc_kmajor_sw128(as + ks * 32, 1024), umma_desc_kmajor(bs + ks * 256, 128, kSboTile), idesc2,
+                 (first && ks == 0) ? 0u : 1u);
+    } else if (wstage) {
+#pragma unroll
+      for (int p = 0; p < NPROJ; ++p)
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+          // A (swizzled TMA layout): k-step ks at byte 32 ks of each row
+          umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
+                   umma_desc_kmajor(bs + p * kTileBytes + ks * 256, 128, kSboTile), idesc,
+                   (first && ks == 0) ? 0u : 1u);
+          if (EXACT)  // the low parts of the same weights
+            umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
+                     umma_desc_kmajor(bs + (NPROJ + p) * kTileBytes + ks * 256, 128, kSboTile), idesc, 1u);
+        }
+    } else {
+      constexpr uint32_t sbo = 4 * 128u;  // 32 rank columns a LoRA stage
+      for (int p = 0; p < NPROJ; ++p)
+        for (int ks = 0; ks < kLoraK / 16; ++ks)
+          umma_f16(th + p * kBN, umma_desc_kmajor(as + p * (kBM * kLoraK * 2) + ks * 256, 128, sbo),
+                   umma_desc_kmajor(bs + p * (kBN * kLoraK * 2) + ks * 256, 128, sbo), idesc,
+                   (first && ks == 0) ? 0u : 1u);
+    }
+  }
+}
+
+// Output of 8 consecutive rows nb .. nb + 7 of token m from the fp32 sums g
+// (and u for gate/up): h = SiLU(rs g) * (rs u) (also in binary16 when asked),
+// or y = g + residual in bf16 or fp32.  `vec`: 16-byte stores (N and the
+// binary16 row length multiples of 8).
+template <int NPROJ>
+__device__ __forceinline__ void gemm_finish(const GemmArgs &a, int m, int nb, float rs, const float (&g)[8],
+                                            const float (&u)[8], bool vec) {
+  if (m >= a.M || nb >= a.N) return;
+  float v[8];
+  if (NPROJ == 2) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float gv = rs * g[e], uv = rs * u[e];
+      v[e] = __bfloat162float(__float2bfloat16_rn(__fdividef(gv, 1.f + __expf(-gv)) * uv));  // h as stored
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = g[e];
+    if (a.residual) {
+      if (vec) {
+        const uint4 rv =
+            *reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.residual) + (size_t)m * a.N + nb);
+        const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] += __uint_as_float(e & 1 ? (rw[e >> 1] & 0xffff0000u) : (rw[e >> 1] << 16));
+      } else {
+        for (int e = 0; e < 8 && nb + e < a.N; ++e)
+          v[e] += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + nb + e]);
+      }
+    }
+  }
+  if (vec) {
+    if (NPROJ == 1 && a.out_f32) {
+      float4 *o = reinterpret_cast<float4 *>(reinterpret_cast<float *>(a.out) + (size_t)m * a.N + nb);
+      o[0] = make_float4(v[0], v[1], v[2], v[3]);
+      o[1] = make_float4(v[4], v[5], v[6], v[7]);
+    } else {
+      uint32_t w[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+        w[e] = *reinterpret_cast<const uint32_t *>(&b2);
+      }
+      *reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) + (size_t)m * a.N + nb) =
+          make_uint4(w[0], w[1], w[2], w[3]);
+      if (NPROJ == 2 && a.out_f16) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) w[e] = h2bits(__floats2half2_rn(v[2 * e], v[2 * e + 1]));
+        *reinterpret_cast<uint4 *>(a.out_f16 + (size_t)m * a.ldo16 + nb) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
+  } else {
+    for (int e = 0; e < 8 && nb + e < a.N; ++e) {
+      const size_t o = (size_t)m * a.N + nb + e;
+      if (NPROJ == 1 && a.out_f32) {
+        reinterpret_cast<float *>(a.out)[o] = v[e];
+      } else {
+        reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v[e]);
+        if (NPROJ == 2 && a.out_f16) a.out_f16[(size_t)m * a.ldo16 + nb + e] = __half_as_ushort(__float2half_rn(v[e]));
+      }
+    }
+  }
+}
+
+// Shared memory of a launch: the barriers behind the rings, then the TMEM
+// base address, the abort flag and the stream-K "last part" flag.
+template <class C>
+struct GemmSmem {
+  uint8_t *base;
+  uint64_t *raw_full, *raw_empty, *a_full, *a_empty, *b_full, *b_empty, *acc_full;
+  uint32_t *tmem_s;
+  volatile int *abort_s, *last_s;
+  __device__ explicit GemmSmem(uint8_t *smem_raw) {
+    // the swizzled activation tiles need 1024-byte alignment
+    base = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    raw_full = reinterpret_cast<uint64_t *>(base + C::OFF_BAR);
+    raw_empty = raw_full + C::R;
+    a_full = raw_empty + C::R;
+    a_empty = a_full + C::SA;
+    b_full = a_empty + C::SA;
+    b_empty = b_full + C::SB;
+    acc_full = b_empty + C::SB;
+    tmem_s = reinterpret_cast<uint32_t *>(acc_full + 2);
+    abort_s = reinterpret_cast<volatile int *>(tmem_s + 1);
+    last_s = abort_s + 1;
+  }
+  // thread 0: barrier initialisation; the MMA warp: TMEM allocation
+  __device__ void init(int tid, int warp) {
+    if (tid == 0) {
+      for (int q = 0; q < C::R; ++q) {
+        mbar_init(&raw_full[q], 1);
+        mbar_init(&raw_empty[q], kDeqWarps);
+      }
+      for (int s = 0; s < C::SA; ++s) {
+        mbar_init(&a_full[s], 1);
+        mbar_init(&a_empty[s], 1);
+      }
+      for (int s = 0; s < C::SB; ++s) {
+        mbar_init(&b_full[s], kDeqWarps);
+        mbar_init(&b_empty[s], 1);
+      }
+      mbar_init(acc_full, 1);
+      *abort_s = 0;
+      fence_barrier_init();
+    }
+    if (warp == kMmaWarp) tmem_alloc(tmem_s, C::NCOLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+  }
+};
+
+// ---------------------------------------------------------------------------
+// One tile a CTA: grid (token tiles, row tiles).
+// ---------------------------------------------------------------------------
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+__global__ void __launch_bounds__(kGemmThreads, 1) qgemm_tile_kernel(const GemmArgs a, const __grid_constant__ GemmMaps tm) {
+  using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  constexpr int SA = C::SA, SB = C::SB, R = C::R, GPB = C::GPB;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  GemmSmem<C> sm(smem_raw);
+  uint8_t *smem = sm.base;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.x * a.mt * kBM, n0 = blockIdx.y * kBN;
   const int mth = min(a.mt, (a.M - m0 + kBM - 1) / kBM);  // token halves with tokens in them
@@ -156,35 +447,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   const int nws = 2 * KB;  // weight stages (64 features each)
   const int nlora = NPROJ == 2 && a.r > 0 ? (a.r + kLoraK - 1) / kLoraK : 0;
   const int nit = nws + nlora;
-
-  if (tid == 0) {
-    for (int q = 0; q < R; ++q) {
-      mbar_init(&raw_full[q], 1);
-      mbar_init(&raw_empty[q], kDeqWarps);
-    }
-    for (int s = 0; s < SA; ++s) {
-      mbar_init(&a_full[s], 1);
-      mbar_init(&a_empty[s], 1);
-    }
-    for (int s = 0; s < SB; ++s) {
-      mbar_init(&b_full[s], kDeqWarps);
-      mbar_init(&b_empty[s], 1);
-    }
-    mbar_init(acc_full, 1);
-    *abort_s = 0;
-    fence_barrier_init();
-  }
-  if (warp == kMmaWarp) tmem_alloc(tmem_s, C::NCOLS);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_s;
+  sm.init(tid, warp);
+  const uint32_t tmem = *sm.tmem_s;
 
   // bounded wait; a timeout (or an earlier one) makes the caller skip its work
   auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
-    if (*abort_s) return false;
+    if (*sm.abort_s) return false;
     if (mbar_wait_sleep(bar, parity)) return true;
-    *abort_s = 1;
+    *sm.abort_s = 1;
     if (lane == 0) gemm_timeout();
     return false;
   };
@@ -195,283 +465,353 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     if (lane == 0)
       for (int it = 0; it < KB; ++it) {
         const int q = it % R;
-        if (it >= R && !wait(&raw_empty[q], (it / R - 1) & 1)) break;
-        mbar_arrive_expect_tx(&raw_full[q], (uint32_t)C::RAW);
+        if (it >= R && !wait(&sm.raw_empty[q], (it / R - 1) & 1)) break;
+        mbar_arrive_expect_tx(&sm.raw_full[q], (uint32_t)C::RAW);
         for (int p = 0; p < NPROJ; ++p) {
           uint8_t *dst = smem + C::OFF_RAW + q * C::RAW + p * C::RAWP;
-          tma_load_3d(dst, &tm.codes[p], 0, it * (C::BPK / 128), n0 / 16, &raw_full[q]);
-          tma_load_3d(dst + 8 * C::BPK, &tm.meta[p], 0, it * GPB, n0 / 16, &raw_full[q]);
+          tma_load_3d(dst, &tm.codes[p], 0, it * (C::BPK / 128), n0 / 16, &sm.raw_full[q]);
+          tma_load_3d(dst + 8 * C::BPK, &tm.meta[p], 0, it * GPB, n0 / 16, &sm.raw_full[q]);
         }
       }
     __syncwarp();
   } else if (warp == kProducerWarp) {
-    // ---- activation tiles (TMA); the LoRA stage's by cp.async ----
+    // ---- activation tiles (TMA); the LoRA stages' by cp.async ----
     for (int it = 0; it < nit; ++it) {
       const int s = it % SA;
-      if (it >= SA && !wait(&a_empty[s], (it / SA - 1) & 1)) break;
+      if (it >= SA && !wait(&sm.a_empty[s], (it / SA - 1) & 1)) break;
       uint8_t *As = smem + C::OFF_A + s * C::AT;
       if (it < nws) {
         if (lane == 0) {
-          // activation tiles: per token half one box of 64 features x 128
-          // tokens, a 128-byte row per token, swizzled (8-row groups 1 KB apart)
-          mbar_arrive_expect_tx(&a_full[s], (uint32_t)(mth * kTileBytes));
-          for (int h = 0; h < mth; ++h) tma_load_2d(As + h * kTileBytes, &tm.act, it * 64, m0 + h * kBM, &a_full[s]);
+          // per token half one box of 64 features x 128 tokens, a 128-byte row
+          // per token, swizzled (8-row groups 1 KB apart)
+          mbar_arrive_expect_tx(&sm.a_full[s], (uint32_t)(mth * kTileBytes));
+          for (int h = 0; h < mth; ++h) tma_load_2d(As + h * kTileBytes, &tm.act, it * 64, m0 + h * kBM, &sm.a_full[s]);
         }
       } else {
-        // LoRA stage l: lora_scale * t, rank columns 32 l .. 32 l + 31 of gate
-        // (first r columns of ta) and of up (next r), zeros past r
-        const int l = it - nws;
-        for (int i = lane; i < mth * NPROJ * kBM * 4; i += 32) {
-          const int h = i / (NPROJ * kBM * 4), hr = i - h * NPROJ * kBM * 4;
-          const int p = hr / (kBM * 4), rem = hr - p * kBM * 4;
-          const int ml = rem >> 2, c = rem & 3;
-          const int m = m0 + h * kBM + ml, col = l * kLoraK + c * 8;
-          const bool ok = m < a.M && col < a.r;
-          const uint16_t *src = ok ? a.ta + (size_t)m * 2 * a.r + p * a.r + col : a.ta;
-          cp_async16_zfill(As + h * kTileBytes + p * (kBM * kLoraK * 2) + kmajor_off(ml, c * 8, 4 * 128u), src,
-                           ok ? 16u : 0u);
-        }
-        // once landed, each lane fences its generic-proxy writes against the
-        // tensor cores' reads, then lane 0 arrives
-        cp_async_wait_all();
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&a_full[s]);
+        gemm_lora_a_stage<NPROJ>(a, As, m0, mth, it - nws, lane, &sm.a_full[s]);
       }
     }
   } else if (warp == kMmaWarp) {
     // ---- MMA issue ----
     if (lane == 0) {
-      // gate/up: one MMA of N = 256 a k-step (the gate tile and the up tile
-      // are adjacent, 256 rows), so the activation tile is read once
-      constexpr uint32_t idesc = umma_idesc_f16(kBM, kBN);
-      constexpr uint32_t idesc2 = umma_idesc_f16(kBM, 2 * kBN);
       for (int it = 0; it < nit; ++it) {
         const int sa = it % SA, sb = it % SB;
-        if (!wait(&a_full[sa], (it / SA) & 1) || !wait(&b_full[sb], (it / SB) & 1)) break;
+        if (!wait(&sm.a_full[sa], (it / SA) & 1) || !wait(&sm.b_full[sb], (it / SB) & 1)) break;
         tc_fence_after();
-        const uint32_t as0 = smem_addr(smem + C::OFF_A + sa * C::AT);
-        const uint32_t bs = smem_addr(smem + C::OFF_B + sb * C::BT);
-        // every token half multiplies the same B tile into its own accumulators
-        for (int h = 0; h < mth; ++h) {
-          const uint32_t as = as0 + h * kTileBytes, th = tmem + h * C::NCH;
-          if (it < nws && NPROJ == 2 && !EXACT) {
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-              umma_f16(th, umma_desc_kmajor_sw128(as + ks * 32, 1024), umma_desc_kmajor(bs + ks * 256, 128, kSboTile),
-                       idesc2, (it > 0 || ks > 0) ? 1u : 0u);
-          } else if (it < nws) {
-#pragma unroll
-            for (int p = 0; p < NPROJ; ++p)
-#pragma unroll
-              for (int ks = 0; ks < 4; ++ks) {
-                // A (swizzled TMA layout): k-step ks at byte 32 ks of each row
-                umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
-                         umma_desc_kmajor(bs + p * kTileBytes + ks * 256, 128, kSboTile), idesc,
-                         (it > 0 || ks > 0) ? 1u : 0u);
-                if (EXACT)  // the low parts of the same weights
-                  umma_f16(th + p * kBN, umma_desc_kmajor_sw128(as + ks * 32, 1024),
-                           umma_desc_kmajor(bs + (NPROJ + p) * kTileBytes + ks * 256, 128, kSboTile), idesc, 1u);
-              }
-          } else {
-            constexpr uint32_t sbo = 4 * 128u;  // 32 rank columns a LoRA stage
-            for (int p = 0; p < NPROJ; ++p)
-              for (int ks = 0; ks < kLoraK / 16; ++ks)
-                umma_f16(th + p * kBN, umma_desc_kmajor(as + p * (kBM * kLoraK * 2) + ks * 256, 128, sbo),
-                         umma_desc_kmajor(bs + p * (kBN * kLoraK * 2) + ks * 256, 128, sbo), idesc, 1u);
-          }
-        }
+        gemm_issue_stage<NPROJ, EXACT>(tmem, smem_addr(smem + C::OFF_A + sa * C::AT),
+                                       smem_addr(smem + C::OFF_B + sb * C::BT), mth, it < nws, it == 0);
         // both slots are free once these MMAs have read them
-        umma_commit(&a_empty[sa]);
-        umma_commit(&b_empty[sb]);
+        umma_commit(&sm.a_empty[sa]);
+        umma_commit(&sm.b_empty[sb]);
       }
-      umma_commit(acc_full);
+      umma_commit(sm.acc_full);
     }
     __syncwarp();
   } else {
     // ---- dequantization into the B tiles ----
-    const int dt = tid;  // 0 .. kDeqWarps * 32 - 1
     for (int it = 0; it < nit; ++it) {
       const int s = it % SB, kb = it >> 1, hb = it & 1, q = kb % R;
-      if (it < nws && !wait(&raw_full[q], (kb / R) & 1)) break;
-      if (it >= SB && !wait(&b_empty[s], (it / SB - 1) & 1)) break;
+      if (it < nws && !wait(&sm.raw_full[q], (kb / R) & 1)) break;
+      if (it >= SB && !wait(&sm.b_empty[s], (it / SB - 1) & 1)) break;
       uint8_t *Bs = smem + C::OFF_B + s * C::BT;
-      if (it < nws) {
-        const uint8_t *raw = smem + C::OFF_RAW + q * C::RAW;
-        // item = (projection, 16-row tile, lane of the packed fragment layout)
-        for (int item = dt; item < NPROJ * 8 * 32; item += kDeqWarps * 32) {
-          const int p = item >> 8, j = (item >> 5) & 7, L = item & 31;
-          const int g = L >> 2, t = L & 3;
-          uint8_t *Bp = Bs + p * kTileBytes;
-          // the lane's code words of this half block: 2-bit, words 2 hb, 2 hb + 1
-          // of its 16 bytes; 4-bit, the 16 bytes of half hb
-          uint32_t wds[BITS == 2 ? 2 : 4];
-          const uint8_t *cb = raw + p * C::RAWP + j * C::BPK;               // codes of tile j
-          const uint8_t *mb = raw + p * C::RAWP + 8 * C::BPK + j * GPB * 64;  // its scales/zeros
-          if (BITS == 2) {
-            const uint2 w0 = lds64(cb + L * 16 + hb * 8);
-            wds[0] = w0.x; wds[1] = w0.y;
-          } else {
-            const uint4 w0 = lds128(cb + hb * 512 + L * 16);
-            wds[0] = w0.x; wds[1] = w0.y; wds[2] = w0.z; wds[3] = w0.w;
-          }
-          // this stage: k-steps 4 hb .. 4 hb + 3 of the block
-#pragma unroll
-          for (int gl = 0; gl < (GS >= 4 ? 1 : 4 / GS); ++gl) {
-            const int gi = (4 * hb) / GS + gl;
-            // scales and zeros of rows g and g + 8 in group gi (zero for tiles outside the matrix)
-            const uint2 sz = lds64(mb + gi * 64 + g * 8);
-            // scales of rows g ("lo" row) and g + 8 ("hi" row); EXACT splits each
-            // into a head with the 4 lowest mantissa bits cleared and the tail
-            const uint32_t sg = sz.x & 0xffffu, sg8 = sz.x >> 16;
-            const __half2 s_lo = __half2half2(__ushort_as_half((unsigned short)(EXACT ? (sg & 0xfff0u) : sg)));
-            const __half2 s_hi = __half2half2(__ushort_as_half((unsigned short)(EXACT ? (sg8 & 0xfff0u) : sg8)));
-            const __half2 t_lo = __half2half2(__hsub(__ushort_as_half((unsigned short)sg), __ushort_as_half((unsigned short)(sg & 0xfff0u))));
-            const __half2 t_hi = __half2half2(__hsub(__ushort_as_half((unsigned short)sg8), __ushort_as_half((unsigned short)(sg8 & 0xfff0u))));
-            // 1024 + z: the code read as 1024 + q minus this is q - z exactly
-            const __half2 z_lo = __half2half2(__hadd(__ushort_as_half((unsigned short)(sz.y & 0xffffu)), __float2half(1024.f)));
-            const __half2 z_hi = __half2half2(__hadd(__ushort_as_half((unsigned short)(sz.y >> 16)), __float2half(1024.f)));
-#pragma unroll
-            for (int kk = 0; kk < (GS >= 4 ? 4 : GS); ++kk) {
-              const int ks = (GS >= 4 ? 4 * hb : gi * GS) + kk;
-              uint32_t q[4];  // (row g, k 2t..2t+1), (row g+8, ...), (row g, k 2t+8..), (row g+8, k 2t+8..)
-              const int kl = ks - 4 * hb;  // k-step within the half block
-              if (BITS == 2) {
-                const uint32_t x = wds[(kl >> 1) & 1];
-                const int s4 = (kl & 1) * 4;
-                q[0] = (x >> s4) & 0x00030003u;
-                q[1] = (x >> (s4 + 8)) & 0x00030003u;
-                q[2] = (x >> (s4 + 2)) & 0x00030003u;
-                q[3] = (x >> (s4 + 10)) & 0x00030003u;
-              } else {
-                const uint32_t x = wds[kl & 3];
-                q[0] = x & 0x000F000Fu;
-                q[1] = (x >> 8) & 0x000F000Fu;
-                q[2] = (x >> 4) & 0x000F000Fu;
-                q[3] = (x >> 12) & 0x000F000Fu;
-              }
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const __half2 v = bits2h(q[e] | 0x64006400u);  // 1024 + q, exact
-                const bool hi_row = (e & 1) != 0;
-                const __half2 qz = __hsub2(v, hi_row ? z_hi : z_lo);  // q - z, exact
-                const __half2 w = __hmul2(qz, hi_row ? s_hi : s_lo);
-                const int row = j * 16 + g + (hi_row ? 8 : 0);
-                const int k = kl * 16 + 2 * t + ((e & 2) ? 8 : 0);  // within the stage
-                *reinterpret_cast<uint32_t *>(Bp + kmajor_off(row, k, kSboTile)) = h2bits(w);
-                if (EXACT)
-                  *reinterpret_cast<uint32_t *>(Bp + NPROJ * kTileBytes + kmajor_off(row, k, kSboTile)) =
-                      h2bits(__hmul2(qz, hi_row ? t_hi : t_lo));
-              }
-            }
-          }
-        }
-      } else {
-        // LoRA stage l: B_p rows n0 .. n0+127 (bf16 [N][r]), rank columns
-        // 32 l .. 32 l + 31 -> binary16, zeros past r
-        const int l = it - nws;
-        constexpr uint32_t sbo = 4 * 128u;
-        for (int i = dt; i < NPROJ * kBN * 4; i += kDeqWarps * 32) {
-          const int p = i / (kBN * 4), rem = i - p * kBN * 4;
-          const int nl = rem >> 2, c = rem & 3;
-          const int n = n0 + nl, col = l * kLoraK + c * 8;
-          uint4 v = make_uint4(0u, 0u, 0u, 0u);
-          if (n < a.N && col < a.r) v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_b[p]) + ((size_t)n * a.r + col) * 2));
-          const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-          uint32_t o[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
-            o[e] = h2bits(__floats2half2_rn(lo, hi));
-          }
-          *reinterpret_cast<uint4 *>(Bs + p * (kBN * kLoraK * 2) + kmajor_off(nl, c * 8, sbo)) = make_uint4(o[0], o[1], o[2], o[3]);
-        }
-      }
+      if (it < nws)
+        gemm_deq_stage<BITS, NPROJ, GROUP, EXACT>(smem + C::OFF_RAW + q * C::RAW, Bs, hb, tid);
+      else
+        gemm_lora_b_stage<NPROJ>(a, Bs, n0, it - nws, tid);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
-        mbar_arrive(&b_full[s]);
-        if (it < nws && hb == 1) mbar_arrive(&raw_empty[q]);  // both halves of this block's codes are read
+        mbar_arrive(&sm.b_full[s]);
+        if (it < nws && hb == 1) mbar_arrive(&sm.raw_empty[q]);  // both halves of this block's codes are read
       }
     }
 
     // ---- epilogue: warp w reads TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31
     // (the tokens of each half) and columns 32 (w / 4) .. 32 (w / 4) + 31 ----
-    if (wait(acc_full, 0)) {
+    if (wait(sm.acc_full, 0)) {
       tc_fence_after();
       const int quarter = warp & 3, c0 = (warp >> 2) * 32;
+      const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
       for (int h = 0; h < mth; ++h) {
         const int m = m0 + h * kBM + quarter * 32 + lane;
         const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
         const uint32_t tl = tmem + h * C::NCH + ((uint32_t)(quarter * 32) << 16);
-        // rows n0 + c .. n0 + c + 7 of this token: 16-byte stores when the
-        // row length allows (N a multiple of 8), element stores otherwise
-        const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
         for (int c = c0; c < c0 + 32; c += 8) {
-          uint32_t g[8], uu[8];
-          tmem_ld8(tl + c, g);
-          if (NPROJ == 2) tmem_ld8(tl + kBN + c, uu);
+          uint32_t gw[8], uw[8];
+          tmem_ld8(tl + c, gw);
+          if (NPROJ == 2) tmem_ld8(tl + kBN + c, uw);
           tmem_ld_wait();
-          const int nb = n0 + c;
-          if (m >= a.M || nb >= a.N) continue;
-          float v[8];
-          if (NPROJ == 2) {
-  #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float gv = rs * __uint_as_float(g[e]), uv = rs * __uint_as_float(uu[e]);
-              v[e] = __bfloat162float(__float2bfloat16_rn(gv / (1.f + __expf(-gv)) * uv));  // h as stored
-            }
-          } else {
-  #pragma unroll
-            for (int e = 0; e < 8; ++e) v[e] = __uint_as_float(g[e]);
-            if (a.residual) {
-              if (vec) {
-                const uint4 rv = *reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.residual) +
-                                                                  (size_t)m * a.N + nb);
-                const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
-  #pragma unroll
-                for (int e = 0; e < 8; ++e) v[e] += __uint_as_float(e & 1 ? (rw[e >> 1] & 0xffff0000u) : (rw[e >> 1] << 16));
-              } else {
-                for (int e = 0; e < 8 && nb + e < a.N; ++e)
-                  v[e] += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[(size_t)m * a.N + nb + e]);
-              }
-            }
+          float g[8], u[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            g[e] = __uint_as_float(gw[e]);
+            u[e] = NPROJ == 2 ? __uint_as_float(uw[e]) : 0.f;
           }
-          if (vec) {
-            if (NPROJ == 1 && a.out_f32) {
-              float4 *o = reinterpret_cast<float4 *>(reinterpret_cast<float *>(a.out) + (size_t)m * a.N + nb);
-              o[0] = make_float4(v[0], v[1], v[2], v[3]);
-              o[1] = make_float4(v[4], v[5], v[6], v[7]);
-            } else {
-              uint32_t w[4];
-  #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-                w[e] = *reinterpret_cast<const uint32_t *>(&b2);
-              }
-              *reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) + (size_t)m * a.N + nb) =
-                  make_uint4(w[0], w[1], w[2], w[3]);
-              if (NPROJ == 2 && a.out_f16) {
-  #pragma unroll
-                for (int e = 0; e < 4; ++e) w[e] = h2bits(__floats2half2_rn(v[2 * e], v[2 * e + 1]));
-                *reinterpret_cast<uint4 *>(a.out_f16 + (size_t)m * a.ldo16 + nb) = make_uint4(w[0], w[1], w[2], w[3]);
-              }
-            }
-          } else {
-            for (int e = 0; e < 8 && nb + e < a.N; ++e) {
-              const size_t o = (size_t)m * a.N + nb + e;
-              if (NPROJ == 1 && a.out_f32) {
-                reinterpret_cast<float *>(a.out)[o] = v[e];
-              } else {
-                reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v[e]);
-                if (NPROJ == 2 && a.out_f16) a.out_f16[(size_t)m * a.ldo16 + nb + e] = __half_as_ushort(__float2half_rn(v[e]));
-              }
-            }
-          }
+          gemm_finish<NPROJ>(a, m, n0 + c, rs, g, u, vec);
         }
       }
     }
   }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == kMmaWarp) tmem_dealloc(tmem, C::NCOLS);
+}
+
+// ---------------------------------------------------------------------------
+// Stream-K: gridDim.x persistent CTAs divide the T * U work units evenly.
+// ---------------------------------------------------------------------------
+// The tiles (mt * 128 tokens x 128 rows) are cut into units of one
+// 128-feature block (plus one unit for the LoRA stages); CTA c takes units
+// [c W / P, (c + 1) W / P) of the W = T * U in order, i.e. whole tiles and at
+// most one part of a tile at each end of its range.
+
+// The epilogue of one part of a tile (the 16 dequantizing warps, after the
+// part's accumulators are complete; `have`: no timeout so far).  Warp w reads
+// TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the tokens of each half) and
+// columns 32 (w / 4) .. 32 (w / 4) + 31.  A whole tile is finished from TMEM;
+// a part of a split tile is written to its scratch slot, and the CTA that adds
+// the tile's last part to its counter sums the parts in k order (their CTAs
+// are consecutive) and finishes the tile.  Kept out of line so that the
+// dequantization loop keeps its registers.
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+__device__ __noinline__ void gemm_part_epilogue(const GemmArgs &a, uint32_t tmem, int tile, int ub, int ue, int U,
+                                                long long W, long long P, long long g0, bool have,
+                                                volatile int *abort_s, volatile int *last_s) {
+  using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int quarter = warp & 3, c0 = (warp >> 2) * 32;
+  const int MT = (a.M + a.mt * kBM - 1) / (a.mt * kBM);
+  const int m0 = (tile % MT) * a.mt * kBM, n0 = (tile / MT) * kBN;
+  const int mth = min(a.mt, (a.M - m0 + kBM - 1) / kBM);
+  const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
+  constexpr int SLOT = kHalves * kBM * C::NCH;  // floats of a scratch slot: [half][NCH / 8][128 tokens][8]
+  const bool whole = ub == 0 && ue == U;
+  // a split part's scratch slot: the CTA's first part (0) or its last (1)
+  float *mine = whole ? nullptr : a.sk_part + ((size_t)blockIdx.x * 2 + ((long long)tile * U + ub == g0 ? 0 : 1)) * SLOT;
+  for (int h = 0; h < mth && have; ++h) {
+    const int m = m0 + h * kBM + quarter * 32 + lane;
+    const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+    const uint32_t tl = tmem + h * C::NCH + ((uint32_t)(quarter * 32) << 16);
+    for (int c = c0; c < c0 + 32; c += 8) {
+      uint32_t gw[8], uw[8];
+      tmem_ld8(tl + c, gw);
+      if (NPROJ == 2) tmem_ld8(tl + kBN + c, uw);
+      tmem_ld_wait();
+      float g[8], u[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        g[e] = __uint_as_float(gw[e]);
+        u[e] = NPROJ == 2 ? __uint_as_float(uw[e]) : 0.f;
+      }
+      if (whole) {
+        gemm_finish<NPROJ>(a, m, n0 + c, rs, g, u, vec);
+      } else {
+        // fp32 partial sums, 32 bytes a (token, 8 columns): lanes contiguous
+        float4 *pg = reinterpret_cast<float4 *>(mine + (((size_t)h * (C::NCH / 8) + c / 8) * kBM + quarter * 32 + lane) * 8);
+        __stcg(pg, make_float4(g[0], g[1], g[2], g[3]));
+        __stcg(pg + 1, make_float4(g[4], g[5], g[6], g[7]));
+        if (NPROJ == 2) {
+          float4 *pu = reinterpret_cast<float4 *>(
+              mine + (((size_t)h * (C::NCH / 8) + (kBN + c) / 8) * kBM + quarter * 32 + lane) * 8);
+          __stcg(pu, make_float4(u[0], u[1], u[2], u[3]));
+          __stcg(pu + 1, make_float4(u[4], u[5], u[6], u[7]));
+        }
+      }
+    }
+  }
+  if (whole) return;
+  // the tile's parts lie in CTAs c_lo .. c_hi; the one that brings the
+  // counter to their number sums them and finishes the tile
+  const long long t0u = (long long)tile * U;
+  const int c_lo = (int)(((t0u + 1) * P + W - 1) / W - 1), c_hi = (int)(((t0u + U) * P + W - 1) / W - 1);
+  named_barrier_sync(1, kDeqWarps * 32);
+  if (tid == 0) {
+    int last = 0;
+    if (!*abort_s) {
+      __threadfence();
+      last = atomicAdd(&a.sk_cnt[tile], 1u) == (unsigned)(c_hi - c_lo) ? 1 : 0;
+      if (last) {
+        a.sk_cnt[tile] = 0;  // ready for the next launch
+        __threadfence();
+      }
+    }
+    *last_s = last;
+  }
+  named_barrier_sync(1, kDeqWarps * 32);
+  if (!*last_s) return;
+  for (int h = 0; h < mth; ++h) {
+    const int m = m0 + h * kBM + quarter * 32 + lane;
+    const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+    for (int c = c0; c < c0 + 32; c += 8) {
+      float g[8], u[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) g[e] = u[e] = 0.f;
+      for (int cc = c_lo; cc <= c_hi; ++cc) {
+        // CTA cc's part of this tile is its first (slot 0) unless the tile began inside its range
+        const float *src = a.sk_part + ((size_t)cc * 2 + (t0u <= W * cc / P ? 0 : 1)) * SLOT;
+        const float4 *pg =
+            reinterpret_cast<const float4 *>(src + (((size_t)h * (C::NCH / 8) + c / 8) * kBM + quarter * 32 + lane) * 8);
+        const float4 g0v = __ldcg(pg), g1v = __ldcg(pg + 1);
+        g[0] += g0v.x; g[1] += g0v.y; g[2] += g0v.z; g[3] += g0v.w;
+        g[4] += g1v.x; g[5] += g1v.y; g[6] += g1v.z; g[7] += g1v.w;
+        if (NPROJ == 2) {
+          const float4 *pu = reinterpret_cast<const float4 *>(
+              src + (((size_t)h * (C::NCH / 8) + (kBN + c) / 8) * kBM + quarter * 32 + lane) * 8);
+          const float4 u0v = __ldcg(pu), u1v = __ldcg(pu + 1);
+          u[0] += u0v.x; u[1] += u0v.y; u[2] += u0v.z; u[3] += u0v.w;
+          u[4] += u1v.x; u[5] += u1v.y; u[6] += u1v.z; u[7] += u1v.w;
+        }
+      }
+      gemm_finish<NPROJ>(a, m, n0 + c, rs, g, u, vec);
+    }
+  }
+}
+
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+__global__ void __launch_bounds__(kGemmThreads, 1) qgemm_sk_kernel(const __grid_constant__ GemmArgs a,
+                                                                   const __grid_constant__ GemmMaps tm) {
+  using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  constexpr int SA = C::SA, SB = C::SB, R = C::R, GPB = C::GPB;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  GemmSmem<C> sm(smem_raw);
+  uint8_t *smem = sm.base;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int KB = (a.K + 127) / 128;
+  const int nlora = NPROJ == 2 && a.r > 0 ? (a.r + kLoraK - 1) / kLoraK : 0;
+  const int U = KB + (nlora > 0 ? 1 : 0);
+  const int MT = (a.M + a.mt * kBM - 1) / (a.mt * kBM), NT = (a.N + kBN - 1) / kBN;
+  const long long W = (long long)MT * NT * U, P = gridDim.x;
+  const long long g0 = W * blockIdx.x / P, g1 = W * (blockIdx.x + 1) / P;
+  sm.init(tid, warp);
+  const uint32_t tmem = *sm.tmem_s;
+
+  auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
+    if (*sm.abort_s) return false;
+    if (mbar_wait_sleep(bar, parity)) return true;
+    *sm.abort_s = 1;
+    if (lane == 0) gemm_timeout();
+    return false;
+  };
+  // The parts of tiles in this CTA's range, in order: tile, units [ub, ue),
+  // weight blocks wb, stages nit (two a block, then the LoRA stages); token
+  // tiles vary fastest, so neighbouring CTAs share row tiles.
+#define WQ_FOR_EACH_PART                                                         \
+  for (long long g_ = g0; g_ < g1;)                                              \
+    for (int tile = (int)(g_ / U), ub = (int)(g_ - (long long)tile * U),         \
+             ue = (int)min((long long)U, ub + (g1 - g_)), wb = min(ue, KB) - ub, \
+             nit = 2 * wb + (ue > KB ? nlora : 0), once_ = (g_ += ue - ub, 1);   \
+         once_; once_ = 0)
+  auto tile_m0 = [&](int tile) { return (tile % MT) * a.mt * kBM; };
+  auto halves = [&](int m0) { return min(a.mt, (a.M - m0 + kBM - 1) / kBM); };
+
+  if (warp == kRawWarp) {
+    if (lane == 0) {
+      int gr = 0;  // blocks loaded so far
+      bool ok = true;
+      WQ_FOR_EACH_PART {
+        (void)nit;  // the codes ring follows the blocks only
+        const int n0 = (tile / MT) * kBN;
+        for (int kb = ub; kb < ub + wb && ok; ++kb, ++gr) {
+          const int q = gr % R;
+          if (gr >= R && !wait(&sm.raw_empty[q], (gr / R - 1) & 1)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&sm.raw_full[q], (uint32_t)C::RAW);
+          for (int p = 0; p < NPROJ; ++p) {
+            uint8_t *dst = smem + C::OFF_RAW + q * C::RAW + p * C::RAWP;
+            tma_load_3d(dst, &tm.codes[p], 0, kb * (C::BPK / 128), n0 / 16, &sm.raw_full[q]);
+            tma_load_3d(dst + 8 * C::BPK, &tm.meta[p], 0, kb * GPB, n0 / 16, &sm.raw_full[q]);
+          }
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == kProducerWarp) {
+    int gs = 0;  // stages so far
+    bool ok = true;
+    WQ_FOR_EACH_PART {
+      const int m0 = tile_m0(tile), mth = halves(m0);
+      for (int it = 0; it < nit && ok; ++it, ++gs) {
+        const int s = gs % SA;
+        if (gs >= SA && !wait(&sm.a_empty[s], (gs / SA - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        uint8_t *As = smem + C::OFF_A + s * C::AT;
+        if (it < 2 * wb) {
+          if (lane == 0) {
+            mbar_arrive_expect_tx(&sm.a_full[s], (uint32_t)(mth * kTileBytes));
+            for (int h = 0; h < mth; ++h)
+              tma_load_2d(As + h * kTileBytes, &tm.act, (ub + (it >> 1)) * 128 + (it & 1) * 64, m0 + h * kBM,
+                          &sm.a_full[s]);
+          }
+        } else {
+          gemm_lora_a_stage<NPROJ>(a, As, m0, mth, it - 2 * wb, lane, &sm.a_full[s]);
+        }
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      int gs = 0;
+      bool ok = true;
+      WQ_FOR_EACH_PART {
+        if (!ok) break;
+        const int mth = halves(tile_m0(tile));
+        for (int it = 0; it < nit; ++it, ++gs) {
+          const int sa = gs % SA, sb = gs % SB;
+          if (!wait(&sm.a_full[sa], (gs / SA) & 1) || !wait(&sm.b_full[sb], (gs / SB) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          gemm_issue_stage<NPROJ, EXACT>(tmem, smem_addr(smem + C::OFF_A + sa * C::AT),
+                                         smem_addr(smem + C::OFF_B + sb * C::BT), mth, it < 2 * wb, it == 0);
+          umma_commit(&sm.a_empty[sa]);
+          umma_commit(&sm.b_empty[sb]);
+        }
+        if (ok) umma_commit(sm.acc_full);  // the part's accumulators are complete
+      }
+    }
+    __syncwarp();
+  } else {
+    // dequantization, then each part's epilogue; a warp that met a timeout
+    // skips its work but still passes the epilogue's named barriers
+    int gs = 0, gr = 0, part = 0;
+    bool ok = true;
+    WQ_FOR_EACH_PART {
+      const int n0 = (tile / MT) * kBN;
+      for (int it = 0; it < nit; ++it, ++gs) {
+        const int s = gs % SB, hb = it & 1, kr = gr + (it >> 1), q = kr % R;
+        const bool wstage = it < 2 * wb;
+        if (ok && wstage && !wait(&sm.raw_full[q], (kr / R) & 1)) ok = false;
+        if (ok && gs >= SB && !wait(&sm.b_empty[s], (gs / SB - 1) & 1)) ok = false;
+        if (!ok) continue;
+        uint8_t *Bs = smem + C::OFF_B + s * C::BT;
+        if (wstage)
+          gemm_deq_stage<BITS, NPROJ, GROUP, EXACT>(smem + C::OFF_RAW + q * C::RAW, Bs, hb, tid);
+        else
+          gemm_lora_b_stage<NPROJ>(a, Bs, n0, it - 2 * wb, tid);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&sm.b_full[s]);
+          if (wstage && hb == 1) mbar_arrive(&sm.raw_empty[q]);  // both halves of this block's codes are read
+        }
+      }
+      gr += wb;
+      const bool have = ok && wait(sm.acc_full, part & 1);
+      ++part;
+      tc_fence_after();
+      gemm_part_epilogue<BITS, NPROJ, GROUP, EXACT>(a, tmem, tile, ub, ue, U, W, P, g0, have, sm.abort_s, sm.last_s);
+      // the next part's MMAs overwrite the accumulators only after this warp's
+      // b_full arrival, which follows its TMEM reads
+      tc_fence_before();
+    }
+  }
+#undef WQ_FOR_EACH_PART
 
   tc_fence_before();
   __syncthreads();
@@ -669,27 +1009,62 @@ cudaError_t make_maps(const GemmArgs &a, int nproj, int bits, GemmMaps *m) {
   return cudaSuccess;
 }
 
+cudaError_t num_sms_cached(int *sms) {
+  static int cached[64] = {0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (cached[dev] == 0 && (e = cudaDeviceGetAttribute(&cached[dev], cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return e;
+  *sms = cached[dev];
+  return cudaSuccess;
+}
+
+// Work split of a launch.  A CTA takes two token halves (each weight
+// dequantized once for 256 tokens) whenever there are more than 128 tokens.
+// Tiles are mt * 128 tokens x 128 rows, U work units each (128-feature
+// blocks, plus one for the LoRA stages).  One CTA per tile when the last wave
+// of CTAs is at least 80% full; otherwise stream-K: P CTAs (one per SM at
+// most, 4 units each at least) divide the T * U units evenly.
+struct GemmSched {
+  int mt, T, U, P;
+  bool sk;
+};
+GemmSched gemm_schedule(int M, int N, int K, int nproj, int r, int sms) {
+  GemmSched g;
+  g.mt = M > kBM ? 2 : 1;
+  g.T = (M + g.mt * kBM - 1) / (g.mt * kBM) * ((N + kBN - 1) / kBN);
+  g.U = (K + 127) / 128 + (nproj == 2 && r > 0 ? 1 : 0);
+  const long long W = (long long)g.T * g.U;
+  const int waves = (g.T + sms - 1) / sms;
+  g.sk = 10LL * g.T < 8LL * waves * sms && W >= 8;
+  g.P = g.sk ? (int)std::max(1LL, std::min((long long)sms, W / 4)) : g.T;
+  return g;
+}
+
 template <int BITS, int NPROJ, int GROUP, bool EXACT>
 cudaError_t launch_gemm_t(const GemmArgs &a, cudaStream_t s) {
   using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
-  auto kern = qgemm_kernel<BITS, NPROJ, GROUP, EXACT>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  auto tile_kern = qgemm_tile_kernel<BITS, NPROJ, GROUP, EXACT>;
+  auto sk_kern = qgemm_sk_kernel<BITS, NPROJ, GROUP, EXACT>;
+  cudaError_t e = cudaFuncSetAttribute(tile_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(sk_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   GemmMaps maps;
   if ((e = make_maps(a, NPROJ, BITS, &maps)) != cudaSuccess) return e;
-  // two token halves a CTA (the B tile dequantized once for 256 tokens) when
-  // that still gives every SM a CTA; one otherwise
-  static int sms = 0;
-  if (sms == 0) {
-    int dev = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  }
-  const int nt = (a.N + kBN - 1) / kBN;
+  int sms = 0;
+  if ((e = num_sms_cached(&sms)) != cudaSuccess) return e;
+  const GemmSched g = gemm_schedule(a.M, a.N, a.K, NPROJ, a.r, sms);
   GemmArgs ka = a;
-  ka.mt = (a.M + 2 * kBM - 1) / (2 * kBM) * nt >= sms ? 2 : 1;
-  const dim3 grid((a.M + ka.mt * kBM - 1) / (ka.mt * kBM), nt);
-  kern<<<grid, kGemmThreads, C::SMEM, s>>>(ka, maps);
+  ka.mt = g.mt;
+  if (g.sk && a.sk_part && a.sk_cnt) {
+    sk_kern<<<g.P, kGemmThreads, C::SMEM, s>>>(ka, maps);
+  } else {
+    ka.sk_part = nullptr;
+    ka.sk_cnt = nullptr;
+    tile_kern<<<dim3((a.M + g.mt * kBM - 1) / (g.mt * kBM), (a.N + kBN - 1) / kBN), kGemmThreads, C::SMEM, s>>>(ka, maps);
+  }
   return cudaGetLastError();
 }
 
@@ -712,6 +1087,14 @@ cudaError_t launch_gemm(GemvKind kind, const GemmArgs &a, cudaStream_t s) {
     default: return a.out_f32 ? launch_gemm_g<4, 1, true>(a, s) : launch_gemm_g<4, 1, false>(a, s);
   }
 }
+
+size_t gemm_scratch_floats(int M, int N, int K, int nproj, int num_sms) {
+  if (M <= 0 || N <= 0 || K <= 0 || num_sms <= 0) return 0;
+  const GemmSched g = gemm_schedule(M, N, K, nproj, kMaxRank, num_sms);
+  return g.sk ? (size_t)2 * g.P * kHalves * kBM * nproj * kBN : 0;
+}
+
+size_t gemm_counters(int M, int N) { return (size_t)((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN); }
 
 cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void *lora_a, int r2, float lora_scale,
                              uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t s) {

@@ -104,6 +104,10 @@ struct GemmArgs {
   uint16_t *out_f16;         // gate/up: h also as binary16 [M][ldo16] (the down GEMM's A), or null
   int ldo16;
   int mt;                    // token halves of 128 per CTA (1 or 2; set by launch_gemm)
+  // stream-K scratch (null: one CTA per tile): gemm_scratch_floats() fp32 and
+  // gemm_counters() arrival counters, zero between launches
+  float *sk_part;
+  unsigned *sk_cnt;
 };
 cudaError_t launch_gemm(GemvKind kind, const GemmArgs &args, cudaStream_t stream);
 // x16 [M][lda16] = binary16(x), rs[m] = 1/sqrt(mean(x^2) + eps), ta [M][r2] = lora_scale * x A^T (r2 > 0)
@@ -111,6 +115,10 @@ cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void 
                              uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t stream);
 // x16 [M][lda16] = binary16(x) (zero padded)
 cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, cudaStream_t stream);
+// Stream-K scratch a GEMM launch of this shape can need: fp32 partial sums
+// and per-tile arrival counters (num_sms: the device's SM count).
+size_t gemm_scratch_floats(int M, int N, int K, int nproj, int num_sms);
+size_t gemm_counters(int M, int N);
 int gemm_stages(GemvKind kind, int group);  // depth of the activation-tile ring
 // Reads and clears the GEMM kernels' device status word.
 cudaError_t read_gemm_status(int *status);
