@@ -210,19 +210,23 @@ __device__ __forceinline__ void gemm_deq_stage(const uint8_t *raw, uint8_t *Bs, 
           q[2] = (x >> 4) & 0x000F000Fu;
           q[3] = (x >> 12) & 0x000F000Fu;
         }
+        uint32_t w[4], wl[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const __half2 v = bits2h(q[e] | 0x64006400u);  // 1024 + q, exact
           const bool hi_row = (e & 1) != 0;
           const __half2 qz = __hsub2(v, hi_row ? z_hi : z_lo);  // q - z, exact
-          const __half2 w = __hmul2(qz, hi_row ? s_hi : s_lo);
-          const int row = j * 16 + g + (hi_row ? 8 : 0);
-          const int k = kl * 16 + 2 * t + ((e & 2) ? 8 : 0);  // within the stage
-          *reinterpret_cast<uint32_t *>(Bp + kmajor_off(row, k, kSboTile)) = h2bits(w);
-          if (EXACT)
-            *reinterpret_cast<uint32_t *>(Bp + NPROJ * kTileBytes + kmajor_off(row, k, kSboTile)) =
-                h2bits(__hmul2(qz, hi_row ? t_hi : t_lo));
+          w[e] = h2bits(__hmul2(qz, hi_row ? s_hi : s_lo));
+          if (EXACT) wl[e] = h2bits(__hmul2(qz, hi_row ? t_hi : t_lo));
         }
+        // the four 8x8 blocks (rows +0/+8, k +0/+8) of this k-step are core
+        // matrices of the K-major tile: one matrix store; lane L gives row
+        // L % 8 of block L / 8
+        const int blk = L >> 3;
+        const uint32_t dst = smem_addr(Bp) + (uint32_t)(2 * j + (blk & 1)) * kSboTile +
+                             (uint32_t)(2 * kl + (blk >> 1)) * 128u + (uint32_t)(L & 7) * 16u;
+        stmatrix_x4(dst, w[0], w[1], w[2], w[3]);
+        if (EXACT) stmatrix_x4(dst + NPROJ * kTileBytes, wl[0], wl[1], wl[2], wl[3]);
       }
     }
   }
