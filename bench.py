@@ -12,9 +12,12 @@ Reported besides the step rate: the fused 2-bit gate/up call and the 4-bit
 down call timed on their own (36 distinct layers back to back, one graph) for
 the HBM roofline, the uniform-W4 stack on the same GPU (speedup, Gain%), the
 end-to-end rate through the C ABI with host buffers, SM clocks sampled during
-the timed region, and the CPU oracle on a bounded sample.
+the timed region, the CPU oracle on a bounded sample, and the prefill leg: a
+512-token chunk through 14B-shaped layers (d=5120, inter=17408, LoRA rank 32),
+which runs on the tcgen05 dequant-GEMM path, against the tensor roofline.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl wq|reference]
+  python bench.py --leg prefill --eager --steps 2 --warmup 1   (launches only, for ncu)
 """
 from __future__ import annotations
 
@@ -49,6 +52,9 @@ def parse():
     ap.add_argument("--no-extras", action="store_true", help="skip the comparator / per-kernel / CPU legs")
     ap.add_argument("--eager", action="store_true",
                     help="profiling aid: run the stack with plain stream launches (no CUDA graph), print no JSON")
+    ap.add_argument("--leg", default="decode", choices=["decode", "prefill"],
+                    help="with --eager: which stack to run (the decode stack or the prefill chunk)")
+    ap.add_argument("--prefill-layers", type=int, default=4, help="distinct 14B-shaped layers of the prefill leg")
     return ap.parse_args()
 
 
@@ -90,6 +96,16 @@ def measured_peaks():
             d = json.load(f)
         return float(d["hbm_gbs"]), "measured"
     return 6800.0, "fallback"
+
+
+def measured_tensor_peak():
+    """Dense bf16 (= binary16) tensor TFLOP/s: the burst figure, for a kernel timed on its own."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), "measured"
+    return 1900.0, "fallback"
 
 
 class ClockSampler:
@@ -159,15 +175,30 @@ def algorithmic_bytes(cfg, m, bits_gu=2, lora=True):
     return gateup, down
 
 
-def source_sha():
+PREFILL_CONFIG, PREFILL_M = "dense_14b", 512
+
+
+def prefill_flops(cfg, m):
+    """Algorithmic flops of one layer on m tokens: the gate and up products
+    with their adapters (x A^T, then t B^T for both), and the down product."""
+    gateup = 2 * 2 * m * cfg.d * cfg.inter + 2 * m * cfg.d * 2 * cfg.r + 2 * 2 * m * cfg.r * cfg.inter
+    down = 2 * m * cfg.inter * cfg.d
+    return gateup, down
+
+
+GEMV_SOURCES = ("wq_gemv.cu", "wq_ptx.cuh", "wq_internal.h")
+GEMM_SOURCES = ("wq_gemm.cu", "wq_ptx.cuh", "wq_internal.h")
+
+
+def source_sha(files=GEMV_SOURCES):
     h = hashlib.sha256()
-    for fn in ("wq_gemv.cu", "wq_ptx.cuh", "wq_internal.h"):
+    for fn in files:
         with open(os.path.join(ROOT, "paper_2606_04238_gb300", "csrc", fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel):
+def recorded_traffic(kernel, files=GEMV_SOURCES):
     """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
@@ -175,7 +206,7 @@ def recorded_traffic(kernel):
     with open(p) as f:
         d = json.load(f)
     e = d.get(kernel)
-    if not e or e.get("source_sha") != source_sha():
+    if not e or e.get("source_sha") != source_sha(files):
         return None
     return e.get("dram_bytes_per_launch")
 
@@ -286,6 +317,9 @@ def run_gpu(args):
     n_layers = args.layers or cfg.layers
     m = args.m
     steps, warmup = max(1, args.steps), max(3, args.warmup)
+    if args.eager and args.leg == "prefill":
+        run_prefill(wq, synth, dev, args.prefill_layers, steps, warmup, eager=True)
+        return
 
     layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
     table = wq.LayerTable(layers)
@@ -384,11 +418,78 @@ def run_gpu(args):
                                                        "Device A (50 TOPs, 100 GB/s) / Device B (200 GB/s)"}
         del w4, g4
         torch.cuda.empty_cache()
+        out["prefill"] = run_prefill(wq, synth, dev, args.prefill_layers, max(20, min(steps, 200)), warmup)
+        torch.cuda.empty_cache()
         out["cpu_baseline"] = cpu_oracle_sample(cfg, m)
 
     if rank == 0:
         print(json.dumps(out))
     barrier(ws_)
+
+
+def run_prefill(wq, synth, dev, n_layers, steps, warmup, eager=False):
+    """A 512-token chunk through n_layers distinct 14B-shaped layers (the
+    tcgen05 dequant-GEMM path): whole-stack rate, then the gate/up and the
+    down calls timed on their own for the tensor roofline."""
+    import torch
+    cfg = synth.CONFIGS[PREFILL_CONFIG]
+    m = PREFILL_M
+    layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
+    ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
+    x = synth.activations((m, cfg.d), 512, device=dev)
+    y = torch.empty_like(x)
+
+    def stack():
+        wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws)
+
+    if eager:
+        for _ in range(warmup + steps):
+            stack()
+        torch.cuda.synchronize()
+        assert wq.device_status() == 0
+        print(f"eager: {warmup + steps} prefill steps of {n_layers} layers done", flush=True)
+        return None
+    ms, clocks = time_graph(capture(stack), steps, warmup, 1, ClockSampler(dev.index or 0))
+    h = torch.empty((m, cfg.inter), dtype=torch.bfloat16, device=dev)
+    yk = torch.empty_like(x)
+
+    def gu_chain():
+        for L in layers:
+            wq.gateup_w2_lora(x, L.gate, L.up, L.lora_a, L.lora_b_gate, L.lora_b_up, L.lora_scale, prenorm=True,
+                              h=h, ws=ws)
+
+    def dn_chain():
+        for L in layers:
+            wq.down_w4(h, L.down, residual=x, y=yk, ws=ws)
+
+    ms_gu, _ = time_graph(capture(gu_chain), steps, warmup)
+    ms_dn, _ = time_graph(capture(dn_chain), steps, warmup)
+    assert wq.device_status() == 0
+    f_gu, f_dn = prefill_flops(cfg, m)
+    t_layer = ms / steps / n_layers / 1e3
+    t_gu = ms_gu / steps / n_layers / 1e3
+    t_dn = ms_dn / steps / n_layers / 1e3
+    peak, src = measured_tensor_peak()
+    gu_tf, dn_tf = f_gu / t_gu / 1e12, f_dn / t_dn / 1e12
+    wbytes = sum(algorithmic_bytes(cfg, m)) - (m * cfg.d * 2 * 3 + m * cfg.inter * 2 * 2)
+    return {
+        "workload": f"{cfg.name}_prefill_stack_{n_layers}L_m{m}",
+        "config": {"d": cfg.d, "inter": cfg.inter, "layers": n_layers, "m": m, "group": cfg.group_gu,
+                   "lora_r": cfg.r, "prenorm": True,
+                   "l2": f"no flush: {n_layers * wbytes / 1e9:.2f} GB of packed weights per step (> 129 MB L2)"},
+        "tokens_per_s": m * steps / (ms / 1e3), "us_per_layer": t_layer * 1e6,
+        "tflops": (f_gu + f_dn) / t_layer / 1e12, "flops_per_layer": f_gu + f_dn,
+        "dtype": "binary16 x binary16 tcgen05.mma, fp32 TMEM accumulate (weights dequantized to binary16)",
+        "clocks": clocks,
+        "roofline": {"bound": "tensor", "achieved": gu_tf, "peak": peak, "unit": "TFLOP/s", "frac": gu_tf / peak,
+                     "traffic": recorded_traffic("gemm_gateup_w2_m512", GEMM_SOURCES),
+                     "kernel": "wq_gateup_w2_lora at m=512 (input kernel + tcgen05 dequant-GEMM)",
+                     "algorithmic_flops_per_launch": f_gu, "us_per_launch": t_gu * 1e6,
+                     "peak_source": f"{src} dense bf16 burst (MEASURED_PEAKS.json bf16_tflops)"},
+        "kernels": {"gateup_w2_lora": {"us": t_gu * 1e6, "tflops": gu_tf, "frac": gu_tf / peak, "flops": f_gu},
+                    "down_w4": {"us": t_dn * 1e6, "tflops": dn_tf, "frac": dn_tf / peak, "flops": f_dn,
+                                "traffic": recorded_traffic("gemm_down_w4_m512", GEMM_SOURCES)}},
+    }
 
 
 # --------------------------------------------------------------------------- reference arm
