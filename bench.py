@@ -55,6 +55,9 @@ def parse():
     ap.add_argument("--leg", default="decode", choices=["decode", "prefill"],
                     help="with --eager: which stack to run (the decode stack or the prefill chunk)")
     ap.add_argument("--prefill-layers", type=int, default=4, help="distinct 14B-shaped layers of the prefill leg")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the bench line: decode stacks of the 4B/8B/14B shapes over their token counts, "
+                         "one JSON line")
     return ap.parse_args()
 
 
@@ -320,6 +323,9 @@ def run_gpu(args):
     if args.eager and args.leg == "prefill":
         run_prefill(wq, synth, dev, args.prefill_layers, steps, warmup, eager=True)
         return
+    if args.sweep:
+        print(json.dumps(run_sweep(wq, synth, dev, min(steps, 200), warmup)))
+        return
 
     layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
     table = wq.LayerTable(layers)
@@ -425,6 +431,40 @@ def run_gpu(args):
     if rank == 0:
         print(json.dumps(out))
     barrier(ws_)
+
+
+SWEEP = (("qwen3_4b", (1, 2, 4, 8, 16, 32, 64)), ("dense_8b", (1, 4, 16, 32, 64)), ("dense_14b", (1, 16, 64)))
+
+
+def run_sweep(wq, synth, dev, steps, warmup):
+    """Decode MLP stacks of the 4B, 8B and 14B shapes (all layers, W2 gate/up
+    + LoRA, W4 down, RMSNorm) at their token counts: tokens/s, µs per step and
+    the stack's algorithmic bytes per step over the measured HBM bandwidth."""
+    import torch
+    peak, src = measured_peaks()
+    out = {"metric": "decode MLP-stack tokens/s over token counts", "peak_gbs": peak, "peak_source": src,
+           "data": "synthetic", "rows": []}
+    for name, ms in SWEEP:
+        cfg = synth.CONFIGS[name]
+        layers = build_stack(wq, synth, cfg, cfg.layers, 2, True, dev)
+        table = wq.LayerTable(layers)
+        for m in ms:
+            ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
+            x = synth.activations((m, cfg.d), 4096 + m, device=dev)
+            y = torch.empty_like(x)
+            g = capture(lambda: wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table))
+            ms_tot, clocks = time_graph(g, steps, warmup, 1, ClockSampler(dev.index or 0))
+            t_step = ms_tot / steps / 1e3
+            gu, dn = algorithmic_bytes(cfg, m)
+            gbs = cfg.layers * (gu + dn) / t_step / 1e9
+            out["rows"].append({"config": name, "layers": cfg.layers, "m": m, "tokens_per_s": m / t_step,
+                                "us_per_step": t_step * 1e6, "us_per_layer": t_step * 1e6 / cfg.layers,
+                                "stack_gbs": gbs, "frac_of_hbm": gbs / peak, "clocks": clocks})
+            assert wq.device_status() == 0
+            del g, ws, x, y
+        del layers, table
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_prefill(wq, synth, dev, n_layers, steps, warmup, eager=False):

@@ -20,8 +20,17 @@
  *     `void*` holding IEEE bfloat16 values.
  *   - Quantized weights use the packed format described at wq_qweight.
  *   - Supported: group in {32, 64, 128}; in-features a multiple of the group
- *     (WQ_ERR_SHAPE otherwise); 1 <= m <= 64 tokens (m == 0 is a no-op);
+ *     (WQ_ERR_SHAPE otherwise); 1 <= m <= 16384 tokens (m == 0 is a no-op);
  *     LoRA rank r a multiple of 8, r <= 64 (r == 0: no adapter).
+ *   - Two paths behind the same calls: up to 16 tokens the dequant-GEMV
+ *     kernels (exact products of the codes and binary16 activations on the
+ *     mma.sync tensor-core path, fp32 sums); above 16 tokens, and for a layer
+ *     shape the GEMV kernels have no launch configuration for at the given
+ *     token count, the batched dequant-GEMM on the tcgen05 tensor cores
+ *     (activations and each dequantized weight s (q - z) rounded once to
+ *     binary16, fp32 accumulation; with fp32 output of wq_down_w4 the weights
+ *     enter as two exact binary16 parts).  The workspace size covers the path
+ *     a call takes.
  *   - On error the call returns a negative wq_status and wq_last_error()
  *     describes it (per host thread).  Kernel-side waits are bounded; a wait
  *     that runs out records WQ_ERR_TIMEOUT, read back by wq_device_status().

@@ -67,7 +67,9 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
   size_t cnt1, cnt2, tp, xa, xb, h, hq, hsc, hxs, part1, part2;
-  size_t x16, rs, ta, h16;  // dequant-GEMM path (m > kMaxTokens)
+  // dequant-GEMM path (m > kMaxTokens, or a shape the GEMV path has no plan for)
+  size_t x16, rs, ta, h16, sk_cnt, sk_part;
+  bool gemm;  // the GEMM buffers are laid out
   size_t total;
 };
 
@@ -80,53 +82,68 @@ size_t partial_bytes(const GemvPlan &p, int nproj) {
 // Largest split-K partial buffer any plan of this shape can need (every
 // group size and LoRA rank, including the down launch that writes the next
 // layer's tile partials).
-bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2) {
+bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2, bool *all_fit = nullptr) {
   const int sms = num_sms();
   if (sms <= 0) return false;
   *p1 = *p2 = 0;
+  bool fit = true;
   const int groups[3] = {32, 64, 128};
   for (int g : groups) {
     for (int r = 0; r <= kMaxRank; r += 8) {
       GemvPlan pl;
       if (d % g == 0) {
         if (plan_gemv(kGateUpW2, inter, d, m, g, r, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
-        if (r == 0 && plan_gemv(kGateUpW4, inter, d, m, g, 0, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
+        else fit = false;
+        if (r == 0) {
+          if (plan_gemv(kGateUpW4, inter, d, m, g, 0, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
+          else fit = false;
+        }
       }
-      if (inter % g == 0 && (r == 0 || d % 8 == 0) && plan_gemv(kDownW4, d, inter, m, g, r, sms, &pl))
-        *p2 = std::max(*p2, partial_bytes(pl, 1));
+      if (inter % g == 0 && (r == 0 || d % 8 == 0)) {
+        if (plan_gemv(kDownW4, d, inter, m, g, r, sms, &pl)) *p2 = std::max(*p2, partial_bytes(pl, 1));
+        else fit = false;
+      }
     }
   }
+  if (all_fit) *all_fit = fit;
+  return true;
+}
+
+// The dequant-GEMM buffers from offset `off`: binary16 copies of the GEMM
+// inputs, RMSNorm scales, the LoRA-A products and the stream-K scratch.
+bool gemm_layout(int m, int d, int inter, size_t off, WsLayout *L) {
+  const size_t lda = (size_t)(std::max(d, inter) + 127) / 128 * 128, ldi = (size_t)(inter + 127) / 128 * 128;
+  const int sms = num_sms();
+  if (sms <= 0) return false;
+  const size_t cnt = std::max(gemm_counters(m, inter), gemm_counters(m, d));
+  const size_t part = std::max(gemm_scratch_floats(m, inter, d, 2, sms), gemm_scratch_floats(m, d, inter, 1, sms));
+  L->x16 = off;     off = up256(off + (size_t)m * lda * 2);
+  L->rs = off;      off = up256(off + (size_t)m * 4);
+  L->ta = off;      off = up256(off + (size_t)m * 2 * kMaxRank * 2);
+  L->h16 = off;     off = up256(off + (size_t)m * ldi * 2);
+  L->sk_cnt = off;  off = up256(off + cnt * 4);
+  L->sk_part = off; off = up256(off + part * 4);
+  L->gemm = true;
+  L->total = off;
   return true;
 }
 
 // The arrival counters come first: their offsets depend on (d, inter) only,
 // so a workspace zeroed once stays valid for every token count.
-bool ws_layout(int m, int d, int inter, WsLayout *L) {
+// gemv_only: the decode path's buffers alone (the call without a workspace).
+bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   *L = WsLayout{};
   if (m > kMaxTokens) {
-    // dequant-GEMM path: binary16 copies of the GEMM inputs, the RMSNorm
-    // scales and the LoRA-A products, and the stack's bf16 intermediates
-    const size_t lda = (size_t)(std::max(d, inter) + 127) / 128 * 128, ldi = (size_t)(inter + 127) / 128 * 128;
+    // dequant-GEMM path: the stack's bf16 intermediates, then the GEMM buffers
     size_t off = 0;
     L->xa = off;  off = up256(off + (size_t)m * d * 2);
     L->xb = off;  off = up256(off + (size_t)m * d * 2);
     L->h = off;   off = up256(off + (size_t)m * inter * 2);
-    L->x16 = off; off = up256(off + (size_t)m * lda * 2);
-    L->rs = off;  off = up256(off + (size_t)m * 4);
-    L->ta = off;  off = up256(off + (size_t)m * 2 * kMaxRank * 2);
-    L->h16 = off; off = up256(off + (size_t)m * ldi * 2);
-    // stream-K scratch shared by the gate/up and down launches (one at a time)
-    const int sms = num_sms();
-    if (sms <= 0) return false;
-    const size_t cnt = std::max(gemm_counters(m, inter), gemm_counters(m, d));
-    const size_t part = std::max(gemm_scratch_floats(m, inter, d, 2, sms), gemm_scratch_floats(m, d, inter, 1, sms));
-    L->cnt1 = off;  off = up256(off + cnt * 4);
-    L->part1 = off; off = up256(off + part * 4);
-    L->total = off;
-    return true;
+    return gemm_layout(m, d, inter, off, L);
   }
   size_t p1, p2;
-  if (!max_partials(m, d, inter, &p1, &p2)) return false;
+  bool all_fit = true;
+  if (!max_partials(m, d, inter, &p1, &p2, &all_fit)) return false;
   size_t off = 0;
   L->cnt1 = off; off = up256(off + (size_t)((inter + 15) / 16) * 4);
   L->cnt2 = off; off = up256(off + (size_t)((d + 15) / 16) * 4);
@@ -140,7 +157,25 @@ bool ws_layout(int m, int d, int inter, WsLayout *L) {
   L->part1 = off; off = up256(off + p1);
   L->part2 = off; off = up256(off + p2);
   L->total = off;
+  // above kGemvPreferTokens, or for a shape that lacks a GEMV plan for some
+  // group or rank at this token count, the calls take the dequant-GEMM path
+  if (!gemv_only && (m > kGemvPreferTokens || !all_fit)) return gemm_layout(m, d, inter, off, L);
   return true;
+}
+
+// Whether a call takes the dequant-GEMM path: above kGemvPreferTokens (where
+// it is the faster path on every measured layer shape; the GEMV kernels'
+// work grows faster than linearly with the token count), or where the GEMV
+// path has no launch plan.  The workspace holds the GEMM buffers then.
+bool gateup_uses_gemm(GemvKind kind, int m, const wq_qweight *gate, int r) {
+  if (m > kGemvPreferTokens) return true;
+  GemvPlan pl;
+  return !plan_gemv(kind, gate->n, gate->k, m, gate->group, r, num_sms(), &pl);
+}
+bool down_uses_gemm(int m, const wq_qweight *down, int r_next) {
+  if (m > kGemvPreferTokens) return true;
+  GemvPlan pl;
+  return !plan_gemv(kDownW4, down->n, down->k, m, down->group, r_next, num_sms(), &pl);
 }
 
 // gate/up (2-bit with LoRA, or 4-bit) for one layer.  tp_in: tile partials of
@@ -270,6 +305,7 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
                           unsigned flags, void *h, uint16_t *h16, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
   const int d = gate->k, inter = gate->n;
   const int lda = (d + 127) / 128 * 128;
+  if (!L.gemm) return fail(WQ_ERR_WORKSPACE, "workspace laid out without the dequant-GEMM buffers");
   uint16_t *x16 = reinterpret_cast<uint16_t *>(ws + L.x16);
   float *rs = reinterpret_cast<float *>(ws + L.rs);
   uint16_t *ta = reinterpret_cast<uint16_t *>(ws + L.ta);
@@ -294,8 +330,8 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
   a.out = h;
   a.out_f16 = h16;
   a.ldo16 = (inter + 127) / 128 * 128;
-  a.sk_part = reinterpret_cast<float *>(ws + L.part1);
-  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.cnt1);
+  a.sk_part = reinterpret_cast<float *>(ws + L.sk_part);
+  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.sk_cnt);
   e = launch_gemm(kind, a, s);
   if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
   return WQ_OK;
@@ -304,6 +340,7 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
 // down: from the binary16 h16 (null: converted from the bf16 h first).
 wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qweight *down, const void *residual,
                         void *y, int y_f32, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+  if (!L.gemm) return fail(WQ_ERR_WORKSPACE, "workspace laid out without the dequant-GEMM buffers");
   const int K = down->k, lda = (K + 127) / 128 * 128;
   if (!h16) {
     uint16_t *c = reinterpret_cast<uint16_t *>(ws + L.h16);
@@ -323,8 +360,8 @@ wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qwei
   a.residual = residual;
   a.out = y;
   a.out_f32 = y_f32;
-  a.sk_part = reinterpret_cast<float *>(ws + L.part1);
-  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.cnt1);
+  a.sk_part = reinterpret_cast<float *>(ws + L.sk_part);
+  a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.sk_cnt);
   cudaError_t e = launch_gemm(kDownW4, a, s);
   if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   return WQ_OK;
@@ -386,7 +423,7 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, gate->k, gate->n, &L)) != WQ_OK) return st;
-  if (m > kMaxTokens)
+  if (gateup_uses_gemm(kind, m, gate, r))
     st = run_gateup_gemm(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
                          static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
   else
@@ -512,7 +549,7 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
     return fail(WQ_ERR_UNSUPPORTED, "m=%d: the built-in scratch serves the decode path (m <= %d; use wq_gateup_w2_lora)",
                 m, kMaxTokens);
   WsLayout L;
-  if (!ws_layout(m, gate->k, gate->n, &L)) return fail(WQ_ERR_CUDA, "cannot query the current device");
+  if (!ws_layout(m, gate->k, gate->n, &L, true)) return fail(WQ_ERR_CUDA, "cannot query the current device");
   if (L.total > (size_t)WQ_NOALLOC_SCRATCH_BYTES)
     return fail(WQ_ERR_UNSUPPORTED, "this layer needs %zu bytes of scratch; the built-in scratch holds %u (use wq_gateup_w2_lora)",
                 L.total, (unsigned)WQ_NOALLOC_SCRATCH_BYTES);
@@ -544,7 +581,7 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
     return fail(WQ_ERR_ALIGN, "h, y or residual not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, down->n, down->k, &L)) != WQ_OK) return st;
-  if (m > kMaxTokens)
+  if (down_uses_gemm(m, down, 0))
     st = run_down_gemm(h, nullptr, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
                        static_cast<cudaStream_t>(stream));
   else
@@ -591,7 +628,16 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
   if ((st = check_ws(ws, ws_bytes, m, d, inter, &L)) != WQ_OK) return st;
   uint8_t *w8 = static_cast<uint8_t *>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (m > kMaxTokens) {
+  // the GEMV chain needs a plan for every layer's launches; otherwise the
+  // whole stack takes the dequant-GEMM chain
+  bool gemm_chain = m > kGemvPreferTokens;
+  for (int l = 0; l < n_layers && !gemm_chain; ++l) {
+    const wq_mlp_layer &Ly = layers[l];
+    const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
+    gemm_chain = gateup_uses_gemm(Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4, m, &Ly.gate, Ly.r) ||
+                 down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0);
+  }
+  if (gemm_chain) {
     // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up (h also in
     // binary16), down with the residual
     const void *cur = x;

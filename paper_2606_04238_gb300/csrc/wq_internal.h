@@ -9,7 +9,8 @@
 
 namespace wq {
 
-constexpr int kMaxTokens = 64;      // tokens per call on the dequant-GEMV path
+constexpr int kMaxTokens = 64;      // tokens per call the dequant-GEMV kernels can take
+constexpr int kGemvPreferTokens = 16;  // above this many tokens the calls take the dequant-GEMM path
 constexpr int kMaxGemmTokens = 16384;  // tokens per call on the dequant-GEMM path (above kMaxTokens)
 constexpr int kMaxRank = 64;        // LoRA rank limit
 constexpr float kRmsEps = 1e-6f;    // RMSNorm epsilon of WQ_PRENORM

@@ -167,3 +167,33 @@ def test_gemm_two_token_halves(wq, m):
     ref, _ = orc.down(synth.bf16_bits(hd), qd, group, synth.bf16_bits(res))
     check_bf16(y, ref, f"GEMM y (two halves) m={m}", min_exact=MIN_EXACT)
     check_f32(y32, ref, f"GEMM y(f32) (two halves) m={m}")
+
+
+def test_planless_decode_shape_takes_gemm(wq):
+    """64 tokens of the 14B-shaped layer (d=5120, inter=17408): the decode
+    GEMV kernels have no launch configuration at this size, so the calls (and
+    the stack) take the dequant-GEMM path under the same results contract."""
+    cfg = synth.CONFIGS["dense_14b"]
+    m = 64
+    wg, wu, wd = synth.layer_weights(cfg, 0)
+    qg = orc.quantize(wg.numpy(), cfg.group_gu, 2)[:3]
+    qu = orc.quantize(wu.numpy(), cfg.group_gu, 2)[:3]
+    qd = orc.quantize(wd.numpy(), cfg.group_down, 4)[:3]
+    del wg, wu, wd
+    a, bg, bu = synth.lora(cfg.d, cfg.inter, cfg.r, 17)
+    x = synth.activations((m, cfg.d), 19)
+    layer = wq.MLPLayer(upload_packed(*qg, cfg.group_gu, 2), upload_packed(*qu, cfg.group_gu, 2),
+                        upload_packed(*qd, cfg.group_down, 4), lora_a=a.cuda(), lora_b_gate=bg.cuda(),
+                        lora_b_up=bu.cuda(), lora_scale=cfg.lora_scale)
+    ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
+    h = wq.gateup_w2_lora(x.cuda(), layer.gate, layer.up, layer.lora_a, layer.lora_b_gate, layer.lora_b_up,
+                          cfg.lora_scale, prenorm=True, ws=ws)
+    y = wq.mlp_forward(x.cuda(), [layer], prenorm=True, ws=ws)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    xb = synth.bf16_bits(x)
+    ref_h, hb = orc.gateup(xb, qg, qu, cfg.group_gu, synth.bf16_bits(a), synth.bf16_bits(bg), synth.bf16_bits(bu),
+                           lora_scale=cfg.lora_scale, prenorm=True)
+    check_bf16(h, ref_h, "14B gate/up m=64", min_exact=MIN_EXACT)
+    ref_y, _ = orc.down(synth.bf16_bits(h.cpu()), qd, cfg.group_down, xb)  # teacher-forced on the GPU's h
+    check_bf16(y, ref_y, "14B stack m=64", min_exact=MIN_EXACT)

@@ -79,6 +79,9 @@ def test_gateup_w2_lora(wq, d, inter, group, r, m, prenorm):
 
 @pytest.mark.parametrize("m", [17, 33, 64])
 def test_gateup_w2_many_tokens(wq, m):
+    """Above 16 tokens the call takes the dequant-GEMM path (weights rounded
+    once to binary16): the bound is unchanged, the share of outputs equal to
+    the oracle's own bf16 rounding is that path's (0.6)."""
     d, inter, group, r = 512, 384, 64, 16
     L = _layer(d, inter, group, 64, r, seed=5)
     x = synth.activations((m, d), 7)
@@ -87,7 +90,7 @@ def test_gateup_w2_many_tokens(wq, m):
     h = wq.gateup_w2_lora(x.cuda(), g, u, a, bg, bu, lora_scale=2.0, prenorm=True)
     torch.cuda.synchronize()
     ref, _ = orc.gateup(synth.bf16_bits(x), L["g"], L["u"], group, *_orc_lora(L), lora_scale=2.0, prenorm=True)
-    check_bf16(h, ref, f"h m={m}")
+    check_bf16(h, ref, f"h m={m}", min_exact=0.6)
 
 
 @pytest.mark.parametrize("d,inter,group", [(256, 768, 64), (384, 200, 32), (512, 1000, 128)])
