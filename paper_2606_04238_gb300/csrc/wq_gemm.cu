@@ -154,7 +154,7 @@ __device__ __forceinline__ void gemm_deq_stage(const uint8_t *raw, uint8_t *Bs, 
   constexpr int GPB = C::GPB, GS = GROUP / 16;
   for (int item = dt; item < NPROJ * 8 * 32; item += kDeqWarps * 32) {
     const int p = item >> 8, j = (item >> 5) & 7, L = item & 31;
-    const int g = L >> 2, t = L & 3;
+    const int g = L >> 2;
     uint8_t *Bp = Bs + p * kTileBytes;
     // the lane's code words of this half block: 2-bit, words 2 hb, 2 hb + 1
     // of its 16 bytes; 4-bit, the 16 bytes of half hb
