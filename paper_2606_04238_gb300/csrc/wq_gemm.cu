@@ -827,121 +827,129 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_sk_kernel(const __grid_
 // [M][lda16] (the GEMM's A operand, zeros past K), the RMSNorm scale
 // rs = 1/sqrt(mean(x^2) + eps) and, with an adapter, ta = lora_scale * x A^T
 // as binary16 [M][2r] (gate rows, then up rows).
-// A CTA takes 32 tokens and 16 rows of A.  The products x A^T run on m16n8k16
-// bf16 MMAs (exact products, fp32 sums); the 8 warps take interleaved chunks
-// of 32 features and their partial sums are added in warp order.  A lane
-// loads 8 consecutive features of a row (16 bytes) and feeds features 0..3 and
-// 4..7 of them to two k-steps in the slots of k 2t, 2t+1, 2t+8, 2t+9: the same
-// permutation of k for x and A, so the sums are unchanged.  Every CTA sums x^2
-// of its tokens (row block 0 writes rs) and converts the chunks c with
-// c % gridDim.y == blockIdx.y.
-constexpr int kPrepTok = 32, kPrepRows = 16;
+// A CTA takes 16 tokens and 16 rows of A.  The products x A^T run on m16n8k16
+// bf16 MMAs (exact products, fp32 sums); the 16 warps take interleaved chunks
+// of 32 features, two chunks' loads in flight at a time, and their partial
+// sums are added in warp order.  A lane loads 8 consecutive features of a row
+// (16 bytes) and feeds features 0..3 and 4..7 of them to two k-steps in the
+// slots of k 2t, 2t+1, 2t+8, 2t+9: the same permutation of k for x and A, so
+// the sums are unchanged.  Every CTA sums x^2 of its tokens (row block 0
+// writes rs) and converts the chunks c with c % gridDim.y == blockIdx.y.
+constexpr int kPrepTok = 16, kPrepRows = 16, kPrepWarps = 16, kPrepUnroll = 2;
 
-__global__ void __launch_bounds__(256) gemm_prep_kernel(const __nv_bfloat16 *x, int M, int K, int lda16,
-                                                        const __nv_bfloat16 *lora_a, int r2, float lora_scale,
-                                                        uint16_t *x16, float *rs, uint16_t *ta) {
-  __shared__ float part[8][kPrepTok][kPrepRows + 1];
-  __shared__ float ssp[8][kPrepTok];
+__global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_bfloat16 *x, int M, int K, int lda16,
+                                                                   const __nv_bfloat16 *lora_a, int r2,
+                                                                   float lora_scale, uint16_t *x16, float *rs,
+                                                                   uint16_t *ta) {
+  __shared__ float part[kPrepWarps][kPrepTok][kPrepRows + 1];
+  __shared__ float ssp[kPrepWarps][kPrepTok];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, g = lane >> 2, t = lane & 3;
   const int m0 = blockIdx.x * kPrepTok, j0 = blockIdx.y * kPrepRows;
   const int nchunk = K / 32;
   const bool lora = r2 > 0;
-  float acc[2][2][4];
+  float acc[2][4];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) acc[i >> 3][(i >> 2) & 1][i & 3] = 0.f;
-  float ss[4] = {0.f, 0.f, 0.f, 0.f};  // tokens g, g + 8, g + 16, g + 24 of the block
-  for (int c = warp; c < nchunk; c += 8) {
-    const int k = c * 32 + 8 * t;
-    uint4 xa[4], ab[2];
+  for (int i = 0; i < 8; ++i) acc[i >> 2][i & 3] = 0.f;
+  float ss[2] = {0.f, 0.f};  // tokens g and g + 8 of the block
+  const auto word = [](const uint4 &v, int q) { return q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w; };
+  for (int cb = warp; cb < nchunk; cb += kPrepWarps * kPrepUnroll) {
+    uint4 xa[kPrepUnroll][2], ab[kPrepUnroll][2];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int m = m0 + g + 8 * i;
-      xa[i] = m < M ? __ldg(reinterpret_cast<const uint4 *>(x + (size_t)m * K + k)) : make_uint4(0u, 0u, 0u, 0u);
-    }
+    for (int u = 0; u < kPrepUnroll; ++u) {  // the loads of both chunks first
+      const int c = cb + u * kPrepWarps, k = c * 32 + 8 * t;
+      const bool in = c < nchunk;
 #pragma unroll
-    for (int n = 0; n < 2; ++n) {
-      const int j = j0 + 8 * n + g;
-      ab[n] = lora && j < r2 ? __ldg(reinterpret_cast<const uint4 *>(lora_a + (size_t)j * K + k))
-                             : make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
-        ss[i] = fmaf(lo, lo, ss[i]);
-        ss[i] = fmaf(hi, hi, ss[i]);
-      }
-    }
-    if (c % gridDim.y == blockIdx.y) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
+      for (int i = 0; i < 2; ++i) {
         const int m = m0 + g + 8 * i;
-        if (m >= M) continue;
-        const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
-        uint32_t o[4];
+        xa[u][i] = in && m < M ? __ldg(reinterpret_cast<const uint4 *>(x + (size_t)m * K + k))
+                               : make_uint4(0u, 0u, 0u, 0u);
+      }
 #pragma unroll
-        for (int e = 0; e < 4; ++e)
-          o[e] = h2bits(__floats2half2_rn(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u)));
-        *reinterpret_cast<uint4 *>(x16 + (size_t)m * lda16 + k) = make_uint4(o[0], o[1], o[2], o[3]);
+      for (int n = 0; n < 2; ++n) {
+        const int j = j0 + 8 * n + g;
+        ab[u][n] = in && lora && j < r2 ? __ldg(reinterpret_cast<const uint4 *>(lora_a + (size_t)j * K + k))
+                                        : make_uint4(0u, 0u, 0u, 0u);
       }
     }
-    if (lora) {
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const auto word = [&](const uint4 &v, int q) { return q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w; };
+    for (int u = 0; u < kPrepUnroll; ++u) {
+      const int c = cb + u * kPrepWarps, k = c * 32 + 8 * t;
+      if (c >= nchunk) break;  // the same for the whole warp
 #pragma unroll
-        for (int mt = 0; mt < 2; ++mt) {
-          // rows g, g + 8 of m-tile mt are tokens 16 mt + g (xa[2 mt]) and 16 mt + g + 8 (xa[2 mt + 1])
-          const uint32_t af[4] = {word(xa[2 * mt], 2 * h), word(xa[2 * mt + 1], 2 * h), word(xa[2 * mt], 2 * h + 1),
-                                  word(xa[2 * mt + 1], 2 * h + 1)};
+      for (int i = 0; i < 2; ++i) {
+        const uint32_t w[4] = {xa[u][i].x, xa[u][i].y, xa[u][i].z, xa[u][i].w};
 #pragma unroll
-          for (int nt = 0; nt < 2; ++nt) mma_bf16_16816(acc[mt][nt], af, word(ab[nt], 2 * h), word(ab[nt], 2 * h + 1));
+        for (int e = 0; e < 4; ++e) {
+          const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
+          ss[i] = fmaf(lo, lo, ss[i]);
+          ss[i] = fmaf(hi, hi, ss[i]);
+        }
+      }
+      if (c % gridDim.y == blockIdx.y) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int m = m0 + g + 8 * i;
+          if (m >= M) continue;
+          const uint32_t w[4] = {xa[u][i].x, xa[u][i].y, xa[u][i].z, xa[u][i].w};
+          uint32_t o[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            o[e] = h2bits(__floats2half2_rn(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u)));
+          *reinterpret_cast<uint4 *>(x16 + (size_t)m * lda16 + k) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+      }
+      if (lora) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          // rows g, g + 8 of the m-tile are tokens g (xa[u][0]) and g + 8 (xa[u][1])
+          const uint32_t af[4] = {word(xa[u][0], 2 * h), word(xa[u][1], 2 * h), word(xa[u][0], 2 * h + 1),
+                                  word(xa[u][1], 2 * h + 1)};
+#pragma unroll
+          for (int nt = 0; nt < 2; ++nt)
+            mma_bf16_16816(acc[nt], af, word(ab[u][nt], 2 * h), word(ab[u][nt], 2 * h + 1));
         }
       }
     }
   }
   // sums of squares: the quad's lanes hold disjoint features of the same tokens
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < 2; ++i) {
     ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 1);
     ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 2);
   }
-  if (t == 0)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) ssp[warp][g + 8 * i] = ss[i];
+  if (t == 0) {
+    ssp[warp][g] = ss[0];
+    ssp[warp][g + 8] = ss[1];
+  }
   if (lora) {
-    // accumulator (row, col) of m-tile mt, n-tile nt: rows g / g + 8, cols 2t, 2t+1
+    // accumulator (row, col) of n-tile nt: rows g / g + 8, cols 2t, 2t+1
 #pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-        part[warp][16 * mt + g][8 * nt + 2 * t] = acc[mt][nt][0];
-        part[warp][16 * mt + g][8 * nt + 2 * t + 1] = acc[mt][nt][1];
-        part[warp][16 * mt + g + 8][8 * nt + 2 * t] = acc[mt][nt][2];
-        part[warp][16 * mt + g + 8][8 * nt + 2 * t + 1] = acc[mt][nt][3];
-      }
+    for (int nt = 0; nt < 2; ++nt) {
+      part[warp][g][8 * nt + 2 * t] = acc[nt][0];
+      part[warp][g][8 * nt + 2 * t + 1] = acc[nt][1];
+      part[warp][g + 8][8 * nt + 2 * t] = acc[nt][2];
+      part[warp][g + 8][8 * nt + 2 * t + 1] = acc[nt][3];
+    }
   }
   __syncthreads();
   if (blockIdx.y == 0 && tid < kPrepTok && m0 + tid < M) {
     float tot = 0.f;
-    for (int w = 0; w < 8; ++w) tot += ssp[w][tid];
+    for (int w = 0; w < kPrepWarps; ++w) tot += ssp[w][tid];
     rs[m0 + tid] = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)K), kRmsEps)));
   }
   if (lora) {
-    for (int o = tid; o < kPrepTok * kPrepRows; o += 256) {
+    for (int o = tid; o < kPrepTok * kPrepRows; o += kPrepWarps * 32) {
       const int tl = o / kPrepRows, jl = o % kPrepRows;
       const int m = m0 + tl, j = j0 + jl;
       if (m >= M || j >= r2) continue;
       float v = 0.f;
-      for (int w = 0; w < 8; ++w) v += part[w][tl][jl];
+      for (int w = 0; w < kPrepWarps; ++w) v += part[w][tl][jl];
       ta[(size_t)m * r2 + j] = __half_as_ushort(__float2half_rn(lora_scale * v));
     }
   }
   // zeros past K
   if (blockIdx.y == 0)
-    for (int i = tid; i < kPrepTok * (lda16 - K); i += 256) {
+    for (int i = tid; i < kPrepTok * (lda16 - K); i += kPrepWarps * 32) {
       const int tl = i / (lda16 - K), k = K + i % (lda16 - K);
       if (m0 + tl < M) x16[(size_t)(m0 + tl) * lda16 + k] = 0;
     }
@@ -1105,7 +1113,7 @@ cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void 
   if (M <= 0) return cudaSuccess;
   if (K % 32 != 0 || lda16 < K) return cudaErrorInvalidValue;
   const dim3 grid((M + kPrepTok - 1) / kPrepTok, r2 > 0 ? (r2 + kPrepRows - 1) / kPrepRows : 1);
-  gemm_prep_kernel<<<grid, 256, 0, s>>>(
+  gemm_prep_kernel<<<grid, kPrepWarps * 32, 0, s>>>(
       reinterpret_cast<const __nv_bfloat16 *>(x), M, K, lda16, reinterpret_cast<const __nv_bfloat16 *>(lora_a), r2,
       lora_scale, x16, rs, ta);
   return cudaGetLastError();
