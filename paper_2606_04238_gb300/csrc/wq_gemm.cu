@@ -1036,9 +1036,13 @@ cudaError_t num_sms_cached(int *sms) {
 // Work split of a launch.  A CTA takes two token halves (each weight
 // dequantized once for 256 tokens) whenever there are more than 128 tokens.
 // Tiles are mt * 128 tokens x 128 rows, U work units each (128-feature
-// blocks, plus one for the LoRA stages).  One CTA per tile when the last wave
-// of CTAs is at least 80% full; otherwise stream-K: P CTAs (one per SM at
-// most, 4 units each at least) divide the T * U units evenly.
+// blocks, plus one for the LoRA stages).  Stream-K -- P CTAs (one per SM at
+// most, 4 units each at least) dividing the T * U units evenly -- when it
+// shortens the critical path by more than its own cost, which was measured at
+// about 40 units (the split tiles' partial sums and fixups, and a slower main
+// loop); one CTA per tile otherwise.
+constexpr long long kStreamKCost = 40;  // work units
+
 struct GemmSched {
   int mt, T, U, P;
   bool sk;
@@ -1049,9 +1053,9 @@ GemmSched gemm_schedule(int M, int N, int K, int nproj, int r, int sms) {
   g.T = (M + g.mt * kBM - 1) / (g.mt * kBM) * ((N + kBN - 1) / kBN);
   g.U = (K + 127) / 128 + (nproj == 2 && r > 0 ? 1 : 0);
   const long long W = (long long)g.T * g.U;
-  const int waves = (g.T + sms - 1) / sms;
-  g.sk = 10LL * g.T < 8LL * waves * sms && W >= 8;
-  g.P = g.sk ? (int)std::max(1LL, std::min((long long)sms, W / 4)) : g.T;
+  const long long waves = (g.T + sms - 1) / sms, P = std::max(1LL, std::min((long long)sms, W / 4));
+  g.sk = W >= 8 && waves * g.U > (W + P - 1) / P + kStreamKCost;
+  g.P = g.sk ? (int)P : g.T;
   return g;
 }
 

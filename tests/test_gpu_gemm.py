@@ -197,3 +197,33 @@ def test_planless_decode_shape_takes_gemm(wq):
     check_bf16(h, ref_h, "14B gate/up m=64", min_exact=MIN_EXACT)
     ref_y, _ = orc.down(synth.bf16_bits(h.cpu()), qd, cfg.group_down, xb)  # teacher-forced on the GPU's h
     check_bf16(y, ref_y, "14B stack m=64", min_exact=MIN_EXACT)
+
+
+@pytest.mark.parametrize("m", [65, 200])
+def test_gemm_stream_k_split_tiles(wq, m):
+    """Few output tiles over a long feature axis (8192 features, 64 blocks):
+    the launch runs stream-K, every tile split over several CTAs, the LoRA
+    stages in the last part; gate/up with adapter and RMSNorm, then down
+    (8192 -> 384 rows) with a residual in bf16 and fp32."""
+    d, inter, group, r = 8192, 384, 128, 16
+    qg, qu = _q((inter, d), group, 2, 91), _q((inter, d), group, 2, 92)
+    a, bg, bu = synth.lora(d, inter, r, 93)
+    x = synth.activations((m, d), 94 + m)
+    h = wq.gateup_w2_lora(x.cuda(), upload_packed(*qg, group, 2), upload_packed(*qu, group, 2), prenorm=True,
+                          lora_a=a.cuda(), lora_b_gate=bg.cuda(), lora_b_up=bu.cuda(), lora_scale=2.0)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.gateup(synth.bf16_bits(x), qg, qu, group, synth.bf16_bits(a), synth.bf16_bits(bg),
+                        synth.bf16_bits(bu), lora_scale=2.0, prenorm=True)
+    check_bf16(h, ref, f"GEMM h (stream-K) m={m}", min_exact=MIN_EXACT)
+    qd = _q((inter, d), group, 4, 95)  # down: inter (384) output rows from d (8192) features
+    hd = (synth.activations((m, d), 96 + m) * 0.5).to(torch.bfloat16)
+    res = synth.activations((m, inter), 97 + m)
+    dn = upload_packed(*qd, group, 4)
+    y = wq.down_w4(hd.cuda(), dn, residual=res.cuda())
+    y32 = wq.down_w4(hd.cuda(), dn, residual=res.cuda(), out_f32=True)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.down(synth.bf16_bits(hd), qd, group, synth.bf16_bits(res))
+    check_bf16(y, ref, f"GEMM y (stream-K) m={m}", min_exact=MIN_EXACT)
+    check_f32(y32, ref, f"GEMM y(f32) (stream-K) m={m}")
