@@ -113,7 +113,7 @@ wq_status wq_packed_sizes(int bits, int n, int k, int group, size_t *code_bytes,
 
 /*
  * Stage-1 quantization and packing (Sec. 4.1 selective INT2 quantization of
- * gate/up; INT4 for the remaining layers, Sec. 3.3 and Sec. 6 step 4).
+ * gate/up; INT4 for the remaining layers, Sec. 3.3 and Sec. 7 step 4).
  * Asymmetric min-max round-to-nearest per group of `group` consecutive input
  * features of each row, in IEEE fp32:
  *     s = fp16((max - min) / qmax)  (1.0 if that is zero),

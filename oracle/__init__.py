@@ -13,6 +13,9 @@ What it computes (paper sections cited in ``wq_oracle.c``):
                    gate/up weights, h = SiLU(g) * u (Sec. 3.3), fp64.
   * ``down``       y = residual + h Wd^T on the dequantized 4-bit down weights.
   * ``rms_scale``  unit-weight RMSNorm scale 1/sqrt(mean(x^2)+eps) per token.
+  * ``merge_lora`` the merged matrix deq(W) + alpha B A (Eq. 1; Sec. 4.2 lets
+                   the adapters be merged after training), fp64 then one
+                   rounding to fp32, ready to be quantized again.
 """
 from __future__ import annotations
 
@@ -59,6 +62,7 @@ def _load():
                 "orc_tile_pack": (I, [P, P, P, I, I, I, I, P, P]),
                 "orc_tile_unpack": (I, [P, P, I, I, I, I, P, P, P]),
                 "orc_dequant": (I, [P, P, P, I, I, I, P]),
+                "orc_merge_lora": (I, [P, P, P, I, I, I, P, P, I, D, P]),
                 "orc_rms_scale": (I, [P, I, I, D, P]),
                 "orc_gateup": (I, [P, I, I, I, P, P, P, P, P, P, I, P, P, P, I, D, I, D, P, P]),
                 "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
@@ -168,6 +172,26 @@ def dequant(q, s, z, group: int) -> np.ndarray:
     if _load().orc_dequant(_p(q), _p(s), _p(z), n, k, group, _p(w)) < 0:
         raise ValueError("orc_dequant: bad arguments")
     return w
+
+
+def merge_lora(q, s, z, group: int, lora_b, lora_a, lora_scale: float) -> np.ndarray:
+    """fp32 [n, k] matrix deq(W) + alpha B A (B bf16 bits [n, r], A bf16 bits [r, k]).
+
+    alpha is taken as the fp32 value the library receives (``float`` in its C ABI).
+    """
+    q = _c(q, np.uint8)
+    s = _c(s, np.uint16)
+    z = _c(z, np.uint16)
+    n, k = q.shape
+    lb = _c(lora_b, np.uint16).reshape(n, -1)
+    r = lb.shape[1]
+    la = _c(lora_a, np.uint16).reshape(r, k) if r else np.zeros(1, np.uint16)
+    out = np.empty((n, k), np.float32)
+    rc = _load().orc_merge_lora(_p(q), _p(s), _p(z), n, k, group, _p(lb if r else np.zeros(1, np.uint16)),
+                                _p(la), r, float(np.float32(lora_scale)), _p(out))
+    if rc < 0:
+        raise ValueError("orc_merge_lora: bad arguments")
+    return out
 
 
 # -------------------------------------------------------------------- forward

@@ -281,6 +281,39 @@ int orc_dequant(const uint8_t *q, const uint16_t *s, const uint16_t *z,
     return ORC_OK;
 }
 
+/*
+ * Merging the adapter into the quantized matrix (Sec. 4.2: once trained, the
+ * adapters may be merged into the quantized weights instead of being kept as
+ * a separate module; Sec. 7, step 5 of the deployment pipeline).  By Eq. 1
+ * the merged matrix is W + alpha B A, with W the dequantized matrix:
+ *   w_out[n,k] = fp32( s[n,j] (q[n,k] - z[n,j]) + alpha * sum_rho B[n,rho] A[rho,k] )
+ * with j = k / group, B bf16 [n, r], A bf16 [r, k].  The sum runs over rho
+ * in ascending order in fp64 (every product of two bf16 values is exact in
+ * fp64), alpha multiplies it in fp64, and the result is rounded to fp32 once.
+ * The merged matrix is then quantized again with orc_quantize at the same
+ * bits and group (the paper names no other quantizer for this step).
+ */
+int orc_merge_lora(const uint8_t *q, const uint16_t *s, const uint16_t *z,
+                   int n, int k, int group,
+                   const uint16_t *lora_b, const uint16_t *lora_a, int r,
+                   double lora_scale, float *w_out)
+{
+    if (n < 0 || k < 0 || group <= 0 || k % group != 0 || r < 0) return ORC_ERR_ARG;
+    const int ng = k / group;
+    for (int row = 0; row < n; ++row)
+        for (int col = 0; col < k; ++col) {
+            const size_t gi = (size_t)row * ng + col / group;
+            const double w = orc_f16_to_f64(s[gi]) *
+                             ((double)q[(size_t)row * k + col] - orc_f16_to_f64(z[gi]));
+            double ba = 0.0;
+            for (int rho = 0; rho < r; ++rho)
+                ba += orc_bf16_to_f64(lora_b[(size_t)row * r + rho]) *
+                      orc_bf16_to_f64(lora_a[(size_t)rho * k + col]);
+            w_out[(size_t)row * k + col] = (float)(w + lora_scale * ba);
+        }
+    return ORC_OK;
+}
+
 /* ------------------------------------------------------------------ */
 /* Forward pass.                                                       */
 /* ------------------------------------------------------------------ */

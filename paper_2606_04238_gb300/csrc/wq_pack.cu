@@ -1,6 +1,6 @@
 // wq_pack.cu -- Stage-1 group-wise quantizer and packer (sm_103a).
 //
-// Sec. 4.1 quantizes gate/up to INT2 and (Sec. 3.3, Sec. 6 step 4) every
+// Sec. 4.1 quantizes gate/up to INT2 and (Sec. 3.3, Sec. 7 step 4) every
 // other linear layer to INT4.  The quantizer is asymmetric min-max
 // round-to-nearest per group of `group` consecutive input features of a row,
 // computed in IEEE fp32 with explicit round-to-nearest intrinsics so that the
