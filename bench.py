@@ -11,7 +11,7 @@ needed between steps.
 Reported besides the step rate: the fused 2-bit gate/up call and the 4-bit
 down call timed on their own (36 distinct layers back to back, one graph) for
 the HBM roofline, the uniform-W4 stack on the same GPU (speedup, Gain%), the
-end-to-end rate through the C ABI with host buffers, SM clocks sampled during
+same stack with the adapters merged into the 2-bit codes, the end-to-end rate through the C ABI with host buffers, SM clocks sampled during
 the timed region, the CPU oracle on a bounded sample, and the prefill leg: a
 512-token chunk through 14B-shaped layers (d=5120, inter=17408, LoRA rank 32),
 which runs on the tcgen05 dequant-GEMM path, against the tensor roofline.
@@ -423,6 +423,19 @@ def run_gpu(args):
                              "paper_gain_pct_context": "7.5-23.3% whole-model TPS, LIFE roofline model on "
                                                        "Device A (50 TOPs, 100 GB/s) / Device B (200 GB/s)"}
         del w4, g4
+        # the same stack with each layer's adapters merged into new 2-bit codes (wq_merge_lora; Sec. 4.2
+        # and Sec. 7 step 5 allow either form): no adapter bytes and no LoRA stages on the decode path
+        wm = torch.empty((cfg.inter, cfg.d), dtype=torch.float32, device=dev)
+        merged = [wq.merge_layer(L, w_merged=wm) for L in layers]
+        del wm
+        tmg = wq.LayerTable(merged)
+        gmg = capture(lambda: wq.mlp_forward(x, merged, prenorm=True, y=y, ws=ws, table=tmg))
+        msm, _ = time_graph(gmg, steps, warmup)
+        tpsm = m * steps / (msm / 1e3)
+        out["merged_adapters"] = {"tokens_per_s": tpsm, "ms_per_step": msm / steps, "vs_unmerged": tpsm / tps,
+                                  "algorithmic_gb_per_step": n_layers * sum(algorithmic_bytes(cfg, m, lora=False)) / 1e9,
+                                  "note": "adapters merged into the 2-bit codes and requantized; r = 0 at decode"}
+        del merged, tmg, gmg
         torch.cuda.empty_cache()
         out["prefill"] = run_prefill(wq, synth, dev, args.prefill_layers, max(20, min(steps, 200)), warmup)
         torch.cuda.empty_cache()

@@ -131,6 +131,32 @@ wq_status wq_pack_w2(const float *w, int n, int k, int group, wq_qweight *out, i
 wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream);
 
 /*
+ * Merged adapters (Sec. 4.2: once trained, the adapters may be merged into the
+ * quantized weights instead of kept as a separate module; Sec. 7 step 5
+ * deploys either form).  By Eq. 1 the merged matrix is deq(W) + alpha B A:
+ *     W'[n, k] = fp32( s (q - z) + lora_scale * sum_rho B[n, rho] A[rho, k] ),
+ * evaluated in fp64 (rho ascending, one rounding to fp32 at the end), then
+ * quantized and packed exactly as wq_pack does, at the source's bits and
+ * group.  The merged layer runs with r = 0 on the same calls.
+ *   src:        packed source matrix (device buffers), bits 2 or 4.
+ *   lora_b:     bf16 [n, r] row-major, device.  For gate: lora_b_gate.
+ *   lora_a:     bf16 [r, k] row-major, device.  For gate: the first r rows of
+ *               a layer's lora_a; for up: lora_a + r * k.
+ *   r:          0..64 (0: W' = deq(W), which RTN maps back onto the source
+ *               codes wherever a group holds both end codes).
+ *   lora_scale: alpha of Eq. 1, finite.
+ *   w_merged:   device fp32 [n, k] scratch, caller-owned, 16-byte aligned;
+ *               holds W' afterwards.
+ *   out:        as for wq_pack.  Either src itself (in place: in stream order
+ *               the merge reads src completely before the quantizer writes)
+ *               or buffers disjoint from src's.
+ *   nonfinite:  optional device int, as for wq_pack.
+ * Two launches on `stream`, no synchronization, no allocation.
+ */
+wq_status wq_merge_lora(const wq_qweight *src, const void *lora_b, const void *lora_a, int r, float lora_scale,
+                        float *w_merged, wq_qweight *out, int *nonfinite, void *stream);
+
+/*
  * Workspace (device scratch, caller-owned) needed by wq_gateup_*, wq_down_w4
  * and wq_mlp_forward for up to m tokens of a layer of hidden size d,
  * intermediate size inter and LoRA rank r, on the current device.  Before its

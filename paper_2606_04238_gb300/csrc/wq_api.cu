@@ -2,6 +2,7 @@
 // layout, launch sequencing.  Every check happens on the host before any
 // launch; nothing here allocates device memory or synchronizes (except
 // wq_device_status, which is documented to).
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -11,6 +12,13 @@
 
 #include "wq.h"
 #include "wq_internal.h"
+
+namespace wq {
+// The adapter merge lives in wq_pack.cu beside the quantizer that follows it.
+cudaError_t launch_merge_lora(const uint32_t *codes, const uint16_t *meta, int n, int k, int group, int bits,
+                              const void *lora_b, const void *lora_a, int r, float alpha, float *w,
+                              cudaStream_t stream);
+}  // namespace wq
 
 using namespace wq;
 
@@ -470,6 +478,36 @@ wq_status wq_pack_w2(const float *w, int n, int k, int group, wq_qweight *out, i
 
 wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, int *nonfinite, void *stream) {
   return wq_pack(w, n, k, group, 4, out, nonfinite, stream);
+}
+
+wq_status wq_merge_lora(const wq_qweight *src, const void *lora_b, const void *lora_a, int r, float lora_scale,
+                        float *w_merged, wq_qweight *out, int *nonfinite, void *stream) {
+  if (!src) return fail(WQ_ERR_ARG, "src: null wq_qweight");
+  if (src->bits != 2 && src->bits != 4) return fail(WQ_ERR_SHAPE, "src: bits %d not in {2, 4}", src->bits);
+  wq_status st = check_qweight(src, src->bits, "src");
+  if (st != WQ_OK) return st;
+  if (r < 0 || r > kMaxRank) return fail(WQ_ERR_SHAPE, "LoRA rank %d not in [0, %d]", r, kMaxRank);
+  if (r > 0 && (!lora_a || !lora_b)) return fail(WQ_ERR_ARG, "null LoRA pointer with r=%d", r);
+  if ((reinterpret_cast<uintptr_t>(lora_a) | reinterpret_cast<uintptr_t>(lora_b)) & 1u)
+    return fail(WQ_ERR_ALIGN, "LoRA pointers not 2-byte aligned");
+  if (!std::isfinite(lora_scale)) return fail(WQ_ERR_ARG, "lora_scale is not finite");
+  if (!out) return fail(WQ_ERR_ARG, "null output wq_qweight");
+  if (!w_merged || !out->codes || !out->meta) return fail(WQ_ERR_ARG, "null w_merged, codes or meta pointer");
+  if (!aligned16(w_merged) || !aligned16(out->codes) || !aligned16(out->meta))
+    return fail(WQ_ERR_ALIGN, "w_merged, codes or meta pointer not 16-byte aligned");
+  const wq_qweight s = *src;  // out may be src itself
+  const cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_merge_lora(static_cast<const uint32_t *>(s.codes), static_cast<const uint16_t *>(s.meta),
+                                    s.n, s.k, s.group, s.bits, lora_b, lora_a, r, lora_scale, w_merged, cs);
+  if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+  e = launch_pack(w_merged, s.n, s.k, s.group, s.bits, static_cast<uint32_t *>(out->codes),
+                  static_cast<uint16_t *>(out->meta), nonfinite, cs);
+  if (e != cudaSuccess) return cuda_fail(e, "pack launch");
+  out->n = s.n;
+  out->k = s.k;
+  out->group = s.group;
+  out->bits = s.bits;
+  return ok();
 }
 
 size_t wq_workspace_bytes(int m, int d, int inter, int r) {

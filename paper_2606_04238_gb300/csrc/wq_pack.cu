@@ -10,7 +10,12 @@
 // Two kernels: one warp per (row, group) computes s and z into the packed
 // meta layout; then one thread per packed 32-bit word gathers its 16 (2-bit)
 // or 8 (4-bit) codes.  Offline work: not on the decode path.
+// A third kernel merges a trained adapter into a packed matrix before it is
+// quantized again (below).
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
+
+#include <algorithm>
 
 #include "wq_internal.h"
 
@@ -94,7 +99,66 @@ __global__ void pack_codes_kernel(const float *__restrict__ w, int n, int k, int
   codes[wid] = word;
 }
 
+// Adapter merge (Sec. 4.2 lets the trained adapters be merged into the
+// quantized weights; Sec. 7 step 5 deploys them merged or attached).  By
+// Eq. 1 the merged matrix is deq(W) + alpha B A:
+//   w[row, col] = fp32( s (q - z) + alpha * sum_rho B[row, rho] A[rho, col] ),
+// evaluated in fp64 with rho ascending (a product of two bf16 values is exact)
+// and rounded to fp32 once.  Every operation is an explicit round-to-nearest
+// intrinsic, so no contraction changes the result.  The codes, scales and
+// zeros are read from the packed layout of include/wq.h.  A CTA takes 256
+// features of a row (rows strided by gridDim.y); the row of B is staged in
+// shared memory as fp64.
+constexpr int kMergeThreads = 256;
+
+__global__ void __launch_bounds__(kMergeThreads)
+    merge_lora_kernel(const uint32_t *__restrict__ codes, const uint16_t *__restrict__ meta, int n, int k,
+                      int group, int bits, int KB, int NG, const __nv_bfloat16 *__restrict__ lora_b,
+                      const __nv_bfloat16 *__restrict__ lora_a, int r, double alpha, float *__restrict__ w) {
+  __shared__ double brow[kMaxRank];
+  const int col = blockIdx.x * kMergeThreads + threadIdx.x;
+  const int wpb = bits == 2 ? 128 : 256;
+  const uint32_t mask = (1u << bits) - 1u;
+  for (int row = blockIdx.y; row < n; row += gridDim.y) {
+    __syncthreads();  // the previous row's B is read by every thread first
+    if (threadIdx.x < r) brow[threadIdx.x] = (double)__bfloat162float(lora_b[(size_t)row * r + threadIdx.x]);
+    __syncthreads();
+    if (col >= k) continue;
+    const int rt = row >> 4, i = row & 15, kb = col >> 7, c = col & 127;
+    const int lane = (i & 7) * 4 + ((c & 7) >> 1), half = c & 1;
+    int word, bit;
+    if (bits == 2) {
+      word = lane * 4 + (c >> 5);
+      bit = 16 * half + 8 * (i >> 3) + 2 * (2 * ((c & 31) >> 4) + ((c & 15) >> 3));
+    } else {
+      word = (c >> 6) * 128 + lane * 4 + ((c & 63) >> 4);
+      bit = 16 * half + 8 * (i >> 3) + 4 * ((c & 15) >> 3);
+    }
+    const uint32_t q = (codes[((size_t)rt * KB + kb) * wpb + word] >> bit) & mask;
+    const size_t mb = ((size_t)rt * NG + col / group) * 32 + 4 * (i & 7) + (i >> 3);
+    const double sf = (double)__half2float(__ushort_as_half(meta[mb]));
+    const double zf = (double)__half2float(__ushort_as_half(meta[mb + 2]));
+    double ba = 0.0;
+    for (int rho = 0; rho < r; ++rho)
+      ba = __dadd_rn(ba, __dmul_rn(brow[rho], (double)__bfloat162float(lora_a[(size_t)rho * k + col])));
+    const double v = __dadd_rn(__dmul_rn(sf, __dsub_rn((double)q, zf)), __dmul_rn(alpha, ba));
+    w[(size_t)row * k + col] = __double2float_rn(v);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_merge_lora(const uint32_t *codes, const uint16_t *meta, int n, int k, int group, int bits,
+                              const void *lora_b, const void *lora_a, int r, float alpha, float *w,
+                              cudaStream_t stream) {
+  const int KB = (k + 127) / 128, NG = KB * 128 / group;
+  const dim3 grid((unsigned)((k + kMergeThreads - 1) / kMergeThreads), (unsigned)std::min(n, 65535));
+  merge_lora_kernel<<<grid, kMergeThreads, 0, stream>>>(codes, meta, n, k, group, bits, KB, NG,
+                                                         static_cast<const __nv_bfloat16 *>(lora_b),
+                                                         static_cast<const __nv_bfloat16 *>(lora_a), r,
+                                                         (double)alpha, w);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint32_t *codes, uint16_t *meta,
                         int *nonfinite, cudaStream_t stream) {

@@ -64,6 +64,7 @@ def lib():
             "wq_pack": (I, [P, I, I, I, I, QP, P, P]),
             "wq_pack_w2": (I, [P, I, I, I, QP, P, P]),
             "wq_pack_w4": (I, [P, I, I, I, QP, P, P]),
+            "wq_merge_lora": (I, [QP, P, P, I, F, P, QP, P, P]),
             "wq_workspace_bytes": (S, [I, I, I, I]),
             "wq_workspace_init": (I, [P, S, P]),
             "wq_gateup_w2_lora": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P, S, P]),
@@ -145,6 +146,29 @@ def pack_w2(w, group, nonfinite=None):
 
 def pack_w4(w, group, nonfinite=None):
     return pack(w, group, 4, nonfinite)
+
+
+def merge_lora(src: QWeight, lora_b: torch.Tensor | None, lora_a: torch.Tensor | None, lora_scale: float,
+               out: QWeight | None = None, w_merged: torch.Tensor | None = None,
+               nonfinite: torch.Tensor | None = None) -> QWeight:
+    """Merge an adapter into a packed matrix and quantize it again (wq_merge_lora).
+
+    lora_b is bf16 [n, r] and lora_a bf16 [r, k], contiguous on the device (None
+    for r = 0).  ``out=src`` merges in place; ``w_merged`` (fp32 [n, k]) receives
+    the merged matrix before quantization.
+    """
+    r = 0 if lora_b is None else lora_b.shape[1]
+    if r:
+        assert lora_b.dtype == torch.bfloat16 and lora_a.dtype == torch.bfloat16
+        assert lora_b.is_contiguous() and lora_a.is_contiguous()
+        assert tuple(lora_b.shape) == (src.n, r) and tuple(lora_a.shape) == (r, src.k)
+    if w_merged is None:
+        w_merged = torch.empty(src.n, src.k, dtype=torch.float32, device=src.codes.device)
+    q = out if out is not None else empty_qweight(src.n, src.k, src.group, src.bits, device=src.codes.device)
+    cs, cq = src.c(), q.c()
+    _check(lib().wq_merge_lora(ctypes.byref(cs), _ptr(lora_b) if r else None, _ptr(lora_a) if r else None, r,
+                               float(lora_scale), _ptr(w_merged), ctypes.byref(cq), _ptr(nonfinite), _stream()))
+    return q
 
 
 def workspace_bytes(m: int, d: int, inter: int, r: int = 0) -> int:
@@ -238,6 +262,18 @@ class MLPLayer:
                          None if self.lora_b_gate is None else self.lora_b_gate.data_ptr(),
                          None if self.lora_b_up is None else self.lora_b_up.data_ptr(),
                          self.r, float(self.lora_scale))
+
+
+def merge_layer(layer: MLPLayer, w_merged: torch.Tensor | None = None) -> MLPLayer:
+    """The layer with its gate and up adapters merged into new 2-bit codes
+    (wq_merge_lora on each); the merged layer carries no adapter (r = 0)."""
+    r = layer.r
+    if r == 0:
+        return MLPLayer(layer.gate, layer.up, layer.down)
+    a = layer.lora_a
+    gate = merge_lora(layer.gate, layer.lora_b_gate, a[:r], layer.lora_scale, w_merged=w_merged)
+    up = merge_lora(layer.up, layer.lora_b_up, a[r:], layer.lora_scale, w_merged=w_merged)
+    return MLPLayer(gate, up, layer.down)
 
 
 class LayerTable:
