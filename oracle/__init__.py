@@ -13,6 +13,8 @@ What it computes (paper sections cited in ``wq_oracle.c``):
                    gate/up weights, h = SiLU(g) * u (Sec. 3.3), fp64.
   * ``down``       y = residual + h Wd^T on the dequantized 4-bit down weights.
   * ``rms_scale``  unit-weight RMSNorm scale 1/sqrt(mean(x^2)+eps) per token.
+  * ``down_bf16``  y = residual + h Wd^T with a bf16 Wd (the BF16/W2-GateUp
+                   configuration of the accuracy experiments, Sec. 6.1), fp64.
   * ``merge_lora`` the merged matrix deq(W) + alpha B A (Eq. 1; Sec. 4.2 lets
                    the adapters be merged after training), fp64 then one
                    rounding to fp32, ready to be quantized again.
@@ -66,6 +68,7 @@ def _load():
                 "orc_rms_scale": (I, [P, I, I, D, P]),
                 "orc_gateup": (I, [P, I, I, I, P, P, P, P, P, P, I, P, P, P, I, D, I, D, P, P]),
                 "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
+                "orc_down_bf16": (I, [P, I, I, I, P, P, P, P]),
                 "orc_threads": (I, []),
                 "orc_set_threads": (None, [I]),
                 "orc_f32_to_f16_array": (None, [P, S, P]),
@@ -243,6 +246,21 @@ def down(h_bits, wd, group: int, residual_bits=None):
     rc = _load().orc_down(_p(h), m, inter, d, _p(q), _p(s), _p(z), group, _p(res), _p(y), _p(yb))
     if rc < 0:
         raise ValueError("orc_down: bad arguments")
+    return y, yb
+
+
+def down_bf16(h_bits, wd_bits, residual_bits=None):
+    """y = residual + h Wd^T with Wd bf16 bits [d, inter].  Returns (y_f64, y_bf16_bits)."""
+    h = _c(h_bits, np.uint16)
+    m, inter = h.shape
+    wd = _c(wd_bits, np.uint16)
+    d = wd.shape[0]
+    assert wd.shape == (d, inter)
+    res = None if residual_bits is None else _c(residual_bits, np.uint16)
+    y = np.empty((m, d), np.float64)
+    yb = np.empty((m, d), np.uint16)
+    if _load().orc_down_bf16(_p(h), m, inter, d, _p(wd), _p(res), _p(y), _p(yb)) < 0:
+        raise ValueError("orc_down_bf16: bad arguments")
     return y, yb
 
 

@@ -20,6 +20,9 @@
  *     matrix, evaluated in fp64.
  *   - The gated MLP h = SiLU(gate(x)) * up(x), y = x + down(h) (Sec. 3.3),
  *     optionally preceded by a unit-weight RMSNorm of the MLP input.
+ *   - The down layer of the BF16/W2-GateUp configuration (bf16 weights,
+ *     Sec. 6.1), and the merged matrix deq(W) + alpha B A of an adapter
+ *     folded into the quantized weights (Sec. 4.2).
  *
  * bf16 rounding happens only where the CUDA path stores a bf16 tensor: the
  * hidden activation h and the layer output y.  The RMSNorm-normalized input
@@ -441,6 +444,32 @@ int orc_down(const uint16_t *h, int m, int inter, int d,
         for (int tk = 0; tk < m; ++tk) {
             double y = orc_qdot(qd + (size_t)c * inter, sd + (size_t)c * ng, zd + (size_t)c * ng,
                                 inter, group, h + (size_t)tk * inter);
+            if (residual) y += orc_bf16_to_f64(residual[(size_t)tk * d + c]);
+            if (y_f64) y_f64[(size_t)tk * d + c] = y;
+            if (y_bf16) y_bf16[(size_t)tk * d + c] = orc_f64_to_bf16(y);
+        }
+    }
+    return ORC_OK;
+}
+
+/*
+ * bf16 down projection with residual: the down layer of the BF16/W2-GateUp
+ * configuration of the accuracy experiments (Sec. 6.1 keeps every layer but
+ * gate/up in BF16; Sec. 7 names it beside the deployed W4/W2-GateUp form):
+ *   y[m,c] = residual[m,c] + sum_n h[m,n] Wd[c,n]
+ * h: [m, inter] bf16.  Wd: [d, inter] bf16 row-major.  residual: [m, d] bf16
+ * or NULL.  fp64 sum over n in ascending order; y_f64 / y_bf16 optional.
+ */
+int orc_down_bf16(const uint16_t *h, int m, int inter, int d, const uint16_t *wd,
+                  const uint16_t *residual, double *y_f64, uint16_t *y_bf16)
+{
+    if (m < 0 || d <= 0 || inter <= 0) return ORC_ERR_ARG;
+#pragma omp parallel for schedule(static)
+    for (int c = 0; c < d; ++c) {
+        for (int tk = 0; tk < m; ++tk) {
+            double y = 0.0;
+            for (int n = 0; n < inter; ++n)
+                y += orc_bf16_to_f64(h[(size_t)tk * inter + n]) * orc_bf16_to_f64(wd[(size_t)c * inter + n]);
             if (residual) y += orc_bf16_to_f64(residual[(size_t)tk * d + c]);
             if (y_f64) y_f64[(size_t)tk * d + c] = y;
             if (y_bf16) y_bf16[(size_t)tk * d + c] = orc_f64_to_bf16(y);

@@ -163,3 +163,49 @@ def test_empty_token_batch(orc):
     assert h.shape == (0, 64)
     y, _ = orc.down(hb, dn, 64, x)
     assert y.shape == (0, 128)
+
+
+def _grid_bf16(rng, shape, lim=255, exp=-8):
+    """bf16 bit patterns of m * 2^exp, |m| <= lim < 256 (exact in bf16; fp64 sums of their products are exact)."""
+    v = rng.integers(-lim, lim + 1, size=shape).astype(np.float32) * np.float32(2.0 ** exp)
+    return (v.view(np.uint32) >> 16).astype(np.uint16)
+
+
+def test_down_bf16_matches_numpy(orc):
+    """BF16/W2-GateUp down layer (Sec. 6.1): y = residual + h Wd^T with a bf16 Wd."""
+    rng = np.random.default_rng(17)
+    d, inter, m = 80, 384, 5
+    h, wd, res = _grid_bf16(rng, (m, inter)), _grid_bf16(rng, (d, inter), exp=-12), _grid_bf16(rng, (m, d))
+    y, yb = orc.down_bf16(h, wd, res)
+    want = _bf16_to_f64(res) + _bf16_to_f64(h) @ _bf16_to_f64(wd).T  # every sum exact: equal bit for bit
+    np.testing.assert_array_equal(y, want)
+    np.testing.assert_array_equal(yb, orc.f64_to_bf16_bits(y))
+    y0, _ = orc.down_bf16(h, wd, None)
+    np.testing.assert_array_equal(y0, _bf16_to_f64(h) @ _bf16_to_f64(wd).T)
+    hg, wg = _rand_bf16(rng, (3, inter)), _rand_bf16(rng, (d, inter), 0.02)
+    yg, _ = orc.down_bf16(hg, wg, None)
+    np.testing.assert_allclose(yg, _bf16_to_f64(hg) @ _bf16_to_f64(wg).T, rtol=1e-12, atol=1e-13)
+
+
+def test_down_bf16_agrees_with_the_4bit_down_on_bf16_exact_weights(orc):
+    """A 4-bit matrix whose dequantized values bf16 holds exactly (scale 2^-6,
+    q - z in [-15, 15]) gives the same y through both down definitions."""
+    rng = np.random.default_rng(18)
+    d, inter, group, m = 48, 256, 64, 4
+    q = rng.integers(0, 16, size=(d, inter)).astype(np.uint8)
+    s = np.full((d, inter // group), np.float16(2.0 ** -6)).view(np.uint16)
+    z = rng.integers(0, 16, size=(d, inter // group)).astype(np.float16).view(np.uint16)
+    deq = _np_deq(q, s, z, group)
+    wd = (deq.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    assert np.array_equal(_bf16_to_f64(wd), deq)
+    h, res = _rand_bf16(rng, (m, inter)), _rand_bf16(rng, (m, d))
+    y4, _ = orc.down(h, (q, s, z), group, res)
+    y16, _ = orc.down_bf16(h, wd, res)
+    np.testing.assert_allclose(y16, y4, rtol=1e-13, atol=1e-14)
+
+
+def test_down_bf16_empty_and_bad_args(orc):
+    y, yb = orc.down_bf16(np.zeros((0, 64), np.uint16), np.zeros((32, 64), np.uint16))
+    assert y.shape == (0, 32) and yb.shape == (0, 32)
+    with pytest.raises(AssertionError):
+        orc.down_bf16(np.zeros((1, 64), np.uint16), np.zeros((32, 48), np.uint16))
