@@ -11,7 +11,8 @@ needed between steps.
 Reported besides the step rate: the fused 2-bit gate/up call and the 4-bit
 down call timed on their own (36 distinct layers back to back, one graph) for
 the HBM roofline, the uniform-W4 stack on the same GPU (speedup, Gain%), the
-same stack with the adapters merged into the 2-bit codes, the end-to-end rate through the C ABI with host buffers, SM clocks sampled during
+same stack with the adapters merged into the 2-bit codes, the bf16 down call
+of the BF16/W2-GateUp configuration, the end-to-end rate through the C ABI with host buffers, SM clocks sampled during
 the timed region, the CPU oracle on a bounded sample, and the prefill leg: a
 512-token chunk through 14B-shaped layers (d=5120, inter=17408, LoRA rank 32),
 which runs on the tcgen05 dequant-GEMM path, against the tensor roofline.
@@ -410,6 +411,20 @@ def run_gpu(args):
                         "traffic": recorded_traffic("down_w4")},
         }
 
+        # the bf16 down layer of the BF16/W2-GateUp configuration (Sec. 6.1), 36 distinct matrices back to back
+        wdb = [synth.weights((cfg.d, cfg.inter), 3 * l + 2, device=dev).to(torch.bfloat16) for l in range(n_layers)]
+
+        def bd_chain():
+            for W in wdb:
+                wq.down_bf16(h, W, residual=x, y=yk)
+
+        ms_bd, _ = time_graph(capture(bd_chain), ks, warmup)
+        t_bd = ms_bd / ks / n_layers / 1e3
+        bd_bytes = cfg.d * cfg.inter * 2 + m * cfg.inter * 2 + 2 * m * cfg.d * 2
+        out["kernels"]["down_bf16"] = {"us": t_bd * 1e6, "gbs": bd_bytes / t_bd / 1e9,
+                                       "frac": bd_bytes / t_bd / 1e9 / peak, "bytes": bd_bytes,
+                                       "note": "bf16 down of the BF16/W2-GateUp configuration (wq_down_bf16)"}
+        del wdb
         # the uniform-W4 comparator stack (same workload, 4-bit gate/up, no adapter)
         del g, ge
         w4 = build_stack(wq, synth, cfg, n_layers, 4, False, dev)

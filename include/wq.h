@@ -231,6 +231,19 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
                      void *y, int y_dtype, void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * bf16 down projection with optional residual: the down layer of the
+ * BF16/W2-GateUp configuration that the accuracy experiments use (Sec. 6.1:
+ * gate/up at INT2, every other layer in BF16; Sec. 7):
+ *     y = residual + h Wd^T
+ *   h:  bf16 [m, inter].  wd: bf16 [d, inter] row-major (device, 16-byte
+ *   aligned), inter a multiple of 32.  residual: bf16 [m, d] or NULL.
+ *   y:  [m, d] of y_dtype (as for wq_down_w4).
+ * Needs no workspace; one launch on `stream`.  Products are exact, sums fp32.
+ */
+wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, const void *residual, void *y,
+                       int y_dtype, void *stream);
+
+/*
  * A stack of gated-MLP layers for one decode step of m tokens:
  *     x_0 = x,  x_{l+1} = x_l + down_l( SiLU(gate_l(xin_l)) * up_l(xin_l) ),  y = x_L
  * with xin_l = RMSNorm(x_l) (unrounded, as in wq_gateup_w2_lora) when flags has

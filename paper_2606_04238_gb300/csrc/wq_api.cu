@@ -18,6 +18,9 @@ namespace wq {
 cudaError_t launch_merge_lora(const uint32_t *codes, const uint16_t *meta, int n, int k, int group, int bits,
                               const void *lora_b, const void *lora_a, int r, float alpha, float *w,
                               cudaStream_t stream);
+// The bf16 down projection lives in wq_dense.cu.
+cudaError_t launch_down_bf16(const void *h, int m, const void *wd, int d, int inter, const void *residual, void *y,
+                             bool y_f32, cudaStream_t stream);
 }  // namespace wq
 
 using namespace wq;
@@ -626,6 +629,23 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
     st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, nullptr, 0, nullptr, L, static_cast<uint8_t *>(ws),
                   static_cast<cudaStream_t>(stream));
   return st == WQ_OK ? ok() : st;
+}
+
+wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, const void *residual, void *y,
+                       int y_dtype, void *stream) {
+  wq_status st = check_tokens(m);
+  if (st != WQ_OK) return st;
+  if (d <= 0 || inter <= 0 || inter % 32 != 0)
+    return fail(WQ_ERR_SHAPE, "bad shape d=%d, inter=%d (inter a positive multiple of 32)", d, inter);
+  if (y_dtype != WQ_BF16 && y_dtype != WQ_F32) return fail(WQ_ERR_ARG, "y_dtype %d not WQ_BF16 or WQ_F32", y_dtype);
+  if (m == 0) return ok();
+  if (!h || !wd || !y) return fail(WQ_ERR_ARG, "null h, wd or y");
+  if (!aligned16(h) || !aligned16(wd) || !aligned16(y) || (residual && !aligned16(residual)))
+    return fail(WQ_ERR_ALIGN, "h, wd, y or residual not 16-byte aligned");
+  cudaError_t e = launch_down_bf16(h, m, wd, d, inter, residual, y, y_dtype == WQ_F32,
+                                   static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "bf16 down launch");
+  return ok();
 }
 
 wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, void *y,

@@ -71,6 +71,7 @@ def lib():
             "wq_gateup_w2_lora_noalloc": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P]),
             "wq_gateup_w4": (I, [P, I, QP, QP, U, P, P, S, P]),
             "wq_down_w4": (I, [P, I, QP, P, P, I, P, S, P]),
+            "wq_down_bf16": (I, [P, I, P, I, I, P, P, I, P]),
             "wq_mlp_forward": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, S, P]),
             "wq_plan_info": (I, [I, I, I, I, I, I, ctypes.POINTER(ctypes.c_int64)]),
             "wq_last_error": (ctypes.c_char_p, []),
@@ -239,6 +240,19 @@ def down_w4(h, down: QWeight, residual=None, out_f32: bool = False, y=None, ws=N
     cd = down.c()
     _check(lib().wq_down_w4(_ptr(h), m, ctypes.byref(cd), _ptr(residual), _ptr(y), WQ_F32 if out_f32 else WQ_BF16,
                             _ptr(ws), ws.numel(), _stream()))
+    return y
+
+
+def down_bf16(h, wd, residual=None, out_f32: bool = False, y=None):
+    """y = residual + h Wd^T with a bf16 Wd [d, inter] (wq_down_bf16)."""
+    assert h.dtype == torch.bfloat16 and wd.dtype == torch.bfloat16 and h.is_contiguous() and wd.is_contiguous()
+    m, inter = h.shape
+    d = wd.shape[0]
+    assert wd.shape[1] == inter
+    if y is None:
+        y = torch.empty((m, d), dtype=torch.float32 if out_f32 else torch.bfloat16, device=h.device)
+    _check(lib().wq_down_bf16(_ptr(h), m, _ptr(wd), d, inter, _ptr(residual), _ptr(y), WQ_F32 if out_f32 else WQ_BF16,
+                              _stream()))
     return y
 
 
