@@ -111,6 +111,47 @@ def test_pack_host_validation(wq):
     assert L.wq_pack(ctypes.c_void_p(16), 16, 128, 64, 2, ctypes.byref(q2), None, None) == -3  # misaligned meta
 
 
+def test_merge_host_validation(wq):
+    L = wq.lib()
+    src = _qw(wq, 64, 256, 64, 2)
+    out = _qw(wq, 0, 0, 0, 0)
+
+    def call(src, b=16, a=16, r=8, scale=2.0, wm=16, out=out):
+        return L.wq_merge_lora(None if src is None else ctypes.byref(src), ctypes.c_void_p(b), ctypes.c_void_p(a), r,
+                               scale, ctypes.c_void_p(wm), None if out is None else ctypes.byref(out), None, None)
+
+    assert call(None) == -1                                         # null source
+    assert call(_qw(wq, 64, 256, 64, 3)) == -2                      # bits
+    assert call(_qw(wq, 64, 256, 48, 2)) == -2                      # group
+    assert call(_qw(wq, 64, 256, 64, 2, meta=8)) == -3              # misaligned meta
+    assert call(src, r=65) == -2                                    # rank above 64
+    assert call(src, a=0) == -1                                     # rank without A
+    assert call(src, b=17) == -3                                    # odd B pointer
+    assert call(src, scale=float("inf")) == -1                      # non-finite alpha
+    assert call(src, out=None) == -1                                # null output
+    assert call(src, wm=0) == -1                                    # null scratch
+    assert call(src, wm=20) == -3                                   # misaligned scratch
+    assert call(src, r=0, a=0, b=0, out=_qw(wq, 0, 0, 0, 0, codes=0)) == -1  # null output codes
+
+
+def test_down_bf16_host_validation(wq):
+    L = wq.lib()
+
+    def call(h=16, m=1, wd=16, d=64, inter=128, res=None, y=16, dtype=0):
+        return L.wq_down_bf16(ctypes.c_void_p(h), m, ctypes.c_void_p(wd), d, inter,
+                              None if res is None else ctypes.c_void_p(res), ctypes.c_void_p(y), dtype, None)
+
+    assert call(m=-1) == -1                                         # negative m
+    assert call(m=16385) == -4                                      # beyond the token limit
+    assert call(inter=80) == -2                                     # features not a multiple of 32
+    assert call(d=0) == -2                                          # no rows
+    assert call(dtype=5) == -1                                      # output type
+    assert call(m=0, h=0) == 0                                      # empty batch: no-op
+    assert call(h=0) == -1                                          # null h
+    assert call(wd=8) == -3                                         # misaligned weights
+    assert call(res=40) == -3                                       # misaligned residual
+
+
 def test_product_path_has_no_oracle_import():
     pkg = os.path.join(ROOT, "paper_2606_04238_gb300")
     for dirpath, _, files in os.walk(pkg):
