@@ -38,23 +38,35 @@ _lib = None
 RMS_EPS = 1e-6
 
 
+def compile_source(src: str, out: str) -> str:
+    """gcc with IEEE arithmetic (no fast-math, no FMA contraction) -> shared library ``out``."""
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
+           "-fPIC", "-shared", "-o", tmp, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
 def build(force: bool = False) -> str:
-    """Compile the oracle with gcc (IEEE arithmetic: no fast-math, no FMA contraction)."""
+    """Compile the oracle (see compile_source) unless the library is newer than its source."""
     os.makedirs(_BUILD_DIR, exist_ok=True)
     if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
-        tmp = _LIB_PATH + f".tmp{os.getpid()}"
-        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
-               "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"]
-        subprocess.run(cmd, check=True)
-        os.replace(tmp, _LIB_PATH)
+        compile_source(_SRC, _LIB_PATH)
     return _LIB_PATH
+
+
+def _library_path() -> str:
+    """The compiled oracle.  WQ_ORACLE_LIB names another build of this source
+    instead: the mutation tests load copies with one planted mistake."""
+    return os.environ.get("WQ_ORACLE_LIB") or build()
 
 
 def _load():
     global _lib
     with _lock:
         if _lib is None:
-            lib = ctypes.CDLL(build())
+            lib = ctypes.CDLL(_library_path())
             P = ctypes.c_void_p
             I = ctypes.c_int
             D = ctypes.c_double

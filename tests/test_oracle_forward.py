@@ -93,6 +93,30 @@ def test_lora_rank1_closed_form(orc):
     np.testing.assert_allclose(h[0], want, rtol=1e-12, atol=1e-14)
 
 
+@pytest.mark.parametrize("prenorm", [False, True])
+def test_lora_rank8_matches_numpy_matmul(orc, prenorm):
+    # Eq. 1 on both projections with numpy matmuls as the steps:
+    #   g = xin Wg^T + alpha (xin A_g^T) B_g^T,  u likewise,  h = SiLU(g) u.
+    # A rank above 1 with inter != r != d separates every index of A and B.
+    rng = np.random.default_rng(9)
+    d, inter, r, m = 192, 72, 8, 3
+    g, u, _ = _layer(orc, rng, d, inter, 64, 64)
+    x = _rand_bf16(rng, (m, d))
+    a = _rand_bf16(rng, (2 * r, d), 0.05)
+    bg = _rand_bf16(rng, (inter, r), 0.05)
+    bu = _rand_bf16(rng, (inter, r), 0.05)
+    alpha = 2.0
+    h, _ = orc.gateup(x, g, u, 64, a, bg, bu, lora_scale=alpha, prenorm=prenorm)
+    xf = _bf16_to_f64(x)
+    if prenorm:
+        xf = xf / np.sqrt(np.mean(xf * xf, axis=1, keepdims=True) + 1e-6)
+    af = _bf16_to_f64(a)
+    gg = xf @ _np_deq(*g, 64).T + alpha * (xf @ af[:r].T) @ _bf16_to_f64(bg).T
+    uu = xf @ _np_deq(*u, 64).T + alpha * (xf @ af[r:].T) @ _bf16_to_f64(bu).T
+    want = torch.nn.functional.silu(torch.from_numpy(gg)).numpy() * uu
+    np.testing.assert_allclose(h, want, rtol=1e-11, atol=1e-13)
+
+
 def test_rms_scale_matches_torch_rms_norm(orc):
     rng = np.random.default_rng(5)
     x = _rand_bf16(rng, (4, 512), 3.0)
