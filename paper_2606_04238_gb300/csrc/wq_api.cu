@@ -12,16 +12,7 @@
 
 #include "wq.h"
 #include "wq_internal.h"
-
-namespace wq {
-// The adapter merge lives in wq_pack.cu beside the quantizer that follows it.
-cudaError_t launch_merge_lora(const uint32_t *codes, const uint16_t *meta, int n, int k, int group, int bits,
-                              const void *lora_b, const void *lora_a, int r, float alpha, float *w,
-                              cudaStream_t stream);
-// The bf16 down projection lives in wq_dense.cu.
-cudaError_t launch_down_bf16(const void *h, int m, const void *wd, int d, int inter, const void *residual, void *y,
-                             bool y_f32, cudaStream_t stream);
-}  // namespace wq
+#include "wq_launch.h"
 
 using namespace wq;
 

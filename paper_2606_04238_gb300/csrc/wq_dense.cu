@@ -25,6 +25,7 @@
 #include <cuda_bf16.h>
 
 #include "wq_ptx.cuh"
+#include "wq_launch.h"
 
 namespace wq {
 namespace {

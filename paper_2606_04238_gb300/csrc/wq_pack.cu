@@ -18,6 +18,7 @@
 #include <algorithm>
 
 #include "wq_internal.h"
+#include "wq_launch.h"
 
 namespace wq {
 namespace {
