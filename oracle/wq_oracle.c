@@ -133,7 +133,7 @@ int orc_quantize(const float *w, int n, int k, int group, int bits,
                  uint8_t *q, uint16_t *s_out, uint16_t *z_out)
 {
     if (n < 0 || k < 0 || group <= 0 || k % group != 0) return ORC_ERR_ARG;
-    if (bits != 2 && bits != 4) return ORC_ERR_ARG;
+    if (bits < 2 || bits > 4) return ORC_ERR_ARG;   /* INT2, INT3 (App. B), INT4 */
     const float qmax = (float)((1 << bits) - 1);
     const int ng = k / group;
     int nonfinite = 0;

@@ -44,7 +44,7 @@ def test_golden_worked_examples(orc):
         assert q[0].tolist() == e["q"], e["name"]
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 @pytest.mark.parametrize("group", [32, 64, 128])
 @pytest.mark.parametrize("dist", ["n002", "n1", "uniform", "mixed"])
 def test_matches_numpy_brute_force(orc, bits, group, dist):
@@ -78,7 +78,7 @@ def test_matches_numpy_brute_force(orc, bits, group, dist):
 def test_exact_grid_reconstructs(orc):
     # Groups that are exactly {(i - z0) * s : i = 0..qmax} with a binary16 scale.
     rng = np.random.default_rng(7)
-    for bits in (2, 4):
+    for bits in (2, 3, 4):
         qmax = 2 ** bits - 1
         rows = []
         for _ in range(64):
@@ -93,7 +93,7 @@ def test_exact_grid_reconstructs(orc):
         np.testing.assert_array_equal(deq, w.astype(np.float64))
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_rounding_bound_inside_clamp_range(orc, bits):
     rng = np.random.default_rng(11)
     group = 64
@@ -121,12 +121,13 @@ def test_rtn_error_level_sanity(orc):
     rng = np.random.default_rng(5)
     w = (rng.standard_normal((256, 2048)) * 0.02).astype(np.float32)
     levels = {}
-    for bits, group in ((2, 128), (2, 64), (4, 128)):
+    for bits, group in ((2, 128), (2, 64), (3, 32), (4, 128)):
         q, s, z, _ = orc.quantize(w, group, bits)
         deq = orc.dequant(q, s, z, group)
         levels[(bits, group)] = np.linalg.norm(deq - w) / np.linalg.norm(w)
     assert 0.40 < levels[(2, 128)] < 0.60
     assert levels[(2, 64)] < levels[(2, 128)]
+    assert levels[(4, 128)] < levels[(3, 32)] < levels[(2, 64)]  # App. B's INT3 g32 between INT4 and INT2
     assert 0.06 < levels[(4, 128)] < 0.14
 
 
