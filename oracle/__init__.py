@@ -150,7 +150,7 @@ def quantize(w, group: int, bits: int):
 def packed_sizes(n: int, k: int, group: int, bits: int):
     """(code words, meta halves) of the packed format for an [n, k] matrix."""
     rt, kb = (n + 15) // 16, (k + 127) // 128
-    wpb = 128 if bits == 2 else 256
+    wpb = {2: 128, 3: 192, 4: 256}[bits]
     return rt * kb * wpb, rt * (kb * 128 // group) * 32
 
 

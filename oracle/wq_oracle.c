@@ -185,6 +185,11 @@ int orc_quantize(const float *w, int n, int k, int group, int bits,
  * and, for 4-bit codes (256 words per block, two 64-feature halves):
  *   word  = (c / 64) * 128 + lane * 4 + (c % 64) / 16
  *   bit   = 16*half + 8*(i / 8) + 4*((c % 16) / 8)
+ * and, for 3-bit codes (App. B; 192 words per block, 3 bits a weight), two
+ * bit planes: q % 4 in words 0..127 exactly as a 2-bit code, and q / 4 in
+ * words 128..191:
+ *   word  = 128 + lane * 2 + (c / 32) / 2
+ *   bit   = 16*half + 8*((c / 32) % 2) + 2*( 2*((c % 32) / 16) + (c % 16) / 8 ) + i / 8
  *
  * meta: uint16 (binary16) values, 32 per (row tile, group): for row tile rt
  * and group j (NG = K_pad / group groups per row) the 32 values at
@@ -192,13 +197,13 @@ int orc_quantize(const float *w, int n, int k, int group, int bits,
  *   [4e+0] = s[row 16rt+e]   [4e+1] = s[row 16rt+e+8]
  *   [4e+2] = z[row 16rt+e]   [4e+3] = z[row 16rt+e+8]
  */
-static int orc_words_per_block(int bits) { return bits == 2 ? 128 : 256; }
+static int orc_words_per_block(int bits) { return bits == 2 ? 128 : bits == 3 ? 192 : 256; }
 
 int orc_tile_pack(const uint8_t *q, const uint16_t *s, const uint16_t *z,
                   int n, int k, int group, int bits,
                   uint32_t *codes, uint16_t *meta)
 {
-    if ((bits != 2 && bits != 4) || group <= 0 || k % group != 0 || 128 % group != 0)
+    if (bits < 2 || bits > 4 || group <= 0 || k % group != 0 || 128 % group != 0)
         return ORC_ERR_ARG;
     const int RT = (n + 15) / 16, KB = (k + 127) / 128;
     const int Kp = KB * 128, NG = Kp / group, ngk = k / group;
@@ -213,14 +218,22 @@ int orc_tile_pack(const uint8_t *q, const uint16_t *s, const uint16_t *z,
             const int lane = (i % 8) * 4 + (c % 8) / 2;
             const int half = c % 2;
             int word, bit;
-            if (bits == 2) {
-                word = lane * 4 + c / 32;
-                bit = 16 * half + 8 * (i / 8) + 2 * (2 * ((c % 32) / 16) + (c % 16) / 8);
-            } else {
+            if (bits == 4) {
                 word = (c / 64) * 128 + lane * 4 + (c % 64) / 16;
                 bit = 16 * half + 8 * (i / 8) + 4 * ((c % 16) / 8);
+            } else {
+                word = lane * 4 + c / 32;
+                bit = 16 * half + 8 * (i / 8) + 2 * (2 * ((c % 32) / 16) + (c % 16) / 8);
             }
-            codes[((size_t)rt * KB + kb) * wpb + word] |= code << bit;
+            uint32_t *blk = codes + ((size_t)rt * KB + kb) * wpb;
+            if (bits == 3) {
+                const int cls = 2 * ((c % 32) / 16) + (c % 16) / 8;
+                blk[word] |= (code & 3u) << bit;
+                blk[128 + lane * 2 + (c / 32) / 2] |=
+                    (code >> 2) << (16 * half + 8 * ((c / 32) % 2) + 2 * cls + i / 8);
+            } else {
+                blk[word] |= code << bit;
+            }
         }
         for (int j = 0; j < ngk; ++j) {
             const size_t base = ((size_t)rt * NG + j) * 32;
@@ -236,7 +249,7 @@ int orc_tile_unpack(const uint32_t *codes, const uint16_t *meta,
                     int n, int k, int group, int bits,
                     uint8_t *q, uint16_t *s, uint16_t *z)
 {
-    if ((bits != 2 && bits != 4) || group <= 0 || k % group != 0 || 128 % group != 0)
+    if (bits < 2 || bits > 4 || group <= 0 || k % group != 0 || 128 % group != 0)
         return ORC_ERR_ARG;
     const int KB = (k + 127) / 128;
     const int Kp = KB * 128, NG = Kp / group, ngk = k / group;
@@ -249,15 +262,22 @@ int orc_tile_unpack(const uint32_t *codes, const uint16_t *meta,
             const int lane = (i % 8) * 4 + (c % 8) / 2;
             const int half = c % 2;
             int word, bit;
-            if (bits == 2) {
-                word = lane * 4 + c / 32;
-                bit = 16 * half + 8 * (i / 8) + 2 * (2 * ((c % 32) / 16) + (c % 16) / 8);
-            } else {
+            if (bits == 4) {
                 word = (c / 64) * 128 + lane * 4 + (c % 64) / 16;
                 bit = 16 * half + 8 * (i / 8) + 4 * ((c % 16) / 8);
+            } else {
+                word = lane * 4 + c / 32;
+                bit = 16 * half + 8 * (i / 8) + 2 * (2 * ((c % 32) / 16) + (c % 16) / 8);
             }
-            q[(size_t)r * k + col] =
-                (uint8_t)((codes[((size_t)rt * KB + kb) * wpb + word] >> bit) & mask);
+            const uint32_t *blk = codes + ((size_t)rt * KB + kb) * wpb;
+            if (bits == 3) {
+                const int cls = 2 * ((c % 32) / 16) + (c % 16) / 8;
+                const uint32_t hi = (blk[128 + lane * 2 + (c / 32) / 2] >>
+                                     (16 * half + 8 * ((c / 32) % 2) + 2 * cls + i / 8)) & 1u;
+                q[(size_t)r * k + col] = (uint8_t)(((blk[word] >> bit) & 3u) | (hi << 2));
+            } else {
+                q[(size_t)r * k + col] = (uint8_t)((blk[word] >> bit) & mask);
+            }
         }
         for (int j = 0; j < ngk; ++j) {
             const size_t base = ((size_t)rt * NG + j) * 32;

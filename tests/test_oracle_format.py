@@ -17,7 +17,7 @@ def _rand_codes(rng, n, k, bits, group):
     return q, s, z
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 @pytest.mark.parametrize("n,k,group", [(16, 128, 128), (48, 256, 64), (37, 192, 64), (5, 96, 32), (130, 384, 128)])
 def test_roundtrip(orc, bits, n, k, group):
     rng = np.random.default_rng(n * k + bits)
@@ -29,7 +29,7 @@ def test_roundtrip(orc, bits, n, k, group):
     np.testing.assert_array_equal(z, z2)
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_padding_is_zero(orc, bits):
     n, k, group = 21, 160, 32
     q = np.full((n, k), 2 ** bits - 1, np.uint8)
@@ -99,6 +99,42 @@ def test_w4_layout_matches_mma_fragments(orc):
                         row, col = _fragment_owner(lane, reg, elem)
                         val = (regs[reg] >> (16 * elem)) & 0xF
                         assert val == q[row, 16 * kstep + col]
+
+
+def test_w3_layout_matches_mma_fragments(orc):
+    """3-bit codes (App. B) as two planes, read the way a kernel would: the
+    2-bit plane's class c taken with the mask 3 << 2c (rows g + 8 from the
+    word >> 8), and the plane-1 bit of the same code moved to bit 2c + 2 by
+    one shift of the lane's plane-1 word (<< 2 / << 1 for the even 2-bit
+    word, >> 6 / >> 7 for the odd one, rows g / g + 8) and the mask 4 << 2c.
+    Each 16-bit half of a register must then read q * 4^c for the (row, k)
+    the PTX fragment assigns to it, below 1024 (a binary16 subnormal)."""
+    rng = np.random.default_rng(2)
+    q = rng.integers(0, 8, (16, 128)).astype(np.uint8)
+    codes, _ = orc.tile_pack(q, np.zeros((16, 1), np.uint16), np.zeros((16, 1), np.uint16), 128, 3)
+    assert codes.size == 192
+    lo_words = codes[:128].reshape(32, 4)   # [lane][word]
+    hi_words = codes[128:].reshape(32, 2)   # [lane][word]
+    shifts = {(0, 0): ("<<", 2), (0, 1): ("<<", 1), (1, 0): (">>", 6), (1, 1): (">>", 7)}  # (word parity, row half)
+    for lane in range(32):
+        for wi in range(4):
+            w, hw = int(lo_words[lane, wi]), int(hi_words[lane, wi // 2])
+            for s in range(2):                      # two k-steps per 2-bit word
+                kstep = 2 * wi + s
+                for reg in range(4):
+                    rowhalf = 1 if reg in (1, 3) else 0
+                    cls = 2 * s + (1 if reg in (2, 3) else 0)
+                    src = (w >> 8) if rowhalf else w
+                    lo = src & ((3 << 2 * cls) | (3 << (16 + 2 * cls)))
+                    op, n = shifts[(wi % 2, rowhalf)]
+                    h = ((hw << n) if op == "<<" else (hw >> n)) & 0xFFFFFFFF
+                    hi = h & ((4 << 2 * cls) | (4 << (16 + 2 * cls)))
+                    r = lo | hi
+                    for elem in range(2):
+                        row, col = _fragment_owner(lane, reg, elem)
+                        val = (r >> (16 * elem)) & 0xFFFF
+                        assert val == int(q[row, 16 * kstep + col]) * 4 ** cls
+                        assert val < 1024
 
 
 def test_meta_layout_matches_fragment_rows(orc):

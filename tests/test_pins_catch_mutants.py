@@ -48,6 +48,8 @@ MUTANTS = [
      "word = (c / 64) * 128 + lane * 4 + 3 - (c % 64) / 16;", "all"),
     ("lane from the wrong feature bits (pack and unpack)",
      "const int lane = (i % 8) * 4 + (c % 8) / 2;", "const int lane = (i % 8) * 4 + (c % 4);", "all"),
+    ("3-bit upper plane ignores the row half (pack and unpack)",
+     "8 * ((c / 32) % 2) + 2 * cls + i / 8)", "8 * ((c / 32) % 2) + 2 * cls)", "all"),
     ("zero stored in the scale slot",
      "meta[base + 4 * e + 2 + hi] = z[(size_t)r * ngk + j];",
      "meta[base + 4 * e + 0 + hi] = z[(size_t)r * ngk + j];", 0),
