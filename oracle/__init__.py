@@ -15,6 +15,9 @@ What it computes (paper sections cited in ``wq_oracle.c``):
   * ``rms_scale``  unit-weight RMSNorm scale 1/sqrt(mean(x^2)+eps) per token.
   * ``down_bf16``  y = residual + h Wd^T with a bf16 Wd (the BF16/W2-GateUp
                    configuration of the accuracy experiments, Sec. 6.1), fp64.
+  * ``rope`` / ``attn_decode``  rotary embedding and one decode step of
+                   grouped-query attention over a bf16 KV cache (the rest of
+                   a decoder layer around the MLP), fp64.
   * ``merge_lora`` the merged matrix deq(W) + alpha B A (Eq. 1; Sec. 4.2 lets
                    the adapters be merged after training), fp64 then one
                    rounding to fp32, ready to be quantized again.
@@ -81,6 +84,8 @@ def _load():
                 "orc_gateup": (I, [P, I, I, I, P, P, P, P, P, P, I, P, P, P, I, D, I, D, P, P]),
                 "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
                 "orc_down_bf16": (I, [P, I, I, I, P, P, P, P]),
+                "orc_rope": (I, [P, I, I, ctypes.c_long, D]),
+                "orc_attn_decode": (I, [P, P, P, P, I, I, I, I, I, P]),
                 "orc_threads": (I, []),
                 "orc_set_threads": (None, [I]),
                 "orc_f32_to_f16_array": (None, [P, S, P]),
@@ -274,6 +279,29 @@ def down_bf16(h_bits, wd_bits, residual_bits=None):
     if _load().orc_down_bf16(_p(h), m, inter, d, _p(wd), _p(res), _p(y), _p(yb)) < 0:
         raise ValueError("orc_down_bf16: bad arguments")
     return y, yb
+
+
+def rope(x, pos: int, theta: float) -> np.ndarray:
+    """Rotary embedding of fp64 heads x [n_heads, hd] at position pos (returns a rotated copy)."""
+    out = np.array(x, dtype=np.float64, order="C", copy=True)
+    n_heads, hd = out.shape
+    if _load().orc_rope(_p(out), n_heads, hd, int(pos), float(theta)) < 0:
+        raise ValueError("orc_rope: bad arguments")
+    return out
+
+
+def attn_decode(q, k_bits, v_bits, lens) -> np.ndarray:
+    """o [B, H, hd] from fp64 q [B, H, hd] over bf16-bit caches [B, Hkv, L, hd] and lengths [B]."""
+    q = _c(q, np.float64)
+    kc, vc = _c(k_bits, np.uint16), _c(v_bits, np.uint16)
+    b, h, hd = q.shape
+    _, hkv, lmax, hd2 = kc.shape
+    assert hd2 == hd and vc.shape == kc.shape and kc.shape[0] == b
+    ln = _c(lens, np.int32)
+    o = np.empty((b, h, hd), np.float64)
+    if _load().orc_attn_decode(_p(q), _p(kc), _p(vc), _p(ln), b, h, hkv, hd, lmax, _p(o)) < 0:
+        raise ValueError("orc_attn_decode: bad arguments")
+    return o
 
 
 def threads() -> int:

@@ -498,6 +498,85 @@ int orc_down_bf16(const uint16_t *h, int m, int inter, int d, const uint16_t *wd
     return ORC_OK;
 }
 
+/* ------------------------------------------------------------------ */
+/* Decode-step attention (the rest of a decoder layer; the paper's     */
+/* throughput analysis, Sec. 5, counts its KV-cache reads among the     */
+/* operators whose cost does not depend on the weight precision).       */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Rotary position embedding of heads of dimension hd (even) at position pos,
+ * pairing element i with element i + hd/2 ("rotate half" convention):
+ *   a = pos * theta^(-2i/hd),
+ *   x'[i]        = x[i] cos a - x[i + hd/2] sin a
+ *   x'[i + hd/2] = x[i + hd/2] cos a + x[i] sin a,     i < hd/2.
+ * x: fp64 [n_heads, hd], rotated in place.
+ */
+int orc_rope(double *x, int n_heads, int hd, long pos, double theta)
+{
+    if (n_heads < 0 || hd <= 0 || hd % 2 != 0 || theta <= 0.0) return ORC_ERR_ARG;
+    const int half = hd / 2;
+    for (int h = 0; h < n_heads; ++h) {
+        double *v = x + (size_t)h * hd;
+        for (int i = 0; i < half; ++i) {
+            const double a = (double)pos * pow(theta, -2.0 * i / hd);
+            const double c = cos(a), s = sin(a);
+            const double x0 = v[i], x1 = v[i + half];
+            v[i] = x0 * c - x1 * s;
+            v[i + half] = x1 * c + x0 * s;
+        }
+    }
+    return ORC_OK;
+}
+
+/*
+ * One decode step of grouped-query attention over a bf16 KV cache: for each
+ * sequence b and query head h (kv head g = h / (n_heads / n_kv)),
+ *   s[j] = (q[b,h] . K[b,g,j]) / sqrt(hd),   j < len[b],
+ *   p    = softmax(s),   o[b,h] = sum_j p[j] V[b,g,j].
+ * q: fp64 [B, n_heads, hd].  K, V: bf16 [B, n_kv, max_len, hd].  len: [B],
+ * 1 <= len[b] <= max_len.  o: fp64 [B, n_heads, hd].  The softmax subtracts
+ * max s before exponentiating (the same value in exact arithmetic).
+ */
+int orc_attn_decode(const double *q, const uint16_t *k_cache, const uint16_t *v_cache, const int *len,
+                    int batch, int n_heads, int n_kv, int hd, int max_len, double *o)
+{
+    if (batch < 0 || n_heads <= 0 || n_kv <= 0 || n_heads % n_kv != 0 || hd <= 0 || max_len <= 0)
+        return ORC_ERR_ARG;
+    for (int b = 0; b < batch; ++b)
+        if (len[b] < 1 || len[b] > max_len) return ORC_ERR_ARG;
+    const int rep = n_heads / n_kv;
+    double *s = (double *)malloc(sizeof(double) * (size_t)max_len);
+    if (!s) return ORC_ERR_ARG;
+    for (int b = 0; b < batch; ++b)
+        for (int h = 0; h < n_heads; ++h) {
+            const int g = h / rep;
+            const double *qh = q + ((size_t)b * n_heads + h) * hd;
+            const uint16_t *kb = k_cache + ((size_t)b * n_kv + g) * max_len * hd;
+            const uint16_t *vb = v_cache + ((size_t)b * n_kv + g) * max_len * hd;
+            double mx = -INFINITY;
+            for (int j = 0; j < len[b]; ++j) {
+                double dot = 0.0;
+                for (int e = 0; e < hd; ++e) dot += qh[e] * orc_bf16_to_f64(kb[(size_t)j * hd + e]);
+                s[j] = dot / sqrt((double)hd);
+                if (s[j] > mx) mx = s[j];
+            }
+            double den = 0.0;
+            for (int j = 0; j < len[b]; ++j) {
+                s[j] = exp(s[j] - mx);
+                den += s[j];
+            }
+            double *oh = o + ((size_t)b * n_heads + h) * hd;
+            for (int e = 0; e < hd; ++e) {
+                double acc = 0.0;
+                for (int j = 0; j < len[b]; ++j) acc += s[j] * orc_bf16_to_f64(vb[(size_t)j * hd + e]);
+                oh[e] = acc / den;
+            }
+        }
+    free(s);
+    return ORC_OK;
+}
+
 /* Threads used by the OpenMP loops above (1 without OpenMP). */
 int orc_threads(void)
 {

@@ -84,6 +84,11 @@ MUTANTS = [
      "if (residual) y -= orc_bf16_to_f64(residual[(size_t)tk * d + c]);", 1),
     ("bf16 down weights transposed", "orc_bf16_to_f64(wd[(size_t)c * inter + n]);",
      "orc_bf16_to_f64(wd[(size_t)n * d + c]);", 0),
+    ("attention scores not scaled by sqrt(hd)", "s[j] = dot / sqrt((double)hd);", "s[j] = dot / (double)hd;", 0),
+    ("query heads interleaved over the key/value heads", "const int g = h / rep;", "const int g = h % n_kv;", 0),
+    ("softmax not normalized", "oh[e] = acc / den;", "oh[e] = acc;", 0),
+    ("RoPE rotates the wrong way", "v[i] = x0 * c - x1 * s;", "v[i] = x0 * c + x1 * s;", 0),
+    ("RoPE frequency exponent halved", "pow(theta, -2.0 * i / hd)", "pow(theta, -1.0 * i / hd)", 0),
     ("merge drops alpha", "w_out[(size_t)row * k + col] = (float)(w + lora_scale * ba);",
      "w_out[(size_t)row * k + col] = (float)(w + ba);", 0),
     ("merge A transposed", "orc_bf16_to_f64(lora_a[(size_t)rho * k + col]);",
