@@ -85,6 +85,7 @@ def _load():
                 "orc_down": (I, [P, I, I, I, P, P, P, I, P, P, P]),
                 "orc_down_bf16": (I, [P, I, I, I, P, P, P, P]),
                 "orc_rope": (I, [P, I, I, ctypes.c_long, D]),
+                "orc_qproj": (I, [P, I, I, P, P, P, I, I, P]),
                 "orc_attn_decode": (I, [P, P, P, P, I, I, I, I, I, P]),
                 "orc_threads": (I, []),
                 "orc_set_threads": (None, [I]),
@@ -302,6 +303,19 @@ def attn_decode(q, k_bits, v_bits, lens) -> np.ndarray:
     if _load().orc_attn_decode(_p(q), _p(kc), _p(vc), _p(ln), b, h, hkv, hd, lmax, _p(o)) < 0:
         raise ValueError("orc_attn_decode: bad arguments")
     return o
+
+
+def qproj(x, w, group: int) -> np.ndarray:
+    """out = x deq(W)^T for unrounded fp64 x [m, k]; w is a (q, s, z) tuple of an [n, k] matrix."""
+    x = _c(x, np.float64)
+    q, s, z = (_c(w[0], np.uint8), _c(w[1], np.uint16), _c(w[2], np.uint16))
+    m, k = x.shape
+    n = q.shape[0]
+    assert q.shape[1] == k
+    out = np.empty((m, n), np.float64)
+    if _load().orc_qproj(_p(x), m, k, _p(q), _p(s), _p(z), n, group, _p(out)) < 0:
+        raise ValueError("orc_qproj: bad arguments")
+    return out
 
 
 def threads() -> int:

@@ -577,6 +577,23 @@ int orc_attn_decode(const double *q, const uint16_t *k_cache, const uint16_t *v_
     return ORC_OK;
 }
 
+/*
+ * Projection of unrounded fp64 inputs through a quantized matrix:
+ *   out[t, n] = sum_k x[t, k] deq(W)[n, k],   x: fp64 [m, k], W: [n, k].
+ */
+int orc_qproj(const double *x, int m, int k, const uint8_t *q, const uint16_t *s, const uint16_t *z,
+              int n, int group, double *out)
+{
+    if (m < 0 || k <= 0 || n <= 0 || group <= 0 || k % group != 0) return ORC_ERR_ARG;
+    const int ng = k / group;
+#pragma omp parallel for schedule(static)
+    for (int r = 0; r < n; ++r)
+        for (int t = 0; t < m; ++t)
+            out[(size_t)t * n + r] = orc_qdot_f64(q + (size_t)r * k, s + (size_t)r * ng, z + (size_t)r * ng,
+                                                  k, group, x + (size_t)t * k);
+    return ORC_OK;
+}
+
 /* Threads used by the OpenMP loops above (1 without OpenMP). */
 int orc_threads(void)
 {
