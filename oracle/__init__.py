@@ -18,6 +18,10 @@ What it computes (paper sections cited in ``wq_oracle.c``):
   * ``rope`` / ``attn_decode``  rotary embedding and one decode step of
                    grouped-query attention over a bf16 KV cache (the rest of
                    a decoder layer around the MLP), fp64.
+  * ``qproj``      unrounded fp64 inputs through a quantized matrix.
+  * ``decoder``    (module) one decode step of a whole decoder layer composed
+                   from the functions here; ``moe`` (module) a mixture-of-
+                   experts MLP block composed from ``gateup`` and ``down``.
   * ``merge_lora`` the merged matrix deq(W) + alpha B A (Eq. 1; Sec. 4.2 lets
                    the adapters be merged after training), fp64 then one
                    rounding to fp32, ready to be quantized again.
