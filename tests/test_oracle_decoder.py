@@ -93,3 +93,72 @@ def test_cache_gains_one_position(orc, lens):
             changed = np.any(c0[i] != c1[i], axis=(0, 2))
             assert not np.any(np.delete(changed, n))
     assert np.all(np.isfinite(out["y"]))
+
+
+def _np_deq(w, group):
+    q, s, z = w
+    sf = np.repeat(s.view(np.float16).astype(np.float64), group, axis=1)
+    zf = np.repeat(z.view(np.float16).astype(np.float64), group, axis=1)
+    return sf * (q.astype(np.float64) - zf)
+
+
+def _bf16_round(a):
+    return torch.from_numpy(np.asarray(a, np.float64)).to(torch.bfloat16).double().numpy()
+
+
+def _rope_complex(x, pos, theta):
+    hd = x.shape[-1]
+    half = hd // 2
+    z = x[..., :half] + 1j * x[..., half:]
+    z = z * np.exp(1j * pos * theta ** (-2.0 * np.arange(half) / hd))
+    return np.concatenate([z.real, z.imag], axis=-1)
+
+
+def test_attention_path_matches_library_steps(orc):
+    """Steps 1-8 rebuilt from library routines only (numpy matmul of numpy-
+    dequantized matrices, torch rms_norm, complex RoPE, torch fp64 attention):
+    the appended key and value, the attention output and x1 must agree with
+    the composition over several cached positions."""
+    rng = np.random.default_rng(5)
+    L = _layer(orc, rng)
+    sh = L["shape"]
+    H, Hkv, hd = sh.n_heads, sh.n_kv, sh.head_dim
+    b, lmax, lens = 2, 9, [4, 8]
+    x = _bits(rng.standard_normal((b, 256)))
+    kc = _bits(rng.standard_normal((b, Hkv, lmax, hd)))
+    vc = _bits(rng.standard_normal((b, Hkv, lmax, hd)))
+    out = dec.decoder_layer_decode(x, lens, kc, vc, **L)
+
+    xf = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).double()
+    xin = torch.nn.functional.rms_norm(xf, (256,), eps=1e-6).numpy()
+    q = xin @ _np_deq(L["wq"], 128).T
+    k = xin @ _np_deq(L["wk"], 128).T
+    v = xin @ _np_deq(L["wv"], 128).T
+    norm = lambda a, n: torch.nn.functional.rms_norm(torch.from_numpy(a.reshape(b, n, hd)), (hd,), eps=1e-6).numpy()
+    q, k = norm(q, H), norm(k, Hkv)
+    for i in range(b):
+        q[i] = _rope_complex(q[i], lens[i], sh.theta)
+        k[i] = _rope_complex(k[i], lens[i], sh.theta)
+    kf = torch.from_numpy(np.ascontiguousarray(kc).view(np.int16)).view(torch.bfloat16).double().numpy().copy()
+    vf = torch.from_numpy(np.ascontiguousarray(vc).view(np.int16)).view(torch.bfloat16).double().numpy().copy()
+    x1 = np.empty((b, 256))
+    for i in range(b):
+        kf[i, :, lens[i]] = _bf16_round(k[i])
+        vf[i, :, lens[i]] = _bf16_round(v[i].reshape(Hkv, hd))
+        n = lens[i] + 1
+        kt = torch.from_numpy(kf[i, :, :n]).repeat_interleave(H // Hkv, dim=0)
+        vt = torch.from_numpy(vf[i, :, :n]).repeat_interleave(H // Hkv, dim=0)
+        o = torch.nn.functional.scaled_dot_product_attention(torch.from_numpy(q[i][:, None, :]), kt, vt)[:, 0]
+        o = _bf16_round(o.numpy().reshape(H * hd))
+        got_o = torch.from_numpy(out["o_bits"][i].view(np.int16)).view(torch.bfloat16).double().numpy()
+        np.testing.assert_allclose(got_o, o, rtol=2.0 ** -7, atol=1e-12)       # at most one bf16 rounding flip
+        assert np.mean(got_o == o) > 0.95
+        x1[i] = xf[i].numpy() + got_o @ _np_deq(L["wo"], 128).T
+    got_k = torch.from_numpy(out["k_cache"].view(np.int16)).view(torch.bfloat16).double().numpy()
+    got_v = torch.from_numpy(out["v_cache"].view(np.int16)).view(torch.bfloat16).double().numpy()
+    for i in range(b):
+        np.testing.assert_allclose(got_k[i, :, lens[i]], kf[i, :, lens[i]], rtol=2.0 ** -7, atol=1e-12)
+        np.testing.assert_allclose(got_v[i, :, lens[i]], vf[i, :, lens[i]], rtol=2.0 ** -7, atol=1e-12)
+        assert np.mean(got_k[i, :, lens[i]] == kf[i, :, lens[i]]) > 0.95
+    got_x1 = torch.from_numpy(out["x1_bits"].view(np.int16)).view(torch.bfloat16).double().numpy()
+    np.testing.assert_allclose(got_x1, _bf16_round(x1), rtol=2.0 ** -7, atol=1e-12)
