@@ -193,15 +193,22 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
  * buffer), or a plugin that must not grow its host process's memory.  The
  * paper has no counterpart to this call; it is a deployment convenience.
  *
- * Same arguments and results as wq_gateup_w2_lora minus ws / ws_bytes.  The
- * scratch it needs (per-16-feature RMSNorm and LoRA-A partial sums of x,
- * split-K partial sums and arrival counters) lives in a fixed array of WQ_NOALLOC_SCRATCH_BYTES
- * bytes inside the library, which every GPU that loads the library keeps
- * until the process exits.  A call whose layer needs more scratch than that
- * returns WQ_ERR_UNSUPPORTED and launches nothing.
+ * Same arguments and results as wq_gateup_w2_lora minus ws / ws_bytes, for
+ * the decode token counts 1 <= m <= 16 (the dequant-GEMV path).  The scratch
+ * it needs (per-16-feature RMSNorm and LoRA-A partial sums of x, split-K
+ * partial sums and arrival counters) lives in a fixed array of
+ * WQ_NOALLOC_SCRATCH_BYTES bytes inside the library, which every GPU that
+ * loads the library keeps until the process exits.  It returns
+ * WQ_ERR_UNSUPPORTED and launches nothing when
+ *   - m > 16 (wq_gateup_w2_lora takes the dequant-GEMM path there),
+ *   - the layer shape has no dequant-GEMV launch configuration at this m
+ *     (wq_gateup_w2_lora takes the dequant-GEMM path for it), or
+ *   - the layer needs more scratch than the array holds.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress, which may load the library's device code); make
- *     that first call before any stream capture.
+ *     that first call before any stream capture.  The address is kept for
+ *     the life of the process: do not use this call on a device after a
+ *     device reset (cudaDeviceReset) in the same process.
  *   - Every call clears the array's arrival counters (cudaMemsetAsync on
  *     `stream`) and then reuses the array, which keeps the previous call's
  *     contents otherwise.  All calls share the one array: calls that can

@@ -577,9 +577,14 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
   if (m == 0) return ok();
   if (!x || !h) return fail(WQ_ERR_ARG, "null x or h");
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
-  if (m > kMaxTokens)
+  if (m > kGemvPreferTokens)
     return fail(WQ_ERR_UNSUPPORTED, "m=%d: the built-in scratch serves the decode path (m <= %d; use wq_gateup_w2_lora)",
-                m, kMaxTokens);
+                m, kGemvPreferTokens);
+  GemvPlan plan;
+  if (!plan_gemv(kGateUpW2, gate->n, gate->k, m, gate->group, r, num_sms(), &plan))
+    return fail(WQ_ERR_UNSUPPORTED,
+                "no decode launch configuration fits [%d x %d], m=%d, group %d (use wq_gateup_w2_lora, which can take "
+                "the dequant-GEMM path)", gate->n, gate->k, m, gate->group);
   WsLayout L;
   if (!ws_layout(m, gate->k, gate->n, &L, true)) return fail(WQ_ERR_CUDA, "cannot query the current device");
   if (L.total > (size_t)WQ_NOALLOC_SCRATCH_BYTES)

@@ -2,8 +2,9 @@
 MLP with 2-bit gate/up and 4-bit down), through the C ABI.
 
 Shapes span several row tiles and feature blocks, ragged row and feature
-tails, every supported group size, token counts 1..64 and both panel modes
-(one CTA per row block, and split panels finished by the last-arriving CTA).
+tails, every supported group size and both panel modes (one CTA per row
+block, and split panels finished by the last-arriving CTA).  The GEMV kernels
+take 1..16 tokens; the 17/33/64-token cases here take the dequant-GEMM path.
 """
 import numpy as np
 import pytest

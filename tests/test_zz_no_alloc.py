@@ -49,6 +49,16 @@ def test_noalloc_matches_workspace_entry_point(d, inter, group, r, m, prenorm):
     assert wq.device_status() == 0
     _close(h1, ref, "first no-alloc call")
     _close(h2, ref, "second no-alloc call")
+    if d == 2560:
+        # the Qwen3-4B-shaped case also against the fp64 oracle, with the GEMV tests' bound
+        import oracle as orc
+        from tests.gpu_util import check_bf16
+        qg = orc.quantize(wg.cpu().numpy(), group, 2)[:3]
+        qu = orc.quantize(wu.cpu().numpy(), group, 2)[:3]
+        ora, _ = orc.gateup(synth.bf16_bits(x.cpu()), qg, qu, group, synth.bf16_bits(a.cpu()),
+                            synth.bf16_bits(bg.cpu()), synth.bf16_bits(bu.cpu()), lora_scale=2.0, prenorm=prenorm)
+        check_bf16(h1, ora, "no-alloc call vs oracle")
+        check_bf16(h2, ora, "second no-alloc call vs oracle")
 
 
 def test_noalloc_rejects_a_layer_beyond_its_scratch():
@@ -65,3 +75,19 @@ def test_noalloc_rejects_a_layer_beyond_its_scratch():
     with pytest.raises(wq.WQError) as e:
         wq.gateup_w2_lora_noalloc(x, q, q)
     assert e.value.status == -4 and "scratch" in str(e.value)
+
+
+def test_noalloc_rejects_more_than_16_tokens():
+    """Above 16 tokens the workspace entry point takes the dequant-GEMM path;
+    the built-in scratch only serves the decode path, so the call refuses."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04238_gb300 import wq
+
+    d, inter = 256, 768
+    q = wq.empty_qweight(inter, d, 64, 2)
+    for m in (17, 33, 64):
+        x = torch.zeros((m, d), dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(wq.WQError) as e:
+            wq.gateup_w2_lora_noalloc(x, q, q)
+        assert e.value.status == -4 and "m <= 16" in str(e.value)
