@@ -57,7 +57,10 @@ typedef enum {
 } wq_status;
 
 /* Flags of wq_gateup_* and wq_mlp_forward. */
-#define WQ_PRENORM 1u   /* unit-weight RMSNorm (eps 1e-6) of the MLP input first */
+#define WQ_PRENORM 1u       /* unit-weight RMSNorm (eps 1e-6) of the MLP input first */
+#define WQ_LAUNCH_CHAIN 2u  /* wq_mlp_forward*: run the per-layer launch chain even where the
+                               single-launch stack kernel applies (same results; for tests and
+                               comparisons) */
 
 /* Output element types of wq_down_w4. */
 #define WQ_BF16 0
@@ -263,6 +266,35 @@ wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, c
  */
 wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
                          unsigned flags, void *y, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * wq_mlp_forward that also returns every layer's output (the hidden states of
+ * the stack) and, optionally, every layer's MLP activation h:
+ *   states:   bf16 [n_layers][m][d] (device, 16-byte aligned), states[l] = x_{l+1};
+ *   h_states: bf16 [n_layers][m][inter] or NULL, h_states[l] = layer l's
+ *             h = SiLU(g) * u as stored for its down projection.
+ * y receives x_L as well.  Same launches as wq_mlp_forward with each layer
+ * writing into its own slots, plus one device-to-device copy of the last
+ * slot into y.
+ */
+wq_status wq_mlp_forward_states(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
+                                unsigned flags, void *y, void *states, void *h_states, void *ws, size_t ws_bytes,
+                                void *stream);
+
+/*
+ * How wq_mlp_forward runs this stack on the current device (for tests and
+ * tuning; validates like wq_mlp_forward and launches nothing).  info[16]:
+ *   [0]      route: 0 = per-layer dequant-GEMV launch chain,
+ *                   1 = per-layer dequant-GEMM launch chain
+ *   [1..6]   route 0: layer 0's gate/up launch: row tiles per CTA, blocks per
+ *            panel, warps along k, row tiles per warp, panels, CTAs
+ *   [7..12]  route 0: layer 0's down launch (writing layer 1's partial sums
+ *            when there is a layer 1): the same fields
+ *   [13]     route 0: 1 when the gate/up launch hands the down launch its
+ *            ready binary16 panel of h
+ *   other entries: -1
+ */
+wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, int64_t info[16]);
 
 /*
  * Describes how a dequant-GEMV launch of the current device splits its work

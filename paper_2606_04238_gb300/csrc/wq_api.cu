@@ -644,13 +644,17 @@ wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, c
   return ok();
 }
 
-wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, void *y,
-                         void *ws, size_t ws_bytes, void *stream) {
+}  // extern "C"
+
+namespace {
+
+// Validates a stack and fills in its shape (d, inter).
+wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, int *d_out, int *inter_out) {
   wq_status st = check_tokens(m);
   if (st != WQ_OK) return st;
   if (n_layers < 0) return fail(WQ_ERR_ARG, "n_layers=%d is negative", n_layers);
   if (n_layers > 0 && !layers) return fail(WQ_ERR_ARG, "null layer array");
-  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (flags & ~(WQ_PRENORM | WQ_LAUNCH_CHAIN)) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
   int d = 0, inter = 0;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
@@ -672,42 +676,81 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
                   inter, d);
     }
   }
+  *d_out = d;
+  *inter_out = inter;
+  return WQ_OK;
+}
+
+// How a stack runs: the per-layer dequant-GEMV launch chain or the
+// dequant-GEMM launch chain (every layer's launches need a GEMV plan for the
+// first; above kGemvPreferTokens tokens the second).
+enum StackRoute { kRouteGemvChain = 0, kRouteGemmChain = 1 };
+
+StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags) {
+  if (m > kGemvPreferTokens) return kRouteGemmChain;
+  for (int l = 0; l < n_layers; ++l) {
+    const wq_mlp_layer &Ly = layers[l];
+    const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
+    if (gateup_uses_gemm(Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4, m, &Ly.gate, Ly.r) ||
+        down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0))
+      return kRouteGemmChain;
+  }
+  return kRouteGemvChain;
+}
+
+// wq_mlp_forward, with every layer's output also stored in `states`
+// (bf16 [n_layers][m][d]) when it is not null.
+wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, void *y,
+                           void *states, void *h_states, void *ws, size_t ws_bytes, void *stream) {
+  int d = 0, inter = 0;
+  wq_status st = check_stack(m, layers, n_layers, flags, &d, &inter);
+  if (st != WQ_OK) return st;
   if (m == 0 || n_layers == 0) {
     if (n_layers == 0 && m > 0 && x != y) return fail(WQ_ERR_ARG, "n_layers=0 needs y == x");
     return ok();
   }
   if (!x || !y) return fail(WQ_ERR_ARG, "null x or y");
-  if (!aligned16(x) || !aligned16(y)) return fail(WQ_ERR_ALIGN, "x or y not 16-byte aligned");
+  if (!aligned16(x) || !aligned16(y) || (states && !aligned16(states)) || (h_states && !aligned16(h_states)))
+    return fail(WQ_ERR_ALIGN, "x, y, states or h_states not 16-byte aligned");
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, d, inter, &L)) != WQ_OK) return st;
   uint8_t *w8 = static_cast<uint8_t *>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // the GEMV chain needs a plan for every layer's launches; otherwise the
-  // whole stack takes the dequant-GEMM chain
-  bool gemm_chain = m > kGemvPreferTokens;
-  for (int l = 0; l < n_layers && !gemm_chain; ++l) {
-    const wq_mlp_layer &Ly = layers[l];
-    const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
-    gemm_chain = gateup_uses_gemm(Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4, m, &Ly.gate, Ly.r) ||
-                 down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0);
-  }
-  if (gemm_chain) {
+  const size_t state_bytes = (size_t)m * d * 2;
+  // output of layer l: the caller's state slot, y for the last layer, else a ping-pong buffer
+  auto layer_out = [&](int l) -> void * {
+    if (states) return static_cast<uint8_t *>(states) + (size_t)l * state_bytes;
+    return (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
+  };
+  // h of layer l: the caller's slot, else the workspace buffer
+  auto layer_h = [&](int l) -> void * {
+    return h_states ? static_cast<uint8_t *>(h_states) + (size_t)l * m * inter * 2 : (void *)(w8 + L.h);
+  };
+  auto finish = [&]() -> wq_status {
+    if (states) {
+      cudaError_t e = cudaMemcpyAsync(y, static_cast<uint8_t *>(states) + (size_t)(n_layers - 1) * state_bytes,
+                                      state_bytes, cudaMemcpyDeviceToDevice, s);
+      if (e != cudaSuccess) return cuda_fail(e, "copy of the last state to y");
+    }
+    return ok();
+  };
+  if (stack_route(m, layers, n_layers, flags) == kRouteGemmChain) {
     // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up (h also in
     // binary16), down with the residual
     const void *cur = x;
     for (int l = 0; l < n_layers; ++l) {
       const wq_mlp_layer &Ly = layers[l];
-      void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
+      void *out = layer_out(l);
       const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
       uint16_t *h16 = reinterpret_cast<uint16_t *>(w8 + L.h16);
       st = run_gateup_gemm(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale,
-                           flags, w8 + L.h, h16, L, w8, s);
+                           flags, layer_h(l), h16, L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
       st = run_down_gemm(nullptr, h16, m, &Ly.down, cur, out, 0, L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
       cur = out;
     }
-    return ok();
+    return finish();
   }
   const bool prenorm = (flags & WQ_PRENORM) != 0;
   float *tp = reinterpret_cast<float *>(w8 + L.tp);
@@ -719,10 +762,10 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
     if (e != cudaSuccess) return cuda_fail(e, "tile-partials launch");
   }
   const void *cur = x;
-  void *hbuf = w8 + L.h;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
-    void *out = (l == n_layers - 1) ? y : (void *)(w8 + ((l & 1) ? L.xb : L.xa));
+    void *out = layer_out(l);
+    void *hbuf = layer_h(l);
     const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
     const bool need_tp = prenorm || Ly.r > 0;
     const wq_mlp_layer *nx = l + 1 < n_layers ? &layers[l + 1] : nullptr;
@@ -736,6 +779,48 @@ wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n
                   w8, s, panel);
     if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     cur = out;
+  }
+  return finish();
+}
+
+}  // namespace
+
+extern "C" {
+
+wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, void *y,
+                         void *ws, size_t ws_bytes, void *stream) {
+  return mlp_forward_impl(x, m, layers, n_layers, flags, y, nullptr, nullptr, ws, ws_bytes, stream);
+}
+
+wq_status wq_mlp_forward_states(const void *x, int m, const wq_mlp_layer *layers, int n_layers, unsigned flags,
+                                void *y, void *states, void *h_states, void *ws, size_t ws_bytes, void *stream) {
+  if (!states && n_layers > 0 && m > 0) return fail(WQ_ERR_ARG, "null states");
+  return mlp_forward_impl(x, m, layers, n_layers, flags, y, states, h_states, ws, ws_bytes, stream);
+}
+
+wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, int64_t info[16]) {
+  if (!info) return fail(WQ_ERR_ARG, "null info array");
+  int d = 0, inter = 0;
+  wq_status st = check_stack(m, layers, n_layers, flags, &d, &inter);
+  if (st != WQ_OK) return st;
+  if (m <= 0 || n_layers <= 0) return fail(WQ_ERR_ARG, "m=%d, n_layers=%d: nothing runs", m, n_layers);
+  const int sms = num_sms();
+  if (sms <= 0) return fail(WQ_ERR_CUDA, "cannot query the current device");
+  for (int i = 0; i < 16; ++i) info[i] = -1;
+  const StackRoute route = stack_route(m, layers, n_layers, flags);
+  info[0] = route;
+  if (route == kRouteGemvChain) {
+    const wq_mlp_layer &L0 = layers[0];
+    const GemvKind kind = L0.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+    const bool next_tp = n_layers > 1 && ((flags & WQ_PRENORM) || layers[1].r > 0);
+    const int r_next = next_tp ? layers[1].r : 0;
+    GemvPlan pg, pd;
+    if (!plan_gemv(kind, L0.gate.n, L0.gate.k, m, L0.gate.group, L0.r, sms, &pg) ||
+        !plan_gemv(kDownW4, L0.down.n, L0.down.k, m, L0.down.group, r_next, sms, &pd))
+      return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits");
+    const int64_t v[13] = {pg.RB, pg.KP, pg.WK, pg.TPW, pg.P, pg.units, pd.RB, pd.KP, pd.WK, pd.TPW, pd.P, pd.units,
+                           chain_panel_ok(kind, m, L0.gate, L0.r, L0.down, r_next) ? 1 : 0};
+    for (int i = 0; i < 13; ++i) info[1 + i] = v[i];
   }
   return ok();
 }

@@ -17,6 +17,7 @@ import torch
 from . import _build
 
 WQ_PRENORM = 1
+WQ_LAUNCH_CHAIN = 2
 WQ_BF16 = 0
 WQ_F32 = 1
 
@@ -73,6 +74,8 @@ def lib():
             "wq_down_w4": (I, [P, I, QP, P, P, I, P, S, P]),
             "wq_down_bf16": (I, [P, I, P, I, I, P, P, I, P]),
             "wq_mlp_forward": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, S, P]),
+            "wq_mlp_forward_states": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, P, P, S, P]),
+            "wq_mlp_forward_info": (I, [I, ctypes.POINTER(_MLPLayer), I, U, ctypes.POINTER(ctypes.c_int64)]),
             "wq_plan_info": (I, [I, I, I, I, I, I, ctypes.POINTER(ctypes.c_int64)]),
             "wq_last_error": (ctypes.c_char_p, []),
             "wq_device_status": (I, [ctypes.POINTER(I)]),
@@ -298,8 +301,14 @@ class LayerTable:
         self.array = (_MLPLayer * max(1, len(self.layers)))(*[l.c() for l in self.layers])
 
 
-def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTable | None = None):
-    """Stack of gated-MLP layers (wq_mlp_forward) on the current stream."""
+def _stack_flags(prenorm: bool, chain: bool) -> int:
+    return (WQ_PRENORM if prenorm else 0) | (WQ_LAUNCH_CHAIN if chain else 0)
+
+
+def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTable | None = None,
+                chain: bool = False):
+    """Stack of gated-MLP layers (wq_mlp_forward) on the current stream; chain=True
+    asks for the per-layer launch chain (WQ_LAUNCH_CHAIN)."""
     m, d = x.shape
     if table is None:
         table = LayerTable(layers)
@@ -308,9 +317,52 @@ def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTa
     if ws is None:
         l0 = table.layers[0]
         ws = workspace(max(m, 1), d, l0.gate.n, l0.r, device=x.device)
-    _check(lib().wq_mlp_forward(_ptr(x), m, table.array, len(table.layers), WQ_PRENORM if prenorm else 0, _ptr(y),
+    _check(lib().wq_mlp_forward(_ptr(x), m, table.array, len(table.layers), _stack_flags(prenorm, chain), _ptr(y),
                                 _ptr(ws), ws.numel(), _stream()))
     return y
+
+
+def mlp_forward_states(x, layers, prenorm: bool = True, states=None, h_states=None, y=None, ws=None,
+                       table: LayerTable | None = None, chain: bool = False, with_h: bool = False):
+    """wq_mlp_forward_states: the stack plus every layer's output, bf16 [n_layers, m, d], and with
+    with_h=True every layer's h, bf16 [n_layers, m, inter].  Returns (y, states, h_states)."""
+    m, d = x.shape
+    if table is None:
+        table = LayerTable(layers)
+    n = len(table.layers)
+    inter = table.layers[0].gate.n
+    if states is None:
+        states = torch.empty((n, m, d), dtype=torch.bfloat16, device=x.device)
+    if h_states is None and with_h:
+        h_states = torch.empty((n, m, inter), dtype=torch.bfloat16, device=x.device)
+    if y is None:
+        y = torch.empty_like(x)
+    if ws is None:
+        l0 = table.layers[0]
+        ws = workspace(max(m, 1), d, l0.gate.n, l0.r, device=x.device)
+    _check(lib().wq_mlp_forward_states(_ptr(x), m, table.array, n, _stack_flags(prenorm, chain), _ptr(y),
+                                       _ptr(states), _ptr(h_states), _ptr(ws), ws.numel(), _stream()))
+    return y, states, h_states
+
+
+ROUTE_GEMV_CHAIN, ROUTE_GEMM_CHAIN = 0, 1
+_STEP_FIELDS = ("rb", "kp", "wk", "tpw", "panels", "ctas")
+
+
+def mlp_forward_info(m: int, layers, prenorm: bool = True, table: LayerTable | None = None,
+                     chain: bool = False) -> dict:
+    """How wq_mlp_forward would run this stack (wq_mlp_forward_info)."""
+    if table is None:
+        table = LayerTable(layers)
+    arr = (ctypes.c_int64 * 16)()
+    _check(lib().wq_mlp_forward_info(m, table.array, len(table.layers), _stack_flags(prenorm, chain), arr))
+    v = list(arr)
+    out = {"route": v[0]}
+    if v[0] == ROUTE_GEMV_CHAIN:
+        out["gateup"] = dict(zip(_STEP_FIELDS, v[1:7]))
+        out["down"] = dict(zip(_STEP_FIELDS, v[7:13]))
+        out["panel"] = bool(v[13])
+    return out
 
 
 PLAN_FIELDS = ("row_tiles", "kblocks", "rb", "kp", "wk", "panels", "ctas", "threads", "smem", "tok_chunk")
