@@ -13,6 +13,7 @@
 #include "wq.h"
 #include "wq_internal.h"
 #include "wq_launch.h"
+#include "wq_stack.h"
 
 using namespace wq;
 
@@ -68,10 +69,16 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
 
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
-  size_t cnt1, cnt2, tp, xa, xb, h, hq, hsc, hxs, part1, part2;
+  // arrival counters: at fixed offsets for every token count (zero once, kept
+  // at zero -- or, for the stack kernel's, at a multiple of its grid -- by the calls)
+  size_t cnt1, cnt2, sctr, sk_cnt;
+  size_t tp, xa, xb, h, hq, hsc, hxs, part1, part2;
   // dequant-GEMM path (m > kMaxTokens, or a shape the GEMV path has no plan for)
-  size_t x16, rs, ta, h16, sk_cnt, sk_part;
+  size_t x16, rs, ta, h16, sk_part;
   bool gemm;  // the GEMM buffers are laid out
+  // single-launch stack (1..8 tokens)
+  size_t sxw, stp, shg, spart, sxc;
+  bool stack;
   size_t total;
 };
 
@@ -111,33 +118,56 @@ bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2, bool *all_fit
   return true;
 }
 
+// The counter block every layout starts with: the GEMV split-panel counters
+// of gate/up and down, the stack kernel's grid-barrier counter and the
+// stream-K tile counters of the GEMM path (sized for its largest token count).
+size_t counter_block(int d, int inter, WsLayout *L) {
+  size_t off = 0;
+  L->cnt1 = off;   off = up256(off + (size_t)((inter + 15) / 16) * 4);
+  L->cnt2 = off;   off = up256(off + (size_t)((d + 15) / 16) * 4);
+  L->sctr = off;   off = up256(off + 8);
+  const size_t cnt = std::max(gemm_counters(kMaxGemmTokens, inter), gemm_counters(kMaxGemmTokens, d));
+  L->sk_cnt = off; off = up256(off + cnt * 4);
+  return off;
+}
+
 // The dequant-GEMM buffers from offset `off`: binary16 copies of the GEMM
 // inputs, RMSNorm scales, the LoRA-A products and the stream-K scratch.
 bool gemm_layout(int m, int d, int inter, size_t off, WsLayout *L) {
   const size_t lda = (size_t)(std::max(d, inter) + 127) / 128 * 128, ldi = (size_t)(inter + 127) / 128 * 128;
   const int sms = num_sms();
   if (sms <= 0) return false;
-  const size_t cnt = std::max(gemm_counters(m, inter), gemm_counters(m, d));
   const size_t part = std::max(gemm_scratch_floats(m, inter, d, 2, sms), gemm_scratch_floats(m, d, inter, 1, sms));
   L->x16 = off;     off = up256(off + (size_t)m * lda * 2);
   L->rs = off;      off = up256(off + (size_t)m * 4);
   L->ta = off;      off = up256(off + (size_t)m * 2 * kMaxRank * 2);
   L->h16 = off;     off = up256(off + (size_t)m * ldi * 2);
-  L->sk_cnt = off;  off = up256(off + cnt * 4);
   L->sk_part = off; off = up256(off + part * 4);
   L->gemm = true;
   L->total = off;
   return true;
 }
 
-// The arrival counters come first: their offsets depend on (d, inter) only,
-// so a workspace zeroed once stays valid for every token count.
+// The single-launch stack's buffers from offset `off` (1..8 tokens of a
+// shape it can take).
+void stack_layout(int m, int d, int inter, size_t off, WsLayout *L) {
+  if (m < 1 || m > 8 || d % 128 != 0 || inter % 64 != 0) return;
+  const size_t Qp = WQ_TP_STRIDE(kMaxRank);
+  L->sxw = off;   off = up256(off + (size_t)m * d * 2);
+  L->stp = off;   off = up256(off + (size_t)(d / 16) * m * Qp * 4);
+  L->shg = off;   off = up256(off + (size_t)m * inter * 2);
+  L->spart = off; off = up256(off + (size_t)(inter / 64) * m * d * 4);
+  L->sxc = off;   off = up256(off + (size_t)m * d * 2);
+  L->stack = true;
+  L->total = off;
+}
+
 // gemv_only: the decode path's buffers alone (the call without a workspace).
 bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   *L = WsLayout{};
+  size_t off = counter_block(d, inter, L);
   if (m > kMaxTokens) {
     // dequant-GEMM path: the stack's bf16 intermediates, then the GEMM buffers
-    size_t off = 0;
     L->xa = off;  off = up256(off + (size_t)m * d * 2);
     L->xb = off;  off = up256(off + (size_t)m * d * 2);
     L->h = off;   off = up256(off + (size_t)m * inter * 2);
@@ -146,9 +176,6 @@ bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   size_t p1, p2;
   bool all_fit = true;
   if (!max_partials(m, d, inter, &p1, &p2, &all_fit)) return false;
-  size_t off = 0;
-  L->cnt1 = off; off = up256(off + (size_t)((inter + 15) / 16) * 4);
-  L->cnt2 = off; off = up256(off + (size_t)((d + 15) / 16) * 4);
   L->tp = off;   off = up256(off + (size_t)((d + 15) / 16) * m * WQ_TP_STRIDE(kMaxRank) * 4);
   L->xa = off;   off = up256(off + (size_t)m * d * 2);
   L->xb = off;   off = up256(off + (size_t)m * d * 2);
@@ -159,9 +186,14 @@ bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   L->part1 = off; off = up256(off + p1);
   L->part2 = off; off = up256(off + p2);
   L->total = off;
+  if (gemv_only) return true;
   // above kGemvPreferTokens, or for a shape that lacks a GEMV plan for some
   // group or rank at this token count, the calls take the dequant-GEMM path
-  if (!gemv_only && (m > kGemvPreferTokens || !all_fit)) return gemm_layout(m, d, inter, off, L);
+  if (m > kGemvPreferTokens || !all_fit) {
+    if (!gemm_layout(m, d, inter, off, L)) return false;
+    off = L->total;
+  }
+  stack_layout(m, d, inter, off, L);
   return true;
 }
 
@@ -291,7 +323,7 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
   a.nb_out = (size_t)m * down->n * (y_f32 ? 4 : 2);
   a.nb_an = (size_t)2 * rr * down->n * 2;
   a.nb_tp_out = tp_out ? (size_t)((down->n + 15) / 16) * m * WQ_TP_STRIDE(rr) * 4 : 0;
-  a.nb_part = L.total - L.part2;
+  a.nb_part = (L.gemm ? L.x16 : L.stack ? L.sxw : L.total) - L.part2;
   a.nb_cnt = (size_t)((down->n + 15) / 16) * 4;
   cudaError_t e = launch_gemv(kDownW4, plan, a, s, true);
   if (e != cudaSuccess) return cuda_fail(e, "down launch");
@@ -681,12 +713,40 @@ wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned 
   return WQ_OK;
 }
 
-// How a stack runs: the per-layer dequant-GEMV launch chain or the
+// How a stack runs: the per-layer dequant-GEMV launch chain, the
 // dequant-GEMM launch chain (every layer's launches need a GEMV plan for the
-// first; above kGemvPreferTokens tokens the second).
-enum StackRoute { kRouteGemvChain = 0, kRouteGemmChain = 1 };
+// first; above kGemvPreferTokens tokens the second), or the single-launch
+// stack kernel (1..8 tokens, every layer with the same bits, groups and rank,
+// unless the caller asks for the chain).
+enum StackRoute { kRouteGemvChain = 0, kRouteGemmChain = 1, kRouteStack = 2 };
+
+bool cooperative_ok() {
+  static int cached[64] = {0};  // 0 unknown, 1 yes, -1 no
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (cached[dev] == 0) {
+    int v = 0;
+    cached[dev] = cudaDeviceGetAttribute(&v, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && v ? 1 : -1;
+  }
+  return cached[dev] > 0;
+}
+
+bool stack_kernel_plan(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, StackPlan *plan) {
+  if ((flags & WQ_LAUNCH_CHAIN) || m < 1 || m > 8 || n_layers < 1) return false;
+  const wq_mlp_layer &L0 = layers[0];
+  for (int l = 0; l < n_layers; ++l) {
+    const wq_mlp_layer &Ly = layers[l];
+    if (Ly.gate.bits != L0.gate.bits || Ly.gate.group != L0.gate.group || Ly.down.group != L0.down.group ||
+        Ly.r != L0.r)
+      return false;
+  }
+  if (!cooperative_ok()) return false;
+  return stack_plan(m, L0.gate.k, L0.gate.n, L0.r, L0.gate.bits, L0.gate.group, L0.down.group, num_sms(), plan);
+}
 
 StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags) {
+  StackPlan sp;
+  if (stack_kernel_plan(m, layers, n_layers, flags, &sp)) return kRouteStack;
   if (m > kGemvPreferTokens) return kRouteGemmChain;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
@@ -734,7 +794,57 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     }
     return ok();
   };
-  if (stack_route(m, layers, n_layers, flags) == kRouteGemmChain) {
+  const StackRoute route = stack_route(m, layers, n_layers, flags);
+  if (route == kRouteStack) {
+    StackPlan sp;
+    if (!stack_kernel_plan(m, layers, n_layers, flags, &sp) || !L.stack)
+      return fail(WQ_ERR_UNSUPPORTED, "single-launch stack: no plan or workspace layout");
+    // launches of up to kStackMaxLayers layers; each takes x_in and gives y_out
+    const void *cur = x;
+    for (int l0 = 0; l0 < n_layers; l0 += kStackMaxLayers) {
+      const int nl = std::min(kStackMaxLayers, n_layers - l0);
+      const bool last_launch = l0 + nl == n_layers;
+      StackArgs a = {};
+      a.M = m;
+      a.d = d;
+      a.inter = inter;
+      a.r = layers[0].r;
+      a.g_gu = layers[0].gate.group;
+      a.g_dn = layers[0].down.group;
+      a.bits_gu = layers[0].gate.bits;
+      a.n_layers = nl;
+      a.prenorm = (flags & WQ_PRENORM) ? 1 : 0;
+      a.x_in = static_cast<const uint16_t *>(cur);
+      a.y_out = reinterpret_cast<uint16_t *>(last_launch ? static_cast<uint8_t *>(y) : w8 + L.sxc);
+      a.states = states ? reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(states) + (size_t)l0 * state_bytes) : nullptr;
+      a.h_states = h_states ? reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(h_states) + (size_t)l0 * m * inter * 2)
+                            : nullptr;
+      a.xw = reinterpret_cast<uint16_t *>(w8 + L.sxw);
+      a.tp = reinterpret_cast<float *>(w8 + L.stp);
+      a.hg = reinterpret_cast<uint16_t *>(w8 + L.shg);
+      a.part = reinterpret_cast<float *>(w8 + L.spart);
+      a.ctr = reinterpret_cast<unsigned long long *>(w8 + L.sctr);
+      for (int l = 0; l < nl; ++l) {
+        const wq_mlp_layer &Ly = layers[l0 + l];
+        StackLayerDev &D = a.L[l];
+        D.codes[0] = reinterpret_cast<const uint8_t *>(Ly.gate.codes);
+        D.codes[1] = reinterpret_cast<const uint8_t *>(Ly.up.codes);
+        D.codes[2] = reinterpret_cast<const uint8_t *>(Ly.down.codes);
+        D.meta[0] = reinterpret_cast<const uint8_t *>(Ly.gate.meta);
+        D.meta[1] = reinterpret_cast<const uint8_t *>(Ly.up.meta);
+        D.meta[2] = reinterpret_cast<const uint8_t *>(Ly.down.meta);
+        D.lora_a = static_cast<const uint16_t *>(Ly.lora_a);
+        D.lora_b[0] = static_cast<const uint16_t *>(Ly.lora_b_gate);
+        D.lora_b[1] = static_cast<const uint16_t *>(Ly.lora_b_up);
+        D.lora_scale = Ly.lora_scale;
+      }
+      cudaError_t e = launch_stack(a, sp, s);
+      if (e != cudaSuccess) return cuda_fail(e, "single-launch stack");
+      cur = a.y_out;
+    }
+    return ok();
+  }
+  if (route == kRouteGemmChain) {
     // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up (h also in
     // binary16), down with the residual
     const void *cur = x;
@@ -809,6 +919,12 @@ wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, u
   for (int i = 0; i < 16; ++i) info[i] = -1;
   const StackRoute route = stack_route(m, layers, n_layers, flags);
   info[0] = route;
+  if (route == kRouteStack) {
+    StackPlan sp;
+    if (!stack_kernel_plan(m, layers, n_layers, flags, &sp)) return fail(WQ_ERR_UNSUPPORTED, "no stack plan");
+    const int64_t v[7] = {sp.G, sp.NS, sp.SB, sp.h_barrier, sp.WPT, sp.Tmax, (int64_t)sp.smem};
+    for (int i = 0; i < 7; ++i) info[1 + i] = v[i];
+  }
   if (route == kRouteGemvChain) {
     const wq_mlp_layer &L0 = layers[0];
     const GemvKind kind = L0.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
@@ -855,6 +971,9 @@ wq_status wq_device_status(int *status) {
   if (e != cudaSuccess) return cuda_fail(e, "device status read");
   int g = 0;
   e = read_gemm_status(&g);
+  if (e != cudaSuccess) return cuda_fail(e, "device status read");
+  if (*status == 0) *status = g;
+  e = read_stack_status(&g);
   if (e != cudaSuccess) return cuda_fail(e, "device status read");
   if (*status == 0) *status = g;
   return ok();

@@ -345,7 +345,7 @@ def mlp_forward_states(x, layers, prenorm: bool = True, states=None, h_states=No
     return y, states, h_states
 
 
-ROUTE_GEMV_CHAIN, ROUTE_GEMM_CHAIN = 0, 1
+ROUTE_GEMV_CHAIN, ROUTE_GEMM_CHAIN, ROUTE_STACK = 0, 1, 2
 _STEP_FIELDS = ("rb", "kp", "wk", "tpw", "panels", "ctas")
 
 
@@ -358,6 +358,9 @@ def mlp_forward_info(m: int, layers, prenorm: bool = True, table: LayerTable | N
     _check(lib().wq_mlp_forward_info(m, table.array, len(table.layers), _stack_flags(prenorm, chain), arr))
     v = list(arr)
     out = {"route": v[0]}
+    if v[0] == ROUTE_STACK:
+        out["stack"] = dict(zip(("ctas", "stages", "stage_bytes", "h_barrier", "warps_per_tile", "tiles_per_cta",
+                                 "smem"), v[1:8]))
     if v[0] == ROUTE_GEMV_CHAIN:
         out["gateup"] = dict(zip(_STEP_FIELDS, v[1:7]))
         out["down"] = dict(zip(_STEP_FIELDS, v[7:13]))
