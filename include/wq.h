@@ -59,8 +59,10 @@ typedef enum {
 /* Flags of wq_gateup_* and wq_mlp_forward. */
 #define WQ_PRENORM 1u       /* unit-weight RMSNorm (eps 1e-6) of the MLP input first */
 #define WQ_LAUNCH_CHAIN 2u  /* wq_mlp_forward*: run the per-layer launch chain even where the
-                               single-launch stack kernel applies (same results; for tests and
-                               comparisons) */
+                               single-launch stack kernel would be chosen (for tests and comparisons) */
+#define WQ_LAUNCH_STACK 4u  /* wq_mlp_forward*: run the single-launch stack kernel wherever it can
+                               take the stack (1..8 tokens, every layer with the same bits, groups
+                               and rank), also where the launch chain is the measured-faster route */
 
 /* Output element types of wq_down_w4. */
 #define WQ_BF16 0
@@ -259,10 +261,17 @@ wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, c
  * with xin_l = RMSNorm(x_l) (unrounded, as in wq_gateup_w2_lora) when flags has
  * WQ_PRENORM, else x_l.  Each layer's gate/up are 2-bit (with LoRA) or 4-bit
  * (no LoRA); down is 4-bit.  x, y: bf16 [m, d]; the residual stream is stored
- * in bf16 between layers.  The call launches 2 kernels per layer (plus one
- * for the first layer's input statistics) on `stream` with programmatic
- * dependent launch, each down launch also producing the next layer's RMSNorm
- * and LoRA-A partial sums, and can be captured into a CUDA graph.
+ * in bf16 between layers.  Three routes, chosen per call (wq_mlp_forward_info
+ * reports which):
+ *   - the single-launch stack kernel: every layer in one cooperative launch
+ *     (one CTA per SM; up to 32 layers a launch), for 1..8 tokens when every
+ *     layer has the same bits, groups and rank, where it is the measured-faster
+ *     route (2-bit gate/up at 2..8 tokens, or d >= 4096) or WQ_LAUNCH_STACK asks;
+ *   - the launch chain: 2 kernels per layer (plus one for the first layer's
+ *     input statistics) with programmatic dependent launch, each down launch
+ *     also producing the next layer's RMSNorm and LoRA-A partial sums;
+ *   - the dequant-GEMM chain above 16 tokens.
+ * Every route can be captured into a CUDA graph.
  */
 wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
                          unsigned flags, void *y, void *ws, size_t ws_bytes, void *stream);
@@ -285,13 +294,17 @@ wq_status wq_mlp_forward_states(const void *x, int m, const wq_mlp_layer *layers
  * How wq_mlp_forward runs this stack on the current device (for tests and
  * tuning; validates like wq_mlp_forward and launches nothing).  info[16]:
  *   [0]      route: 0 = per-layer dequant-GEMV launch chain,
- *                   1 = per-layer dequant-GEMM launch chain
+ *                   1 = per-layer dequant-GEMM launch chain,
+ *                   2 = single-launch stack kernel
  *   [1..6]   route 0: layer 0's gate/up launch: row tiles per CTA, blocks per
  *            panel, warps along k, row tiles per warp, panels, CTAs
  *   [7..12]  route 0: layer 0's down launch (writing layer 1's partial sums
  *            when there is a layer 1): the same fields
  *   [13]     route 0: 1 when the gate/up launch hands the down launch its
  *            ready binary16 panel of h
+ *   [1..7]   route 2: CTAs, ring stages, stage bytes, 1 when the down slices
+ *            need other CTAs' h (a grid barrier before each down phase), warps
+ *            per gate/up row tile, gate/up row tiles per CTA, shared memory bytes
  *   other entries: -1
  */
 wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags, int64_t info[16]);

@@ -686,7 +686,9 @@ wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned 
   if (st != WQ_OK) return st;
   if (n_layers < 0) return fail(WQ_ERR_ARG, "n_layers=%d is negative", n_layers);
   if (n_layers > 0 && !layers) return fail(WQ_ERR_ARG, "null layer array");
-  if (flags & ~(WQ_PRENORM | WQ_LAUNCH_CHAIN)) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (flags & ~(WQ_PRENORM | WQ_LAUNCH_CHAIN | WQ_LAUNCH_STACK)) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if ((flags & WQ_LAUNCH_CHAIN) && (flags & WQ_LAUNCH_STACK))
+    return fail(WQ_ERR_ARG, "WQ_LAUNCH_CHAIN and WQ_LAUNCH_STACK together");
   int d = 0, inter = 0;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
@@ -744,9 +746,19 @@ bool stack_kernel_plan(int m, const wq_mlp_layer *layers, int n_layers, unsigned
   return stack_plan(m, L0.gate.k, L0.gate.n, L0.r, L0.gate.bits, L0.gate.group, L0.down.group, num_sms(), plan);
 }
 
+// Where the stack kernel is the measured-faster route (GB300, CUDA-graph
+// replays of whole stacks, us per layer, stack kernel vs launch chain):
+//   2-bit gate/up, d 2560 / inter 9728: m=1 18.5 vs 16.7, m=2 20.1 vs 23.1,
+//     m=4 22.9 vs 24.2, m=8 29.2 vs 29.5;
+//   d 4096 / inter 14336: m=1 33.0 vs 41.6, m=4 44.1 vs 61.5, m=8 68.8 vs 87.2;
+//   d 5120 / inter 17408: m=1 48.7 vs 52.6, m=4 80.1 vs 76.8, m=8 104.1 vs 132.9;
+//   4-bit gate/up, d 2560: m=1 20.9 vs 18.0, m=4 23.6 vs 22.5, m=8 28.0 vs 25.9.
+bool stack_preferred(int m, const wq_mlp_layer &L0) { return L0.gate.bits == 2 && (m >= 2 || L0.gate.k >= 4096); }
+
 StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned flags) {
   StackPlan sp;
-  if (stack_kernel_plan(m, layers, n_layers, flags, &sp)) return kRouteStack;
+  if (((flags & WQ_LAUNCH_STACK) || stack_preferred(m, layers[0])) && stack_kernel_plan(m, layers, n_layers, flags, &sp))
+    return kRouteStack;
   if (m > kGemvPreferTokens) return kRouteGemmChain;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
@@ -824,21 +836,19 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
       a.hg = reinterpret_cast<uint16_t *>(w8 + L.shg);
       a.part = reinterpret_cast<float *>(w8 + L.spart);
       a.ctr = reinterpret_cast<unsigned long long *>(w8 + L.sctr);
+      static thread_local StackMaps maps;  // 24 KB: kept off the stack
       for (int l = 0; l < nl; ++l) {
         const wq_mlp_layer &Ly = layers[l0 + l];
         StackLayerDev &D = a.L[l];
-        D.codes[0] = reinterpret_cast<const uint8_t *>(Ly.gate.codes);
-        D.codes[1] = reinterpret_cast<const uint8_t *>(Ly.up.codes);
-        D.codes[2] = reinterpret_cast<const uint8_t *>(Ly.down.codes);
-        D.meta[0] = reinterpret_cast<const uint8_t *>(Ly.gate.meta);
-        D.meta[1] = reinterpret_cast<const uint8_t *>(Ly.up.meta);
-        D.meta[2] = reinterpret_cast<const uint8_t *>(Ly.down.meta);
         D.lora_a = static_cast<const uint16_t *>(Ly.lora_a);
         D.lora_b[0] = static_cast<const uint16_t *>(Ly.lora_b_gate);
         D.lora_b[1] = static_cast<const uint16_t *>(Ly.lora_b_up);
         D.lora_scale = Ly.lora_scale;
+        cudaError_t e = stack_layer_maps(Ly.gate.codes, Ly.up.codes, Ly.gate.meta, Ly.up.meta, Ly.down.codes,
+                                         Ly.down.meta, d, inter, Ly.gate.bits, Ly.gate.group, sp, maps.m[l]);
+        if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the stack's weights");
       }
-      cudaError_t e = launch_stack(a, sp, s);
+      cudaError_t e = launch_stack(a, sp, maps, s);
       if (e != cudaSuccess) return cuda_fail(e, "single-launch stack");
       cur = a.y_out;
     }

@@ -37,6 +37,11 @@
 #include <algorithm>
 #include <climits>
 #include <cstring>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include <cudaTypedefs.h>
 
 #include "wq_internal.h"
 #include "wq_ptx.cuh"
@@ -112,73 +117,112 @@ struct GuConst {
   static constexpr int BPK = BITS == 2 ? 512 : 1024;  // code bytes per (row tile, 128-feature block)
 };
 
+// 3-D TMA load (coordinates innermost first) with an L2 cache policy,
+// completing on `bar` with the box's byte count.
+__device__ __forceinline__ void tma3(void *dst, const CUtensorMap *map, int x, int y, int z, uint64_t *bar,
+                                     uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, %3, "
+      "%4}], [%5], %6;" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
+}
+
+// The down stages of a CTA: its cells [e0, e0 + ne) in half-block-major order,
+// cut at half-block ends and into runs of at most RPS row tiles (one TMA box).
+__device__ __forceinline__ int dn_stage_count(const StackPlan &p, const Share &sh) {
+  int n = 0;
+  for (int jl = 0; jl < sh.nj; ++jl) {
+    const int j = sh.j0 + jl;
+    const int rb = max(sh.e0 - j * p.RTd, 0), re = min(sh.e0 + sh.ne - j * p.RTd, p.RTd);
+    n += (re - rb + p.RPS - 1) / p.RPS;
+  }
+  return n;
+}
+// Walks the down stages in order: (half block j, first row tile, row tiles).
+struct DnWalk {
+  int jl, rt, re;
+  __device__ __forceinline__ void start(const StackPlan &p, const Share &sh) {
+    jl = 0;
+    const int j = sh.j0;
+    rt = max(sh.e0 - j * p.RTd, 0);
+    re = min(sh.e0 + sh.ne - j * p.RTd, p.RTd);
+  }
+  // the current stage; then advance
+  __device__ __forceinline__ void next(const StackPlan &p, const Share &sh, int *j, int *rt0, int *nrt) {
+    *j = sh.j0 + jl;
+    *rt0 = rt;
+    *nrt = min(p.RPS, re - rt);
+    rt += p.RPS;
+    if (rt >= re) {
+      ++jl;
+      const int jn = sh.j0 + jl;
+      rt = max(sh.e0 - jn * p.RTd, 0);
+      re = min(sh.e0 + sh.ne - jn * p.RTd, p.RTd);
+    }
+  }
+};
+
 // Weight-stream warp: walks the stage sequence of every layer and fills the
-// ring.  Lane 0 arms each stage's barrier; all lanes issue its copies.
+// ring by TMA (lane 0 arms each stage's barrier and issues its boxes).
+//   gate/up stage: k-blocks [kb0, kb0 + kps) of the CTA's T row tiles, both
+//     projections: codes [pj][t][kps][BPK], then meta [pj][t][gmy][64] (blocks
+//     past the matrix zero-filled);
+//   down stage: half block j, row tiles [rt0, rt0 + RPS): codes [RPS][512],
+//     then meta [RPS][GPH * 64] (rows past the matrix zero-filled).
 template <int BITS_GU, int GG, int GD>
-__device__ void stream_weights(const StackArgs &a, const StackPlan &p, const Share &sh, uint8_t *smem,
-                               volatile int *abort_flag, volatile int *issued) {
+__device__ void stream_weights(const StackArgs &a, const StackPlan &p, const StackMaps &maps, const Share &sh,
+                               uint8_t *smem, volatile int *abort_flag, volatile int *issued) {
   constexpr int BPK = GuConst<BITS_GU>::BPK;
   constexpr int GPBg = 128 / GG;
+  constexpr int GPH = GD == 32 ? 2 : 1;  // down groups a half block touches
   const int lane = threadIdx.x & 31;
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + p.off_full);
   uint64_t *empty = reinterpret_cast<uint64_t *>(smem + p.off_empty);
   uint8_t *ring = smem + p.off_ring;
   const uint64_t pol = l2_evict_first_policy();
-  const int NGg = p.KBg * GPBg;
-  const int KBd = (a.inter + 127) / 128, NGd = KBd * 128 / GD;
-  const int GPH = GD == 32 ? 2 : 1;  // down groups a half block touches
   const int nsg = (p.KBg + p.kps - 1) / p.kps;
-  const int nsd = (sh.ne + p.cps - 1) / p.cps;
+  const int nsd = dn_stage_count(p, sh);
+  const uint32_t cbytes = (uint32_t)(2 * sh.T * p.kps * BPK);
+  const uint32_t gu_bytes = cbytes + (uint32_t)(2 * sh.T * p.gmy * 64);
+  const uint32_t dn_bytes = (uint32_t)(p.RPS * (512 + GPH * 64));
+  if (lane != 0) return;
   int q = 0;
   for (int l = 0; l < a.n_layers; ++l) {
-    const StackLayerDev &Ly = a.L[l];
+    const CUtensorMap *mp = maps.m[l];
+    DnWalk w;
+    w.start(p, sh);
     for (int s = 0; s < nsg + nsd; ++s, ++q) {
       const int slot = q % p.NS;
-      bool ok = true;
-      if (q >= p.NS && lane == 0) ok = mbar_wait(&empty[slot], ((q / p.NS) - 1) & 1);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-      if (!ok) {
-        if (lane == 0) {
-          record_timeout();
-          *abort_flag = 1;
-        }
+      if (q >= p.NS && !mbar_wait(&empty[slot], ((q / p.NS) - 1) & 1)) {
+        record_timeout();
+        *abort_flag = 1;
       }
       if (*abort_flag) {
-        if (lane == 0) *issued = q;
+        *issued = q;
         return;
       }
       uint8_t *st = ring + (size_t)slot * p.SB;
       if (s < nsg) {
-        // gate/up stage: k-blocks [kb0, kb1) of the CTA's T tiles, both
-        // projections; layout codes [pj][t][kbl][BPK], then meta [pj][t][kbl*GPB + g][64]
-        const int kb0 = s * p.kps, nk = min(p.kps, p.KBg - kb0);
-        const uint32_t cbytes = (uint32_t)(2 * sh.T * nk * BPK);
-        if (lane == 0) mbar_arrive_expect_tx(&full[slot], cbytes + (uint32_t)(2 * sh.T * nk * GPBg * 64));
-        __syncwarp();
-        for (int i = lane; i < 2 * sh.T; i += 32) {
-          const int pj = i / sh.T, t = i % sh.T, rt = sh.g0 + t;
-          bulk_g2s_hint(st + (size_t)i * nk * BPK, Ly.codes[pj] + ((size_t)rt * p.KBg + kb0) * BPK, nk * BPK, &full[slot],
-                        pol);
-          bulk_g2s_hint(st + cbytes + (size_t)i * nk * GPBg * 64, Ly.meta[pj] + ((size_t)rt * NGg + kb0 * GPBg) * 64,
-                        nk * GPBg * 64, &full[slot], pol);
-        }
+        const int kb0 = s * p.kps;
+        mbar_arrive_expect_tx(&full[slot], gu_bytes);
+        for (int pj = 0; pj < 2; ++pj)
+          for (int t0 = 0; t0 < sh.T; t0 += p.Tbox) {
+            tma3(st + (size_t)(pj * sh.T + t0) * p.kps * BPK, &mp[pj], 0, kb0 * (BPK / 128), sh.g0 + t0, &full[slot], pol);
+            tma3(st + cbytes + (size_t)(pj * sh.T + t0) * p.gmy * 64, &mp[2 + pj], 0, kb0 * GPBg, sh.g0 + t0,
+                 &full[slot], pol);
+          }
       } else {
-        // down stage: cells [c0, c0 + nc) of the CTA; layout codes [cell][512], then meta [cell][GPH*64]
-        const int c0 = (s - nsg) * p.cps, nc = min(p.cps, sh.ne - c0);
-        if (lane == 0) mbar_arrive_expect_tx(&full[slot], (uint32_t)(nc * (512 + GPH * 64)));
-        __syncwarp();
-        for (int i = lane; i < nc; i += 32) {
-          const int e = sh.e0 + c0 + i, j = e / p.RTd, rt = e % p.RTd;
-          bulk_g2s_hint(st + (size_t)i * 512, Ly.codes[2] + ((size_t)rt * KBd + (j >> 1)) * 1024 + (j & 1) * 512, 512,
-                        &full[slot], pol);
-          const int g = GD == 32 ? 2 * j : GD == 64 ? j : (j >> 1);
-          bulk_g2s_hint(st + (size_t)nc * 512 + (size_t)i * GPH * 64, Ly.meta[2] + ((size_t)rt * NGd + g) * 64,
-                        GPH * 64, &full[slot], pol);
-        }
+        int j, rt0, nrt;
+        w.next(p, sh, &j, &rt0, &nrt);
+        const int g = GD == 32 ? 2 * j : GD == 64 ? j : (j >> 1);
+        mbar_arrive_expect_tx(&full[slot], dn_bytes);
+        tma3(st, &mp[4], 0, 4 * j, rt0, &full[slot], pol);
+        tma3(st + p.RPS * 512, &mp[5], 0, g, rt0, &full[slot], pol);
       }
     }
   }
-  if (lane == 0) *issued = q;
+  *issued = q;
 }
 
 // Grid barrier: arrive (after the CTA's writes) / wait for generation `gen`.
@@ -204,16 +248,108 @@ __device__ __forceinline__ void grid_wait(const unsigned long long *ctr, unsigne
   math_sync();
 }
 
+// The dot products of NB k-blocks of one row tile, both projections, their
+// MMA chains interleaved (2 NB independent accumulators): per k-step the
+// exact products code x binary16 activation on mma.sync, per group
+//   ctot += s * (sx * sum q x' - z * sum x)
+// (the affine dequantization s (q - z), x' = x / sx with the block's scale
+// sx).  Codes [pj][T][kps][BPK], meta [pj][T][gmy][64] in the stage.
+template <int BITS_GU, int GG, int NB>
+__device__ __forceinline__ void gu_blocks(float (&ctot)[2][4], const int (&kb)[NB], const int (&kbl)[NB],
+                                          const uint8_t *stg, uint32_t cbytes, int T, int tl, int kps, int gmy,
+                                          const __half *xp, int xstride, const float *xsc, const float *xs, int M,
+                                          int lane) {
+  constexpr int BPK = BITS_GU == 2 ? 512 : 1024;
+  constexpr int GPBg = 128 / GG, GSg = GG / 16;
+  constexpr int NW = BITS_GU == 2 ? 4 : 8;
+  const int col = 2 * (lane & 3);
+  uint32_t b[NB][8][2];
+#pragma unroll
+  for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      uint2 v = make_uint2(0u, 0u);  // tokens past M: zero columns
+      if ((lane >> 2) < M) v = lds64(xp + (size_t)(lane >> 2) * xstride + (kb[nb] * 8 + ks) * 16 + 4 * (lane & 3));
+      b[nb][ks][0] = v.x;
+      b[nb][ks][1] = v.y;
+    }
+  uint32_t wds[NB][2][NW];
+#pragma unroll
+  for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+    for (int pj = 0; pj < 2; ++pj) {
+      const uint8_t *cb = stg + ((size_t)(pj * T + tl) * kps + kbl[nb]) * BPK + lane * 16;
+      const uint4 w0 = lds128(cb);
+      wds[nb][pj][0] = w0.x; wds[nb][pj][1] = w0.y; wds[nb][pj][2] = w0.z; wds[nb][pj][3] = w0.w;
+      if (BITS_GU == 4) {
+        const uint4 w1 = lds128(cb + 512);
+        wds[nb][pj][NW - 4] = w1.x; wds[nb][pj][NW - 3] = w1.y; wds[nb][pj][NW - 2] = w1.z; wds[nb][pj][NW - 1] = w1.w;
+      }
+    }
+  float acc[NB][2][4];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+      for (int pj = 0; pj < 2; ++pj) {
+        uint32_t af[4];
+        if (BITS_GU == 2) {
+          const uint32_t x = wds[nb][pj][(ks >> 1) & 3], x8 = x >> 8;
+          const int s4 = (ks & 1) * 4;
+          af[0] = x & (0x00030003u << s4);
+          af[1] = x8 & (0x00030003u << s4);
+          af[2] = x & (0x000C000Cu << s4);
+          af[3] = x8 & (0x000C000Cu << s4);
+        } else {
+          const uint32_t x = wds[nb][pj][ks], x8 = x >> 8;
+          af[0] = x & 0x000F000Fu;
+          af[1] = x8 & 0x000F000Fu;
+          af[2] = x & 0x00F000F0u;
+          af[3] = x8 & 0x00F000F0u;
+        }
+        if (ks % GSg == 0)
+          mma_f16_16816_zc(acc[nb][pj], af, b[nb][ks][0], b[nb][ks][1]);
+        else
+          mma_f16_16816(acc[nb][pj], af, b[nb][ks][0], b[nb][ks][1]);
+      }
+    if ((ks + 1) % GSg == 0) {
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb) {
+        const int gl = kb[nb] * GPBg + ks / GSg;
+        const float2 gsum = *reinterpret_cast<const float2 *>(xs + gl * 8 + col);
+        const float2 sc = *reinterpret_cast<const float2 *>(xsc + kb[nb] * 8 + col);
+#pragma unroll
+        for (int pj = 0; pj < 2; ++pj) {
+          const uint2 sz = lds64(stg + cbytes + ((size_t)(pj * T + tl) * gmy + kbl[nb] * GPBg + ks / GSg) * 64 +
+                                 (lane >> 2) * 8);
+          const float s_lo = half_bits(sz.x), s_hi = half_bits(sz.x >> 16);
+          const float zs_lo = -s_lo * half_bits(sz.y), zs_hi = -s_hi * half_bits(sz.y >> 16);
+          float *ct = ctot[pj];
+          ct[0] = fmaf(s_lo * sc.x, acc[nb][pj][0], ct[0]);
+          ct[1] = fmaf(s_lo * sc.y, acc[nb][pj][1], ct[1]);
+          ct[2] = fmaf(s_hi * sc.x, acc[nb][pj][2], ct[2]);
+          ct[3] = fmaf(s_hi * sc.y, acc[nb][pj][3], ct[3]);
+          ct[0] = fmaf(zs_lo, gsum.x, ct[0]);
+          ct[1] = fmaf(zs_lo, gsum.y, ct[1]);
+          ct[2] = fmaf(zs_hi, gsum.x, ct[2]);
+          ct[3] = fmaf(zs_hi, gsum.y, ct[3]);
+        }
+      }
+    }
+  }
+}
+
 using bf16 = __nv_bfloat16;
 __device__ __forceinline__ const bf16 *B16(const uint16_t *p) { return reinterpret_cast<const bf16 *>(p); }
 __device__ __forceinline__ bf16 *B16(uint16_t *p) { return reinterpret_cast<bf16 *>(p); }
 
 template <int BITS_GU, int GG, int GD>
-__global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_constant__ StackArgs a, const StackPlan p) {
+__global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_constant__ StackArgs a, const StackPlan p,
+                                                              const __grid_constant__ StackMaps maps) {
   extern __shared__ __align__(1024) uint8_t smem[];
   constexpr int BPK = GuConst<BITS_GU>::BPK;
   constexpr int GPBg = 128 / GG;      // gate/up groups per block
-  constexpr int GSg = GG / 16;        // gate/up k-steps per group
   constexpr int LPG = GG / 4;         // conversion lanes per gate/up group (4 features a lane)
   constexpr int GPH = GD == 32 ? 2 : 1;
 
@@ -235,7 +371,8 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
   __nv_bfloat16 *lb = reinterpret_cast<__nv_bfloat16 *>(smem + p.off_lb);  // [2][Tmax*16][r]
   __nv_bfloat16 *la = reinterpret_cast<__nv_bfloat16 *>(smem + p.off_la);  // [own_max*16][2r]
   float *rt = reinterpret_cast<float *>(smem + p.off_rt);          // [M][Qp] tile partials summed
-  float *red = reinterpret_cast<float *>(smem + p.off_red);        // scratch of the reductions
+  float *yo = reinterpret_cast<float *>(smem + p.off_yo);          // [own][M][16] the owned tiles of y
+  float *red = reinterpret_cast<float *>(smem + p.off_red);        // [512 x 4] scratch of the reductions
   uint8_t *ring = smem + p.off_ring;
 
   if (tid == 0) {
@@ -253,7 +390,7 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
   }
   __syncthreads();
   if (warp == kSW) {
-    stream_weights<BITS_GU, GG, GD>(a, p, sh, smem, &misc[0], &misc[1]);
+    stream_weights<BITS_GU, GG, GD>(a, p, maps, sh, smem, &misc[0], &misc[1]);
     return;
   }
   const unsigned long long base = base_s[0];
@@ -261,7 +398,7 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
   const int KBd = (a.inter + 127) / 128;
   (void)KBd;
   const int nsg = (p.KBg + p.kps - 1) / p.kps;
-  const int nsd = (sh.ne + p.cps - 1) / p.cps;
+  const int nsd = dn_stage_count(p, sh);
   int q = 0;  // stage sequence position
 
   // ---- the first layer's tile partials of x_in (owned tiles), barrier ----
@@ -293,7 +430,20 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
       a.tp[((size_t)t * M + m) * Qp + qq] = s;
     }
   };
+  // the LoRA-B rows of layer l's gate/up tiles, by cp.async (waited for with
+  // the activation panel): issued before the barrier that opens the layer
+  auto prefetch_lb = [&](int l) {
+    if (r <= 0) return;
+    const int per_row = r / 8, rows = sh.T * 16;
+    for (int i = tid; i < 2 * rows * per_row; i += kSMathThreads) {
+      const int pj = i / (rows * per_row), rem = i % (rows * per_row), rl = rem / per_row, c = rem % per_row;
+      cp_async16(lb + ((size_t)pj * p.Tmax * 16 + rl) * r + c * 8,
+                 B16(a.L[l].lora_b[pj]) + (size_t)(sh.g0 * 16 + rl) * r + c * 8);
+    }
+    cp_async_commit();
+  };
   owner_stats(B16(a.x_in), B16(a.L[0].lora_a));
+  prefetch_lb(0);
   math_sync();
   grid_arrive(a.ctr);
   ++gen;
@@ -305,53 +455,59 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
     grid_wait(a.ctr, base + (unsigned long long)p.G * gen, &misc[0]);
 
     // ================= gate/up =================
-    // (a) inputs: the activation panel (raw bf16, converted in place below),
-    // the LoRA-B rows of the CTA's tiles, and the tile partials (summed in chunks)
+    // (a) inputs: the activation panel (raw bf16, converted in place below)
+    // and the tile partials
     {
       const int cpr = p.KBg * 16;  // 16-byte chunks per token row
       for (int i = tid; i < M * cpr; i += kSMathThreads) {
         const int m = i / cpr, c = i % cpr;
         cp_async16(xp + (size_t)m * p.xstride + c * 8, cur + (size_t)m * a.d + c * 8);
       }
-      if (r > 0) {
-        const int per_row = r / 8, rows = sh.T * 16;
-        for (int i = tid; i < 2 * rows * per_row; i += kSMathThreads) {
-          const int pj = i / (rows * per_row), rem = i % (rows * per_row), rl = rem / per_row, c = rem % per_row;
-          cp_async16(lb + ((size_t)pj * p.Tmax * 16 + rl) * r + c * 8,
-                     B16(Ly.lora_b[pj]) + (size_t)(sh.g0 * 16 + rl) * r + c * 8);
-        }
-      }
       cp_async_commit();
-      // tile partials: item = (chunk, m, 4 values); chunks of tiles summed in order
-      const int Q4 = Qp / 4, nchk = p.nchk, tpc = (p.RTd + nchk - 1) / nchk;
-      for (int item = tid; item < nchk * M * Q4; item += kSMathThreads) {
-        const int c = item / (M * Q4), rem = item % (M * Q4), m = rem / Q4, j = rem % Q4;
-        const int t0 = c * tpc, t1 = min(t0 + tpc, p.RTd);
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int tb = t0; tb < t1; tb += 8) {
-          float4 v[8];
+      // tile partials summed over the RTd tiles: thread (item, split) adds
+      // the tiles t = split, split + S, ... (eight loads in flight; adjacent
+      // threads read adjacent 16 bytes), then a fixed tree over the S splits
+      {
+        const int Q4 = Qp / 4, items = M * Q4;
+        int S = 1;
+        while (S * 2 * items <= kSMathThreads && S * 2 <= p.RTd) S *= 2;
+        float4 *tr = reinterpret_cast<float4 *>(red);  // [S][items]
+        if (tid < S * items) {
+          const int item = tid % items, sp = tid / items, m = item / Q4, j = item % Q4;
+          float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int tb = sp; tb < p.RTd; tb += 8 * S) {
+            float4 v[8];
 #pragma unroll
-          for (int u = 0; u < 8; ++u)
-            v[u] = tb + u < t1 ? __ldcg(reinterpret_cast<const float4 *>(a.tp + ((size_t)(tb + u) * M + m) * Qp) + j)
-                               : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int u = 0; u < 8; ++u)
+              v[u] = tb + u * S < p.RTd
+                         ? __ldcg(reinterpret_cast<const float4 *>(a.tp + ((size_t)(tb + u * S) * M + m) * Qp) + j)
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            acc.x += v[u].x;
-            acc.y += v[u].y;
-            acc.z += v[u].z;
-            acc.w += v[u].w;
+            for (int u = 0; u < 8; ++u) {
+              acc.x += v[u].x;
+              acc.y += v[u].y;
+              acc.z += v[u].z;
+              acc.w += v[u].w;
+            }
+          }
+          tr[tid] = acc;
+        }
+        for (int h = S >> 1; h >= 1; h >>= 1) {
+          math_sync();
+          if (tid < h * items) {
+            const float4 b2 = tr[tid + h * items];
+            float4 v = tr[tid];
+            v.x += b2.x;
+            v.y += b2.y;
+            v.z += b2.z;
+            v.w += b2.w;
+            tr[tid] = v;
           }
         }
-        reinterpret_cast<float4 *>(red)[item] = acc;
+        math_sync();
+        if (tid < items) reinterpret_cast<float4 *>(rt)[tid] = tr[tid];
       }
       cp_async_wait_all();
-      math_sync();
-      for (int i = tid; i < M * Qp; i += kSMathThreads) {
-        const int m = i / Qp, qq = i % Qp;
-        float s = 0.f;
-        for (int c = 0; c < nchk; ++c) s += red[((size_t)c * M + m) * Qp + qq];
-        rt[i] = s;
-      }
       math_sync();
       if (a.prenorm)
         for (int m = tid; m < M; m += kSMathThreads)
@@ -364,14 +520,14 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
       const int st = lane >> 2, hi = (lane >> 1) & 1;
       const int shc = BITS_GU == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
       const int u0 = 4 * (lane & 1) + hi;
-      for (int it = warp; it < p.KBg * 8; it += kSW) {
-        const int kb = it >> 3, m = it & 7;
-        if (m >= M) {
-          // padding tokens: zero scales and sums
-          if (lane == 0) xsc[kb * 8 + m] = 0.f;
-          if (lane < GPBg) xs[(kb * GPBg + lane) * 8 + m] = 0.f;
-          continue;
-        }
+      for (int i = tid; i < p.KBg * (8 - M); i += kSMathThreads) {
+        // padding tokens: zero scales and group sums
+        const int kb = i / (8 - M), m = M + i % (8 - M);
+        xsc[kb * 8 + m] = 0.f;
+        for (int g = 0; g < GPBg; ++g) xs[(kb * GPBg + g) * 8 + m] = 0.f;
+      }
+      for (int it = warp; it < p.KBg * M; it += kSW) {
+        const int kb = it / M, m = it % M;
         const uint2 raw = lds64(xp + (size_t)m * p.xstride + kb * 128 + 4 * lane);
         const float f0 = bf16_lo(raw.x), f1 = bf16_hi(raw.x), f2 = bf16_lo(raw.y), f3 = bf16_hi(raw.y);
         const uint32_t v = __float_as_uint(fmaxf(fmaxf(fabsf(f0), fabsf(f1)), fmaxf(fabsf(f2), fabsf(f3))));
@@ -390,7 +546,7 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
     }
     math_sync();
     // (c) the dot products: warp (tile tl, k-slice ksl) takes the stage's
-    // k-blocks kb with kb % WPT == ksl
+    // k-blocks ksl and ksl + WPT
     {
       const int tl = warp / p.WPT, ksl = warp % p.WPT;
       const bool active = tl < sh.T;
@@ -409,78 +565,15 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
         }
         const int kb0 = s * p.kps, nk = min(p.kps, p.KBg - kb0);
         const uint8_t *stg = ring + (size_t)sl * p.SB;
-        const uint32_t cbytes = (uint32_t)(2 * sh.T * nk * BPK);
-        if (active && ok && !misc[0]) {
-          for (int kbl = (ksl - kb0 % p.WPT + p.WPT) % p.WPT; kbl < nk; kbl += p.WPT) {
-            const int kb = kb0 + kbl;
-            uint32_t b[8][2];
-#pragma unroll
-            for (int ks = 0; ks < 8; ++ks) {
-              uint2 v = make_uint2(0u, 0u);  // tokens past M: zero columns
-              if ((lane >> 2) < M) v = lds64(xp + (size_t)(lane >> 2) * p.xstride + (kb * 8 + ks) * 16 + 4 * (lane & 3));
-              b[ks][0] = v.x;
-              b[ks][1] = v.y;
-            }
-            const float2 sc = *reinterpret_cast<const float2 *>(xsc + kb * 8 + col);
-            constexpr int NW = BITS_GU == 2 ? 4 : 8;
-            uint32_t wds[2][NW];
-#pragma unroll
-            for (int pj = 0; pj < 2; ++pj) {
-              const uint8_t *cb = stg + ((size_t)(pj * sh.T + tl) * nk + kbl) * BPK + lane * 16;
-              const uint4 w0 = lds128(cb);
-              wds[pj][0] = w0.x; wds[pj][1] = w0.y; wds[pj][2] = w0.z; wds[pj][3] = w0.w;
-              if (BITS_GU == 4) {
-                const uint4 w1 = lds128(cb + 512);
-                wds[pj][NW - 4] = w1.x; wds[pj][NW - 3] = w1.y; wds[pj][NW - 2] = w1.z; wds[pj][NW - 1] = w1.w;
-              }
-            }
-            float acc[2][4];
-#pragma unroll
-            for (int ks = 0; ks < 8; ++ks) {
-#pragma unroll
-              for (int pj = 0; pj < 2; ++pj) {
-                uint32_t af[4];
-                if (BITS_GU == 2) {
-                  const uint32_t x = wds[pj][(ks >> 1) & 3], x8 = x >> 8;
-                  const int s4 = (ks & 1) * 4;
-                  af[0] = x & (0x00030003u << s4);
-                  af[1] = x8 & (0x00030003u << s4);
-                  af[2] = x & (0x000C000Cu << s4);
-                  af[3] = x8 & (0x000C000Cu << s4);
-                } else {
-                  const uint32_t x = wds[pj][ks], x8 = x >> 8;
-                  af[0] = x & 0x000F000Fu;
-                  af[1] = x8 & 0x000F000Fu;
-                  af[2] = x & 0x00F000F0u;
-                  af[3] = x8 & 0x00F000F0u;
-                }
-                if (ks % GSg == 0)
-                  mma_f16_16816_zc(acc[pj], af, b[ks][0], b[ks][1]);
-                else
-                  mma_f16_16816(acc[pj], af, b[ks][0], b[ks][1]);
-              }
-              if ((ks + 1) % GSg == 0) {
-                // group epilogue: ctot += s * (sx * sum q x' - z * sum x)
-                const int gl = kb * GPBg + ks / GSg;
-                const float2 gsum = *reinterpret_cast<const float2 *>(xs + gl * 8 + col);
-#pragma unroll
-                for (int pj = 0; pj < 2; ++pj) {
-                  const uint2 sz = lds64(stg + cbytes + ((size_t)(pj * sh.T + tl) * nk * GPBg + kbl * GPBg + ks / GSg) * 64 +
-                                         (lane >> 2) * 8);
-                  const float s_lo = half_bits(sz.x), s_hi = half_bits(sz.x >> 16);
-                  const float zs_lo = -s_lo * half_bits(sz.y), zs_hi = -s_hi * half_bits(sz.y >> 16);
-                  float *ct = ctot[pj];
-                  ct[0] = fmaf(s_lo * sc.x, acc[pj][0], ct[0]);
-                  ct[1] = fmaf(s_lo * sc.y, acc[pj][1], ct[1]);
-                  ct[2] = fmaf(s_hi * sc.x, acc[pj][2], ct[2]);
-                  ct[3] = fmaf(s_hi * sc.y, acc[pj][3], ct[3]);
-                  ct[0] = fmaf(zs_lo, gsum.x, ct[0]);
-                  ct[1] = fmaf(zs_lo, gsum.y, ct[1]);
-                  ct[2] = fmaf(zs_hi, gsum.x, ct[2]);
-                  ct[3] = fmaf(zs_hi, gsum.y, ct[3]);
-                }
-              }
-            }
+        const uint32_t cbytes = (uint32_t)(2 * sh.T * p.kps * BPK);
+        // the warp's blocks in this stage: ksl and ksl + WPT, two in flight
+        if (active && ok && !misc[0] && ksl < nk) {
+          if (ksl + p.WPT < nk) {
+            const int kb[2] = {kb0 + ksl, kb0 + ksl + p.WPT}, kbl[2] = {ksl, ksl + p.WPT};
+            gu_blocks<BITS_GU, GG, 2>(ctot, kb, kbl, stg, cbytes, sh.T, tl, p.kps, p.gmy, xp, p.xstride, xsc, xs, M, lane);
+          } else {
+            const int kb[1] = {kb0 + ksl}, kbl[1] = {ksl};
+            gu_blocks<BITS_GU, GG, 1>(ctot, kb, kbl, stg, cbytes, sh.T, tl, p.kps, p.gmy, xp, p.xstride, xsc, xs, M, lane);
           }
         }
         __syncwarp();
@@ -595,6 +688,8 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
     // (c) the cells: warp w takes cells w, w + 16, ... of each stage; a cell
     // (half block j, row tile t) is 4 MMAs and yields y's partial sums of the
     // tile's 16 rows over the half block's 64 features
+    DnWalk dw;
+    dw.start(p, sh);
     for (int s = 0; s < nsd; ++s, ++q) {
       const int sl = q % p.NS;
       const bool ok = !misc[0] && mbar_wait(&full[sl], (q / p.NS) & 1);
@@ -602,48 +697,66 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
         record_timeout();
         misc[0] = 1;
       }
-      const int c0 = s * p.cps, nc = min(p.cps, sh.ne - c0);
+      int j, rt0, nc;
+      dw.next(p, sh, &j, &rt0, &nc);
       const uint8_t *stg = ring + (size_t)sl * p.SB;
-      if (ok && !misc[0]) {
-        for (int cl = warp; cl < nc; cl += kSW) {
-          const int e = sh.e0 + c0 + cl, j = e / p.RTd, t = e % p.RTd, jl = j - sh.j0;
-          const uint4 wv = lds128(stg + (size_t)cl * 512 + lane * 16);
-          const uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
-          float acc[2][4];
+      if (ok && !misc[0] && warp < nc) {
+        // cells warp, warp + 16, warp + 32, warp + 48 of the stage (same half
+        // block): their MMA chains interleaved on the shared B fragments
+        constexpr int CW = 4;
+        const int jl = j - sh.j0;
+        uint32_t wd[CW][4];
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks) {
-            const uint2 bv = hp[((size_t)(jl * 4 + ks) * 8 + (lane >> 2)) * 4 + (lane & 3)];
-            const uint32_t x = wd[ks], x8 = x >> 8;
+        for (int c2 = 0; c2 < CW; ++c2) {
+          const int cl = warp + c2 * kSW;
+          const uint4 wv = cl < nc ? lds128(stg + (size_t)cl * 512 + lane * 16) : make_uint4(0u, 0u, 0u, 0u);
+          wd[c2][0] = wv.x; wd[c2][1] = wv.y; wd[c2][2] = wv.z; wd[c2][3] = wv.w;
+        }
+        float acc[CW][2][4];
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+          const uint2 bv = hp[((size_t)(jl * 4 + ks) * 8 + (lane >> 2)) * 4 + (lane & 3)];
+          const int ch = GD == 32 ? (ks >> 1) : 0;
+#pragma unroll
+          for (int c2 = 0; c2 < CW; ++c2) {
+            const uint32_t x = wd[c2][ks], x8 = x >> 8;
             const uint32_t af[4] = {x & 0x000F000Fu, x8 & 0x000F000Fu, x & 0x00F000F0u, x8 & 0x00F000F0u};
-            const int ch = GD == 32 ? (ks >> 1) : 0;
             if (GD == 32 ? (ks & 1) == 0 : ks == 0)
-              mma_f16_16816_zc(acc[ch], af, bv.x, bv.y);
+              mma_f16_16816_zc(acc[c2][ch], af, bv.x, bv.y);
             else
-              mma_f16_16816(acc[ch], af, bv.x, bv.y);
+              mma_f16_16816(acc[c2][ch], af, bv.x, bv.y);
           }
-          const int col = 2 * (lane & 3);
-          const float2 sc = *reinterpret_cast<const float2 *>(hsc + jl * 8 + col);
+        }
+        const int col = 2 * (lane & 3);
+        const float2 sc = *reinterpret_cast<const float2 *>(hsc + jl * 8 + col);
+        float2 gs[GPH];
+#pragma unroll
+        for (int ch = 0; ch < GPH; ++ch) {
+          if (GD == 32) {
+            gs[ch] = make_float2(hxs[(jl * 2 + ch) * 8 + col], hxs[(jl * 2 + ch) * 8 + col + 1]);
+          } else {
+            gs[ch] = make_float2(hxs[(jl * 2) * 8 + col] + hxs[(jl * 2 + 1) * 8 + col],
+                                 hxs[(jl * 2) * 8 + col + 1] + hxs[(jl * 2 + 1) * 8 + col + 1]);
+          }
+        }
+#pragma unroll
+        for (int c2 = 0; c2 < CW; ++c2) {
+          const int cl = warp + c2 * kSW, t = rt0 + cl;
+          if (cl >= nc) break;
           float y[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int ch = 0; ch < GPH; ++ch) {
-            const uint2 sz = lds64(stg + (size_t)nc * 512 + ((size_t)cl * GPH + ch) * 64 + (lane >> 2) * 8);
+            const uint2 sz = lds64(stg + (size_t)p.RPS * 512 + ((size_t)cl * GPH + ch) * 64 + (lane >> 2) * 8);
             const float s_lo = half_bits(sz.x), s_hi = half_bits(sz.x >> 16);
             const float zs_lo = -s_lo * half_bits(sz.y), zs_hi = -s_hi * half_bits(sz.y >> 16);
-            float2 gsum;
-            if (GD == 32) {
-              gsum = make_float2(hxs[(jl * 2 + ch) * 8 + col], hxs[(jl * 2 + ch) * 8 + col + 1]);
-            } else {
-              gsum = make_float2(hxs[(jl * 2) * 8 + col] + hxs[(jl * 2 + 1) * 8 + col],
-                                 hxs[(jl * 2) * 8 + col + 1] + hxs[(jl * 2 + 1) * 8 + col + 1]);
-            }
-            y[0] = fmaf(s_lo * sc.x, acc[ch][0], y[0]);
-            y[1] = fmaf(s_lo * sc.y, acc[ch][1], y[1]);
-            y[2] = fmaf(s_hi * sc.x, acc[ch][2], y[2]);
-            y[3] = fmaf(s_hi * sc.y, acc[ch][3], y[3]);
-            y[0] = fmaf(zs_lo, gsum.x, y[0]);
-            y[1] = fmaf(zs_lo, gsum.y, y[1]);
-            y[2] = fmaf(zs_hi, gsum.x, y[2]);
-            y[3] = fmaf(zs_hi, gsum.y, y[3]);
+            y[0] = fmaf(s_lo * sc.x, acc[c2][ch][0], y[0]);
+            y[1] = fmaf(s_lo * sc.y, acc[c2][ch][1], y[1]);
+            y[2] = fmaf(s_hi * sc.x, acc[c2][ch][2], y[2]);
+            y[3] = fmaf(s_hi * sc.y, acc[c2][ch][3], y[3]);
+            y[0] = fmaf(zs_lo, gs[ch].x, y[0]);
+            y[1] = fmaf(zs_lo, gs[ch].y, y[1]);
+            y[2] = fmaf(zs_hi, gs[ch].x, y[2]);
+            y[3] = fmaf(zs_hi, gs[ch].y, y[3]);
           }
           const int r0 = t * 16 + (lane >> 2);
 #pragma unroll
@@ -664,46 +777,56 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
     grid_wait(a.ctr, base + (unsigned long long)p.G * gen, &misc[0]);
 
     // ================= owner: y tiles =================
-    // output (tile, m, row): sum over half blocks j of part[j][m][row], in
-    // chunks of half blocks (fixed split), then the chunks in order
+    // output (tile, m, row): sum over half blocks j of part[j][m][row]:
+    // thread (output, split) adds j = split, split + S, ... (eight loads in
+    // flight; adjacent threads read adjacent rows), then a fixed tree over
+    // the S splits; plus the residual, kept in shared memory from the
+    // previous layer
     {
       const int nout = sh.no * 16 * M;
-      const int splits = nout > 0 ? max(1, min(kSMathThreads / nout, p.U)) : 1;
-      const int jpc = (p.U + splits - 1) / splits;
-      for (int i = tid; i < nout * splits; i += kSMathThreads) {
-        const int o = i % nout, sp = i / nout;
-        const int tl = o / (16 * M), rem = o % (16 * M), m = rem / 16, row = rem % 16;
-        const int n = (sh.o0 + tl) * 16 + row;
-        const int j0 = sp * jpc, j1 = min(j0 + jpc, p.U);
-        float s = 0.f;
-        for (int jb = j0; jb < j1; jb += 8) {
-          float v[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) v[u] = jb + u < j1 ? __ldcg(a.part + ((size_t)(jb + u) * M + m) * a.d + n) : 0.f;
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            if (jb + u < j1) s += v[u];
-        }
-        red[(size_t)sp * nout + o] = s;
-      }
-      math_sync();
+      int S = 1;
+      while (S * 2 * nout <= kSMathThreads && S * 2 <= p.U) S *= 2;
       bf16 *dst = last ? B16(a.y_out) : B16(a.xw);
-      for (int o = tid; o < nout; o += kSMathThreads) {
-        const int tl = o / (16 * M), rem = o % (16 * M), m = rem / 16, row = rem % 16;
-        const int n = (sh.o0 + tl) * 16 + row;
-        float s = 0.f;
-        for (int sp = 0; sp < splits; ++sp) s += red[(size_t)sp * nout + o];
-        const float yv = s + __bfloat162float(cur[(size_t)m * a.d + n]);
-        const __nv_bfloat16 yb = __float2bfloat16_rn(yv);
-        dst[(size_t)m * a.d + n] = yb;
-        if (a.states) B16(a.states)[((size_t)l * M + m) * a.d + n] = yb;
-        red[(size_t)splits * nout + o] = __bfloat162float(yb);  // for the tile partials below
+      for (int base = 0; base < nout; base += kSMathThreads) {  // one round unless nout > 512
+        const int nb = min(nout - base, kSMathThreads);
+        const int SS = base == 0 ? S : 1;
+        if (tid < SS * nb) {
+          const int o = base + tid % nb, sp = tid / nb;
+          const int tl = o / (16 * M), rem = o % (16 * M), m = rem / 16, row = rem % 16;
+          const int n = (sh.o0 + tl) * 16 + row;
+          float sum = 0.f;
+          for (int jb = sp; jb < p.U; jb += 8 * SS) {
+            float v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              v[u] = jb + u * SS < p.U ? __ldcg(a.part + ((size_t)(jb + u * SS) * M + m) * a.d + n) : 0.f;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) sum += v[u];
+          }
+          red[tid] = sum;
+        }
+        for (int h = SS >> 1; h >= 1; h >>= 1) {
+          math_sync();
+          if (tid < h * nb) red[tid] += red[tid + h * nb];
+        }
+        math_sync();
+        if (tid < nb) {
+          const int o = base + tid;
+          const int tl = o / (16 * M), rem = o % (16 * M), m = rem / 16, row = rem % 16;
+          const int n = (sh.o0 + tl) * 16 + row;
+          const float res = l == 0 ? __bfloat162float(cur[(size_t)m * a.d + n]) : yo[o];
+          const __nv_bfloat16 yb = __float2bfloat16_rn(red[tid] + res);
+          dst[(size_t)m * a.d + n] = yb;
+          if (a.states) B16(a.states)[((size_t)l * M + m) * a.d + n] = yb;
+          yo[o] = __bfloat162float(yb);  // the next layer's residual and tile partials
+        }
+        math_sync();
       }
       math_sync();
       // the next layer's tile partials of the stored y: same fma order as the
       // first layer's (w_c * y_c over the tile's features in order)
       if (!last) {
-        const float *yv = red + (size_t)splits * nout;  // [tl][m][16]
+        const float *yv = yo;  // [tl][m][16]
         for (int i = tid; i < sh.no * M * Qp; i += kSMathThreads) {
           const int tl = i / (M * Qp), rem = i % (M * Qp), m = rem / Qp, qq = rem % Qp;
           const int t = sh.o0 + tl;
@@ -720,6 +843,7 @@ __global__ void __launch_bounds__(kSThreads, 1) stack_kernel(const __grid_consta
         }
       }
     }
+    if (!last) prefetch_lb(l + 1);
     math_sync();
     if (!last) {
       grid_arrive(a.ctr);
@@ -782,15 +906,8 @@ bool stack_plan(int M, int d, int inter, int r, int bits_gu, int g_gu, int g_dn,
     if (s.ne > 0 && (s.j0 * 4 < s.g0 || (s.j0 + s.nj) * 4 > s.g0 + s.T)) p.h_barrier = 1;
   }
   const int BPK = bits_gu == 2 ? 512 : 1024, GPBg = 128 / g_gu, GPH = g_dn == 32 ? 2 : 1;
-  const int gu_unit = 2 * p.Tmax * (BPK + GPBg * 64);  // one k-block of the CTA's rows
-  const int dn_cell = 512 + GPH * 64;
-  p.SB = std::max(gu_unit, 16 * dn_cell);
-  p.SB = (p.SB + 127) / 128 * 128;
-  p.kps = std::max(1, p.SB / gu_unit);
-  p.cps = p.SB / dn_cell;
   const int MP = 8;  // token columns of the MMA
   const int nout = p.own_max * 16 * M;
-  const int splits = std::max(1, std::min(kSMathThreads / std::max(nout, 1), p.U));
   p.nchk = std::max(1, std::min(kSMathThreads / (M * (p.Qp / 4)), p.RTd));
   uint32_t off = 0;
   p.off_full = off;  off = up128(off + 64 * 8);
@@ -808,15 +925,31 @@ bool stack_plan(int M, int d, int inter, int r, int bits_gu, int g_gu, int g_dn,
   p.off_lb = off;    off = up128(off + (uint32_t)2 * p.Tmax * 16 * r * 2);
   p.off_la = off;    off = up128(off + (uint32_t)p.own_max * 16 * 2 * r * 2);
   p.off_rt = off;    off = up128(off + (uint32_t)M * p.Qp * 4);
-  const uint32_t red_tp = (uint32_t)p.nchk * M * p.Qp * 4;
-  // a CTA owning fewer tiles splits its sums further: at most (512 + nout) values
-  const uint32_t red_own = (uint32_t)(kSMathThreads + nout) * 4;
-  (void)splits;
-  p.off_red = off;   off = up128(off + std::max(red_tp, red_own));
+  p.off_yo = off;    off = up128(off + (uint32_t)nout * 4);
+  p.off_red = off;   off = up128(off + (uint32_t)kSMathThreads * 16);
   off = (off + 1023) / 1024 * 1024;
   p.off_ring = off;
   constexpr uint32_t kSmemLimit = 232448;
-  if (off + 2u * (uint32_t)p.SB > kSmemLimit) return false;
+  // The ring's stages.  A gate/up stage: `depth` k-blocks for each of the
+  // WPT k-slice warps of a tile (kps blocks of the CTA's rows; codes and gmy
+  // groups of meta per projection and row tile); a down stage: RPS = 32 depth
+  // row tiles of a half block (2 depth cells for each of the 16 warps).
+  // Depth 2 (two independent MMA chains per warp and projection) unless
+  // fewer than four such stages fit.
+  const int dn_cell = 512 + GPH * 64;
+  auto gmy_of = [&](int k) { return (k * GPBg + 1) / 2 * 2; };
+  auto gu_stage = [&](int k) { return 2 * p.Tmax * (k * BPK + gmy_of(k) * 64); };
+  for (int depth = 2; depth >= 1; --depth) {
+    p.kps = std::min(depth * p.WPT, p.KBg);
+    p.RPS = 2 * depth * kSW;
+    p.SB = std::max(gu_stage(p.kps), p.RPS * dn_cell);
+    p.SB = (p.SB + 127) / 128 * 128;
+    if (off + 4u * (uint32_t)p.SB <= kSmemLimit) break;
+  }
+  p.gmy = gmy_of(p.kps);
+  p.cps = p.RPS;
+  p.Tbox = p.RTg % p.G == 0 ? p.Tmax : 1;
+  if (p.gmy > 256 || p.kps * BPK / 128 > 256) return false;  // TMA box limits
   p.NS = std::min(64, (int)((kSmemLimit - off) / (uint32_t)p.SB));
   if (p.NS < 4) return false;
   p.smem = off + (uint32_t)p.NS * p.SB;
@@ -827,7 +960,7 @@ bool stack_plan(int M, int d, int inter, int r, int bits_gu, int g_gu, int g_dn,
 namespace {
 
 template <int B, int GG, int GD>
-cudaError_t launch_stack_t(const StackArgs &a, const StackPlan &p, cudaStream_t s) {
+cudaError_t launch_stack_t(const StackArgs &a, const StackPlan &p, const StackMaps &maps, cudaStream_t s) {
   auto kern = stack_kernel<B, GG, GD>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
   if (e != cudaSuccess) return e;
@@ -841,24 +974,82 @@ cudaError_t launch_stack_t(const StackArgs &a, const StackPlan &p, cudaStream_t 
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a, p);
+  return cudaLaunchKernelEx(&cfg, kern, a, p, maps);
 }
 
 template <int B>
-cudaError_t launch_stack_b(const StackArgs &a, const StackPlan &p, cudaStream_t s) {
+cudaError_t launch_stack_b(const StackArgs &a, const StackPlan &p, const StackMaps &maps, cudaStream_t s) {
   if (a.g_gu != a.g_dn) return cudaErrorInvalidValue;
   switch (a.g_gu) {
-    case 32: return launch_stack_t<B, 32, 32>(a, p, s);
-    case 64: return launch_stack_t<B, 64, 64>(a, p, s);
-    case 128: return launch_stack_t<B, 128, 128>(a, p, s);
+    case 32: return launch_stack_t<B, 32, 32>(a, p, maps, s);
+    case 64: return launch_stack_t<B, 64, 64>(a, p, maps, s);
+    case 128: return launch_stack_t<B, 128, 128>(a, p, maps, s);
   }
   return cudaErrorInvalidValue;
 }
 
+// cuTensorMapEncodeTiled from the driver (looked up once).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// A 3-D byte view [z][y][x] of a packed buffer (x = inner bytes), boxes of bx x by x bz.
+cudaError_t encode3(const void *base, uint64_t x, uint64_t y, uint64_t z, uint32_t by, uint32_t bz, CUtensorMap *out) {
+  using Key = std::tuple<const void *, uint64_t, uint64_t, uint64_t, uint32_t, uint32_t>;
+  static std::mutex mu;
+  static std::map<Key, CUtensorMap> cache;
+  const Key key{base, x, y, z, by, bz};
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *out = it->second;
+    return cudaSuccess;
+  }
+  PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[3] = {x, y, z};
+  const cuuint64_t strides[2] = {x, x * y};
+  const cuuint32_t box[3] = {(cuuint32_t)x, by, bz};
+  const cuuint32_t e1[3] = {1, 1, 1};
+  if (fn(out, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void *>(base), dims, strides, box, e1,
+         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  if (cache.size() > 65536) cache.clear();
+  cache[key] = *out;
+  return cudaSuccess;
+}
+
 }  // namespace
 
-cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, cudaStream_t s) {
-  return a.bits_gu == 2 ? launch_stack_b<2>(a, p, s) : launch_stack_b<4>(a, p, s);
+cudaError_t stack_layer_maps(const void *gate_codes, const void *up_codes, const void *gate_meta, const void *up_meta,
+                             const void *down_codes, const void *down_meta, int d, int inter, int bits_gu, int group,
+                             const StackPlan &p, CUtensorMap out[6]) {
+  const uint64_t BPK = bits_gu == 2 ? 512 : 1024, GPB = 128 / group, GPH = group == 32 ? 2 : 1;
+  const uint64_t RTg = (uint64_t)inter / 16, KBg = (uint64_t)d / 128, RTd = (uint64_t)d / 16, KBd = (uint64_t)inter / 128;
+  const uint64_t NGd = KBd * 128 / group;
+  cudaError_t e;
+  if ((e = encode3(gate_codes, 128, KBg * BPK / 128, RTg, (uint32_t)(p.kps * BPK / 128), p.Tbox, &out[0])) != cudaSuccess ||
+      (e = encode3(up_codes, 128, KBg * BPK / 128, RTg, (uint32_t)(p.kps * BPK / 128), p.Tbox, &out[1])) != cudaSuccess ||
+      (e = encode3(gate_meta, 64, KBg * GPB, RTg, (uint32_t)p.gmy, p.Tbox, &out[2])) != cudaSuccess ||
+      (e = encode3(up_meta, 64, KBg * GPB, RTg, (uint32_t)p.gmy, p.Tbox, &out[3])) != cudaSuccess ||
+      (e = encode3(down_codes, 128, KBd * 8, RTd, 4, (uint32_t)p.RPS, &out[4])) != cudaSuccess ||
+      (e = encode3(down_meta, 64, NGd, RTd, (uint32_t)GPH, (uint32_t)p.RPS, &out[5])) != cudaSuccess)
+    return e;
+  return cudaSuccess;
+}
+
+cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, const StackMaps &maps, cudaStream_t s) {
+  return a.bits_gu == 2 ? launch_stack_b<2>(a, p, maps, s) : launch_stack_b<4>(a, p, maps, s);
 }
 
 cudaError_t read_stack_status(int *status) {

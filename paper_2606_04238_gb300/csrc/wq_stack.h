@@ -6,6 +6,7 @@
 #include <cstddef>
 #include <cstdint>
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace wq {
@@ -23,21 +24,33 @@ struct StackPlan {
   int Qp;                // tile-partial stride
   int h_barrier;         // a CTA's down slice needs other CTAs' h: barrier before the down phase
   int nchk;              // chunks of the tile-partial sum
+  int Tbox;              // row tiles per gate/up TMA box (all of a CTA's when every CTA has Tmax, else 1)
+  int gmy;               // groups per gate/up meta box row: kps * 128 / group rounded up to even (128-byte rows)
+  int RPS;               // down row tiles per stage (one TMA box)
   uint32_t smem;
   uint32_t off_full, off_empty, off_misc, off_x, off_xsc, off_xs, off_slot, off_h, off_hp, off_hsc, off_hxs, off_lb,
-      off_la, off_rt, off_red, off_ring;
+      off_la, off_rt, off_yo, off_red, off_ring;
   int xstride;           // halves per token row of the activation panel
 };
 
 struct StackLayerDev {
-  const uint8_t *codes[3];    // packed codes of gate, up, down
-  const uint8_t *meta[3];     // packed binary16 scales / zeros
   const uint16_t *lora_a;     // bf16 [2r][d]
   const uint16_t *lora_b[2];  // bf16 [inter][r]
   float lora_scale;
 };
 
-constexpr int kStackMaxLayers = 64;  // layers a launch carries (longer stacks take several launches)
+// Layers a launch carries (longer stacks take several launches): the tensor
+// maps of a layer take 768 bytes of the launch's 32 KB parameter space.
+constexpr int kStackMaxLayers = 32;
+
+// TMA tensor maps of a layer's packed weights (3-D views of the packed format):
+//   gate/up codes [RT][KB * BPK / 128][128 B], boxes of Tbox row tiles x kps blocks;
+//   gate/up meta  [RT][KB * 128 / group][64 B], boxes of Tbox row tiles x gmy groups;
+//   down codes    [RT][KB * 8][128 B], boxes of RPS row tiles x one 64-feature half block;
+//   down meta     [RT][NG][64 B], boxes of RPS row tiles x the groups of a half block.
+struct StackMaps {
+  CUtensorMap m[kStackMaxLayers][6];  // gate codes, up codes, gate meta, up meta, down codes, down meta
+};
 
 struct StackArgs {
   int M, d, inter, r, g_gu, g_dn, bits_gu, n_layers, prenorm;
@@ -58,7 +71,11 @@ struct StackArgs {
 bool stack_plan(int M, int d, int inter, int r, int bits_gu, int g_gu, int g_dn, int num_sms, StackPlan *out);
 // Workspace bytes of its buffers (after the arrival counter).
 size_t stack_buffer_bytes(int M, int d, int inter, int r);
-cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, cudaStream_t s);
+// The tensor maps of one layer (cached by pointer and shape).
+cudaError_t stack_layer_maps(const void *gate_codes, const void *up_codes, const void *gate_meta, const void *up_meta,
+                             const void *down_codes, const void *down_meta, int d, int inter, int bits_gu, int group,
+                             const StackPlan &p, CUtensorMap out[6]);
+cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, const StackMaps &maps, cudaStream_t s);
 // Reads and clears the stack kernel's device status word.
 cudaError_t read_stack_status(int *status);
 

@@ -18,6 +18,7 @@ from . import _build
 
 WQ_PRENORM = 1
 WQ_LAUNCH_CHAIN = 2
+WQ_LAUNCH_STACK = 4
 WQ_BF16 = 0
 WQ_F32 = 1
 
@@ -301,14 +302,15 @@ class LayerTable:
         self.array = (_MLPLayer * max(1, len(self.layers)))(*[l.c() for l in self.layers])
 
 
-def _stack_flags(prenorm: bool, chain: bool) -> int:
-    return (WQ_PRENORM if prenorm else 0) | (WQ_LAUNCH_CHAIN if chain else 0)
+def _stack_flags(prenorm: bool, chain: bool, stack: bool = False) -> int:
+    return (WQ_PRENORM if prenorm else 0) | (WQ_LAUNCH_CHAIN if chain else 0) | (WQ_LAUNCH_STACK if stack else 0)
 
 
 def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTable | None = None,
-                chain: bool = False):
+                chain: bool = False, stack: bool = False):
     """Stack of gated-MLP layers (wq_mlp_forward) on the current stream; chain=True
-    asks for the per-layer launch chain (WQ_LAUNCH_CHAIN)."""
+    asks for the per-layer launch chain (WQ_LAUNCH_CHAIN), stack=True for the
+    single-launch stack kernel (WQ_LAUNCH_STACK)."""
     m, d = x.shape
     if table is None:
         table = LayerTable(layers)
@@ -317,13 +319,14 @@ def mlp_forward(x, layers, prenorm: bool = True, y=None, ws=None, table: LayerTa
     if ws is None:
         l0 = table.layers[0]
         ws = workspace(max(m, 1), d, l0.gate.n, l0.r, device=x.device)
-    _check(lib().wq_mlp_forward(_ptr(x), m, table.array, len(table.layers), _stack_flags(prenorm, chain), _ptr(y),
+    _check(lib().wq_mlp_forward(_ptr(x), m, table.array, len(table.layers), _stack_flags(prenorm, chain, stack), _ptr(y),
                                 _ptr(ws), ws.numel(), _stream()))
     return y
 
 
 def mlp_forward_states(x, layers, prenorm: bool = True, states=None, h_states=None, y=None, ws=None,
-                       table: LayerTable | None = None, chain: bool = False, with_h: bool = False):
+                       table: LayerTable | None = None, chain: bool = False, with_h: bool = False,
+                       stack: bool = False):
     """wq_mlp_forward_states: the stack plus every layer's output, bf16 [n_layers, m, d], and with
     with_h=True every layer's h, bf16 [n_layers, m, inter].  Returns (y, states, h_states)."""
     m, d = x.shape
@@ -340,7 +343,7 @@ def mlp_forward_states(x, layers, prenorm: bool = True, states=None, h_states=No
     if ws is None:
         l0 = table.layers[0]
         ws = workspace(max(m, 1), d, l0.gate.n, l0.r, device=x.device)
-    _check(lib().wq_mlp_forward_states(_ptr(x), m, table.array, n, _stack_flags(prenorm, chain), _ptr(y),
+    _check(lib().wq_mlp_forward_states(_ptr(x), m, table.array, n, _stack_flags(prenorm, chain, stack), _ptr(y),
                                        _ptr(states), _ptr(h_states), _ptr(ws), ws.numel(), _stream()))
     return y, states, h_states
 
@@ -350,12 +353,12 @@ _STEP_FIELDS = ("rb", "kp", "wk", "tpw", "panels", "ctas")
 
 
 def mlp_forward_info(m: int, layers, prenorm: bool = True, table: LayerTable | None = None,
-                     chain: bool = False) -> dict:
+                     chain: bool = False, stack: bool = False) -> dict:
     """How wq_mlp_forward would run this stack (wq_mlp_forward_info)."""
     if table is None:
         table = LayerTable(layers)
     arr = (ctypes.c_int64 * 16)()
-    _check(lib().wq_mlp_forward_info(m, table.array, len(table.layers), _stack_flags(prenorm, chain), arr))
+    _check(lib().wq_mlp_forward_info(m, table.array, len(table.layers), _stack_flags(prenorm, chain, stack), arr))
     v = list(arr)
     out = {"route": v[0]}
     if v[0] == ROUTE_STACK:

@@ -52,12 +52,12 @@ def _layers(wq, d, inter, group, r, n, bits_gu=2, seed=0):
 def _check(wq, layers, ents, group, m, prenorm, what, x_seed=5):
     d = layers[0].gate.k
     inter = layers[0].gate.n
-    info = wq.mlp_forward_info(m, layers, prenorm=prenorm)
+    info = wq.mlp_forward_info(m, layers, prenorm=prenorm, stack=True)
     assert info["route"] == wq.ROUTE_STACK, info
     x = synth.activations((m, d), x_seed).cuda()
     ws = wq.workspace(m, d, inter, layers[0].r)
-    y, states, h_states = wq.mlp_forward_states(x, layers, prenorm=prenorm, ws=ws, with_h=True)
-    y2 = wq.mlp_forward(x, layers, prenorm=prenorm, ws=ws)
+    y, states, h_states = wq.mlp_forward_states(x, layers, prenorm=prenorm, ws=ws, with_h=True, stack=True)
+    y2 = wq.mlp_forward(x, layers, prenorm=prenorm, ws=ws, stack=True)
     torch.cuda.synchronize()
     assert wq.device_status() == 0
     assert torch.equal(y.view(torch.int16), y2.view(torch.int16)), "two runs differ"
@@ -118,16 +118,16 @@ def test_stack_kernel_in_cuda_graph(wq):
     x = synth.activations((m, cfg.d), 11).cuda()
     ws = wq.workspace(m, cfg.d, cfg.inter, 16)
     table = wq.LayerTable(layers)
-    y_eager = wq.mlp_forward(x, layers, prenorm=True, ws=ws, table=table).clone()
+    y_eager = wq.mlp_forward(x, layers, prenorm=True, ws=ws, table=table, stack=True).clone()
     y = torch.empty_like(x)
     s = torch.cuda.Stream()
     s.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(s):
-        wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table)
+        wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table, stack=True)
     torch.cuda.current_stream().wait_stream(s)
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
-        wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table)
+        wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table, stack=True)
     for _ in range(5):
         y.zero_()
         g.replay()
@@ -145,8 +145,17 @@ def test_stack_kernel_and_chain_share_a_workspace(wq):
     for rep in range(2):
         for m, chain in ((1, False), (1, True), (130, False), (4, False)):
             x = synth.activations((m, cfg.d), 40 + m).cuda()
-            outs.append(wq.mlp_forward(x, layers, prenorm=True, ws=ws, chain=chain))
+            outs.append(wq.mlp_forward(x, layers, prenorm=True, ws=ws, chain=chain, stack=not chain))
     torch.cuda.synchronize()
     assert wq.device_status() == 0
     for a_, b_ in zip(outs[:4], outs[4:]):
         assert torch.equal(a_.view(torch.int16), b_.view(torch.int16))
+
+
+def test_default_route_follows_the_measured_crossover(wq):
+    cfg = synth.CONFIGS["qwen3_4b"]
+    layers, _ = _layers(wq, cfg.d, cfg.inter, 128, 16, 2, seed=12)
+    assert wq.mlp_forward_info(1, layers)["route"] == wq.ROUTE_GEMV_CHAIN
+    for m in (2, 4, 8):
+        assert wq.mlp_forward_info(m, layers)["route"] == wq.ROUTE_STACK
+    assert wq.mlp_forward_info(16, layers)["route"] == wq.ROUTE_GEMV_CHAIN
