@@ -74,7 +74,7 @@ struct WsLayout {
   size_t cnt1, cnt2, sctr, sk_cnt;
   size_t tp, xa, xb, h, hq, hsc, hxs, part1, part2;
   // dequant-GEMM path (m > kMaxTokens, or a shape the GEMV path has no plan for)
-  size_t x16, rs, ta, h16, sk_part;
+  size_t x16, rs, ta, h16, hsx, sk_part;
   bool gemm;  // the GEMM buffers are laid out
   // single-launch stack (1..8 tokens)
   size_t sxw, stp, shg, spart, sxc;
@@ -142,6 +142,7 @@ bool gemm_layout(int m, int d, int inter, size_t off, WsLayout *L) {
   L->rs = off;      off = up256(off + (size_t)m * 4);
   L->ta = off;      off = up256(off + (size_t)m * 2 * kMaxRank * 2);
   L->h16 = off;     off = up256(off + (size_t)m * ldi * 2);
+  L->hsx = off;     off = up256(off + (size_t)m * 4);
   L->sk_part = off; off = up256(off + part * 4);
   L->gemm = true;
   L->total = off;
@@ -332,18 +333,18 @@ wq_status run_down(const void *h, int m, const wq_qweight *down, const void *res
 
 // ---- dequant-GEMM path (m > kMaxTokens): tcgen05 tensor cores ----
 // gate/up: binary16 copy of x, RMSNorm scales and lora_scale * x A^T first,
-// then the GEMM (h in bf16, and in binary16 at h16 for the down GEMM when
-// h16 is not null).
+// then the GEMM (h in bf16).
 wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
                           const void *lora_a, const void *lora_bg, const void *lora_bu, int r, float lora_scale,
-                          unsigned flags, void *h, uint16_t *h16, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
+                          unsigned flags, void *h, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
   const int d = gate->k, inter = gate->n;
   const int lda = (d + 127) / 128 * 128;
   if (!L.gemm) return fail(WQ_ERR_WORKSPACE, "workspace laid out without the dequant-GEMM buffers");
   uint16_t *x16 = reinterpret_cast<uint16_t *>(ws + L.x16);
   float *rs = reinterpret_cast<float *>(ws + L.rs);
   uint16_t *ta = reinterpret_cast<uint16_t *>(ws + L.ta);
-  cudaError_t e = launch_gemm_prep(x, m, d, lda, r > 0 ? lora_a : nullptr, r > 0 ? 2 * r : 0, lora_scale, x16, rs, ta, s);
+  cudaError_t e = launch_gemm_prep(x, m, d, lda, r > 0 ? lora_a : nullptr, r > 0 ? 2 * r : 0, lora_scale,
+                                   (flags & WQ_PRENORM) ? 1 : 0, x16, rs, ta, s);
   if (e != cudaSuccess) return cuda_fail(e, "GEMM input launch");
   GemmArgs a = {};
   a.act = x16;
@@ -360,10 +361,8 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
   a.r = r;
   a.lora_b[0] = lora_bg;
   a.lora_b[1] = lora_bu;
-  a.rs = (flags & WQ_PRENORM) ? rs : nullptr;
+  a.rs = rs;
   a.out = h;
-  a.out_f16 = h16;
-  a.ldo16 = (inter + 127) / 128 * 128;
   a.sk_part = reinterpret_cast<float *>(ws + L.sk_part);
   a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.sk_cnt);
   e = launch_gemm(kind, a, s);
@@ -371,17 +370,15 @@ wq_status run_gateup_gemm(GemvKind kind, const void *x, int m, const wq_qweight 
   return WQ_OK;
 }
 
-// down: from the binary16 h16 (null: converted from the bf16 h first).
-wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qweight *down, const void *residual,
+// down: h converted to binary16 first (scaled per token), then the GEMM.
+wq_status run_down_gemm(const void *h, int m, const wq_qweight *down, const void *residual,
                         void *y, int y_f32, const WsLayout &L, uint8_t *ws, cudaStream_t s) {
   if (!L.gemm) return fail(WQ_ERR_WORKSPACE, "workspace laid out without the dequant-GEMM buffers");
   const int K = down->k, lda = (K + 127) / 128 * 128;
-  if (!h16) {
-    uint16_t *c = reinterpret_cast<uint16_t *>(ws + L.h16);
-    cudaError_t e = launch_to_f16(h, m, K, lda, c, s);
-    if (e != cudaSuccess) return cuda_fail(e, "GEMM input launch");
-    h16 = c;
-  }
+  uint16_t *h16 = reinterpret_cast<uint16_t *>(ws + L.h16);
+  float *hsx = reinterpret_cast<float *>(ws + L.hsx);
+  cudaError_t e = launch_to_f16(h, m, K, lda, h16, hsx, s);
+  if (e != cudaSuccess) return cuda_fail(e, "GEMM input launch");
   GemmArgs a = {};
   a.act = h16;
   a.lda = lda;
@@ -392,11 +389,12 @@ wq_status run_down_gemm(const void *h, const uint16_t *h16, int m, const wq_qwei
   a.codes[0] = down->codes;
   a.meta[0] = down->meta;
   a.residual = residual;
+  a.rs = hsx;
   a.out = y;
   a.out_f32 = y_f32;
   a.sk_part = reinterpret_cast<float *>(ws + L.sk_part);
   a.sk_cnt = reinterpret_cast<unsigned *>(ws + L.sk_cnt);
-  cudaError_t e = launch_gemm(kDownW4, a, s);
+  e = launch_gemm(kDownW4, a, s);
   if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   return WQ_OK;
 }
@@ -458,7 +456,7 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, gate->k, gate->n, &L)) != WQ_OK) return st;
   if (gateup_uses_gemm(kind, m, gate, r))
-    st = run_gateup_gemm(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
+    st = run_gateup_gemm(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, L,
                          static_cast<uint8_t *>(ws), static_cast<cudaStream_t>(stream));
   else
     st = run_gateup(kind, x, m, gate, up, lora_a, bg, bu, r, lora_scale, flags, h, nullptr, L,
@@ -651,7 +649,7 @@ wq_status wq_down_w4(const void *h, int m, const wq_qweight *down, const void *r
   WsLayout L;
   if ((st = check_ws(ws, ws_bytes, m, down->n, down->k, &L)) != WQ_OK) return st;
   if (down_uses_gemm(m, down, 0))
-    st = run_down_gemm(h, nullptr, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
+    st = run_down_gemm(h, m, down, residual, y, y_dtype == WQ_F32, L, static_cast<uint8_t *>(ws),
                        static_cast<cudaStream_t>(stream));
   else
     st = run_down(h, m, down, residual, y, y_dtype == WQ_F32, nullptr, 0, nullptr, L, static_cast<uint8_t *>(ws),
@@ -855,18 +853,17 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     return ok();
   }
   if (route == kRouteGemmChain) {
-    // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up (h also in
-    // binary16), down with the residual
+    // dequant-GEMM chain: per layer the GEMM inputs of x, gate/up, the
+    // binary16 copy of h (scaled per token), down with the residual
     const void *cur = x;
     for (int l = 0; l < n_layers; ++l) {
       const wq_mlp_layer &Ly = layers[l];
       void *out = layer_out(l);
       const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
-      uint16_t *h16 = reinterpret_cast<uint16_t *>(w8 + L.h16);
       st = run_gateup_gemm(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale,
-                           flags, layer_h(l), h16, L, w8, s);
+                           flags, layer_h(l), L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
-      st = run_down_gemm(nullptr, h16, m, &Ly.down, cur, out, 0, L, w8, s);
+      st = run_down_gemm(layer_h(l), m, &Ly.down, cur, out, 0, L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
       cur = out;
     }

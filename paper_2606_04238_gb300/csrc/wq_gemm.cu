@@ -323,9 +323,10 @@ __device__ __forceinline__ void gemm_issue_stage(uint32_t tmem, uint32_t as0, ui
 }
 
 // Output of 8 consecutive rows nb .. nb + 7 of token m from the fp32 sums g
-// (and u for gate/up): h = SiLU(rs g) * (rs u) (also in binary16 when asked),
-// or y = g + residual in bf16 or fp32.  `vec`: 16-byte stores (N and the
-// binary16 row length multiples of 8).
+// (and u for gate/up): h = SiLU(rs g) * (rs u),
+// or y = rs g + residual in bf16 or fp32 (rs: the token's factor that undoes
+// the power-of-two scale of its binary16 activations, times its RMSNorm scale
+// for gate/up).  `vec`: 16-byte stores (N a multiple of 8).
 template <int NPROJ>
 __device__ __forceinline__ void gemm_finish(const GemmArgs &a, int m, int nb, float rs, const float (&g)[8],
                                             const float (&u)[8], bool vec) {
@@ -339,7 +340,7 @@ __device__ __forceinline__ void gemm_finish(const GemmArgs &a, int m, int nb, fl
     }
   } else {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = g[e];
+    for (int e = 0; e < 8; ++e) v[e] = rs * g[e];
     if (a.residual) {
       if (vec) {
         const uint4 rv =
@@ -367,11 +368,6 @@ __device__ __forceinline__ void gemm_finish(const GemmArgs &a, int m, int nb, fl
       }
       *reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) + (size_t)m * a.N + nb) =
           make_uint4(w[0], w[1], w[2], w[3]);
-      if (NPROJ == 2 && a.out_f16) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) w[e] = h2bits(__floats2half2_rn(v[2 * e], v[2 * e + 1]));
-        *reinterpret_cast<uint4 *>(a.out_f16 + (size_t)m * a.ldo16 + nb) = make_uint4(w[0], w[1], w[2], w[3]);
-      }
     }
   } else {
     for (int e = 0; e < 8 && nb + e < a.N; ++e) {
@@ -380,7 +376,6 @@ __device__ __forceinline__ void gemm_finish(const GemmArgs &a, int m, int nb, fl
         reinterpret_cast<float *>(a.out)[o] = v[e];
       } else {
         reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v[e]);
-        if (NPROJ == 2 && a.out_f16) a.out_f16[(size_t)m * a.ldo16 + nb + e] = __half_as_ushort(__float2half_rn(v[e]));
       }
     }
   }
@@ -535,10 +530,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_tile_kernel(const GemmA
     if (wait(sm.acc_full, 0)) {
       tc_fence_after();
       const int quarter = warp & 3, c0 = (warp >> 2) * 32;
-      const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
+      const bool vec = (a.N & 7) == 0;
       for (int h = 0; h < mth; ++h) {
         const int m = m0 + h * kBM + quarter * 32 + lane;
-        const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+        const float rs = (a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
         const uint32_t tl = tmem + h * C::NCH + ((uint32_t)(quarter * 32) << 16);
         for (int c = c0; c < c0 + 32; c += 8) {
           uint32_t gw[8], uw[8];
@@ -589,14 +584,14 @@ __device__ __noinline__ void gemm_part_epilogue(const GemmArgs &a, uint32_t tmem
   const int MT = (a.M + a.mt * kBM - 1) / (a.mt * kBM);
   const int m0 = (tile % MT) * a.mt * kBM, n0 = (tile / MT) * kBN;
   const int mth = min(a.mt, (a.M - m0 + kBM - 1) / kBM);
-  const bool vec = (a.N & 7) == 0 && (!a.out_f16 || (a.ldo16 & 7) == 0);
+  const bool vec = (a.N & 7) == 0;
   constexpr int SLOT = kHalves * kBM * C::NCH;  // floats of a scratch slot: [half][NCH / 8][128 tokens][8]
   const bool whole = ub == 0 && ue == U;
   // a split part's scratch slot: the CTA's first part (0) or its last (1)
   float *mine = whole ? nullptr : a.sk_part + ((size_t)blockIdx.x * 2 + ((long long)tile * U + ub == g0 ? 0 : 1)) * SLOT;
   for (int h = 0; h < mth && have; ++h) {
     const int m = m0 + h * kBM + quarter * 32 + lane;
-    const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+    const float rs = (a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
     const uint32_t tl = tmem + h * C::NCH + ((uint32_t)(quarter * 32) << 16);
     for (int c = c0; c < c0 + 32; c += 8) {
       uint32_t gw[8], uw[8];
@@ -647,7 +642,7 @@ __device__ __noinline__ void gemm_part_epilogue(const GemmArgs &a, uint32_t tmem
   if (!*last_s) return;
   for (int h = 0; h < mth; ++h) {
     const int m = m0 + h * kBM + quarter * 32 + lane;
-    const float rs = (NPROJ == 2 && a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
+    const float rs = (a.rs != nullptr && m < a.M) ? a.rs[m] : 1.f;
     for (int c = c0; c < c0 + 32; c += 8) {
       float g[8], u[8];
 #pragma unroll
@@ -839,10 +834,12 @@ constexpr int kPrepTok = 16, kPrepRows = 16, kPrepWarps = 16, kPrepUnroll = 2;
 
 __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_bfloat16 *x, int M, int K, int lda16,
                                                                    const __nv_bfloat16 *lora_a, int r2,
-                                                                   float lora_scale, uint16_t *x16, float *rs,
-                                                                   uint16_t *ta) {
+                                                                   float lora_scale, int prenorm, uint16_t *x16,
+                                                                   float *rs, uint16_t *ta) {
   __shared__ float part[kPrepWarps][kPrepTok][kPrepRows + 1];
   __shared__ float ssp[kPrepWarps][kPrepTok];
+  __shared__ uint32_t mxp[kPrepWarps][kPrepTok];
+  __shared__ float scl[kPrepTok];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, g = lane >> 2, t = lane & 3;
   const int m0 = blockIdx.x * kPrepTok, j0 = blockIdx.y * kPrepRows;
   const int nchunk = K / 32;
@@ -851,6 +848,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
 #pragma unroll
   for (int i = 0; i < 8; ++i) acc[i >> 2][i & 3] = 0.f;
   float ss[2] = {0.f, 0.f};  // tokens g and g + 8 of the block
+  uint32_t mx[2] = {0u, 0u};  // their largest |x| (bit patterns of non-negative floats order like the values)
   const auto word = [](const uint4 &v, int q) { return q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w; };
   for (int cb = warp; cb < nchunk; cb += kPrepWarps * kPrepUnroll) {
     uint4 xa[kPrepUnroll][2], ab[kPrepUnroll][2];
@@ -883,19 +881,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
           const float lo = __uint_as_float(w[e] << 16), hi = __uint_as_float(w[e] & 0xffff0000u);
           ss[i] = fmaf(lo, lo, ss[i]);
           ss[i] = fmaf(hi, hi, ss[i]);
-        }
-      }
-      if (c % gridDim.y == blockIdx.y) {
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const int m = m0 + g + 8 * i;
-          if (m >= M) continue;
-          const uint32_t w[4] = {xa[u][i].x, xa[u][i].y, xa[u][i].z, xa[u][i].w};
-          uint32_t o[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            o[e] = h2bits(__floats2half2_rn(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u)));
-          *reinterpret_cast<uint4 *>(x16 + (size_t)m * lda16 + k) = make_uint4(o[0], o[1], o[2], o[3]);
+          mx[i] = max(mx[i], max((w[e] << 16) & 0x7fffffffu, w[e] & 0x7fff0000u));
         }
       }
       if (lora) {
@@ -917,9 +903,16 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
     ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 1);
     ss[i] += __shfl_xor_sync(0xffffffffu, ss[i], 2);
   }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    mx[i] = max(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 1));
+    mx[i] = max(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 2));
+  }
   if (t == 0) {
     ssp[warp][g] = ss[0];
     ssp[warp][g + 8] = ss[1];
+    mxp[warp][g] = mx[0];
+    mxp[warp][g + 8] = mx[1];
   }
   if (lora) {
     // accumulator (row, col) of n-tile nt: rows g / g + 8, cols 2t, 2t+1
@@ -932,10 +925,58 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
     }
   }
   __syncthreads();
-  if (blockIdx.y == 0 && tid < kPrepTok && m0 + tid < M) {
-    float tot = 0.f;
-    for (int w = 0; w < kPrepWarps; ++w) tot += ssp[w][tid];
-    rs[m0 + tid] = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)K), kRmsEps)));
+  // Per token an exact power of two 2^e puts its largest |x| in [2^4, 2^5):
+  // the binary16 copies of x and of t = lora_scale x A^T are taken of the
+  // values times 2^e (no overflow: 2^11 below the binary16 maximum even for
+  // |t| up to 2^10 |x|; every element within 2^-22 of the largest stays
+  // exact), and the epilogue multiplies the fp32 sums by rs 2^-e, which
+  // undoes it exactly.
+  if (tid < kPrepTok) {
+    uint32_t mxb = 0u;
+    for (int w = 0; w < kPrepWarps; ++w) mxb = max(mxb, mxp[w][tid]);
+    const int be = (int)(mxb >> 23);
+    const int e = mxb == 0u || be >= 255 ? 0 : max(-100, min(100, 131 - be));
+    scl[tid] = __int_as_float((e + 127) << 23);
+    if (blockIdx.y == 0 && m0 + tid < M) {
+      float tot = 0.f;
+      for (int w = 0; w < kPrepWarps; ++w) tot += ssp[w][tid];
+      const float r = prenorm ? __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)K), kRmsEps))) : 1.f;
+      rs[m0 + tid] = r * __int_as_float((127 - e) << 23);
+    }
+  }
+  __syncthreads();
+  // the binary16 copy of x (2^e x): this CTA's chunks c = blockIdx.y + cc
+  // gridDim.y, 16 bytes an item, four loads in flight a thread
+  {
+    const int ncc = (nchunk - (int)blockIdx.y + (int)gridDim.y - 1) / (int)gridDim.y;
+    const int items = kPrepTok * ncc * 4;
+    constexpr int NT = kPrepWarps * 32;
+    for (int i0 = tid; i0 < items; i0 += 4 * NT) {
+      uint4 v[4];
+      int tl[4];
+      size_t dst[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * NT;
+        tl[u] = i / (ncc * 4);
+        const int rem = i % (ncc * 4), c = (int)blockIdx.y + (rem / 4) * (int)gridDim.y, k = c * 32 + 8 * (rem % 4);
+        const int m = m0 + tl[u];
+        const bool ok = i < items && m < M;
+        dst[u] = ok ? (size_t)m * lda16 + k : ~(size_t)0;
+        v[u] = ok ? __ldg(reinterpret_cast<const uint4 *>(x + (size_t)m * K + k)) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (dst[u] == ~(size_t)0) continue;
+        const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+        const float sc = scl[tl[u]];
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          o[e] = h2bits(__floats2half2_rn(__uint_as_float(w[e] << 16) * sc, __uint_as_float(w[e] & 0xffff0000u) * sc));
+        *reinterpret_cast<uint4 *>(x16 + dst[u]) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
   }
   if (lora) {
     for (int o = tid; o < kPrepTok * kPrepRows; o += kPrepWarps * 32) {
@@ -944,7 +985,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
       if (m >= M || j >= r2) continue;
       float v = 0.f;
       for (int w = 0; w < kPrepWarps; ++w) v += part[w][tl][jl];
-      ta[(size_t)m * r2 + j] = __half_as_ushort(__float2half_rn(lora_scale * v));
+      ta[(size_t)m * r2 + j] = __half_as_ushort(__float2half_rn(lora_scale * v * scl[tl]));
     }
   }
   // zeros past K
@@ -955,13 +996,44 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
     }
 }
 
-// bf16 [M, K] -> binary16 [M, lda16] (zero padded), the down GEMM's A operand.
-__global__ void __launch_bounds__(256) to_f16_kernel(const __nv_bfloat16 *x, int M, int K, int lda16, uint16_t *x16) {
-  const size_t n = (size_t)M * lda16;
-  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-    const size_t m = i / lda16, k = i % lda16;
-    x16[i] = k < (size_t)K ? __half_as_ushort(__float2half_rn(__bfloat162float(x[m * K + k]))) : (uint16_t)0;
+// bf16 [M, K] -> binary16 [M, lda16] (zero padded), the down GEMM's A
+// operand, one CTA per token: an exact power of two 2^e puts the token's
+// largest |x| in [2^4, 2^5) (no overflow, every element within 2^-22 of the
+// largest exact); sx[m] = 2^-e, by which the epilogue multiplies the sums.
+// K a multiple of 8.
+__global__ void __launch_bounds__(256) to_f16_kernel(const __nv_bfloat16 *x, int M, int K, int lda16, uint16_t *x16,
+                                                     float *sx) {
+  __shared__ uint32_t wmax[8];
+  const int m = blockIdx.x, tid = threadIdx.x;
+  if (m >= M) return;
+  const uint4 *row = reinterpret_cast<const uint4 *>(x + (size_t)m * K);
+  const int n8 = K / 8;
+  uint32_t mx = 0u;
+  for (int i = tid; i < n8; i += blockDim.x) {
+    const uint4 v = __ldg(row + i);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) mx = max(mx, max((w[e] << 16) & 0x7fffffffu, w[e] & 0x7fff0000u));
   }
+  mx = __reduce_max_sync(0xffffffffu, mx);
+  if ((tid & 31) == 0) wmax[tid >> 5] = mx;
+  __syncthreads();
+  mx = 0u;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) mx = max(mx, wmax[w]);
+  const int be = (int)(mx >> 23);
+  const int e = mx == 0u || be >= 255 ? 0 : max(-100, min(100, 131 - be));
+  const float sc = __int_as_float((e + 127) << 23);
+  if (tid == 0) sx[m] = __int_as_float((127 - e) << 23);
+  for (int i = tid; i < n8; i += blockDim.x) {
+    const uint4 v = __ldg(row + i);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      o[q] = h2bits(__floats2half2_rn(__uint_as_float(w[q] << 16) * sc, __uint_as_float(w[q] & 0xffff0000u) * sc));
+    *reinterpret_cast<uint4 *>(x16 + (size_t)m * lda16 + 8 * i) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+  for (int k = K + tid; k < lda16; k += blockDim.x) x16[(size_t)m * lda16 + k] = 0;
 }
 
 // cuTensorMapEncodeTiled from the driver (looked up once).
@@ -1113,21 +1185,19 @@ size_t gemm_scratch_floats(int M, int N, int K, int nproj, int num_sms) {
 size_t gemm_counters(int M, int N) { return (size_t)((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN); }
 
 cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void *lora_a, int r2, float lora_scale,
-                             uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t s) {
+                             int prenorm, uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
   if (K % 32 != 0 || lda16 < K) return cudaErrorInvalidValue;
   const dim3 grid((M + kPrepTok - 1) / kPrepTok, r2 > 0 ? (r2 + kPrepRows - 1) / kPrepRows : 1);
   gemm_prep_kernel<<<grid, kPrepWarps * 32, 0, s>>>(
       reinterpret_cast<const __nv_bfloat16 *>(x), M, K, lda16, reinterpret_cast<const __nv_bfloat16 *>(lora_a), r2,
-      lora_scale, x16, rs, ta);
+      lora_scale, prenorm, x16, rs, ta);
   return cudaGetLastError();
 }
-
-cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, cudaStream_t s) {
+cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, float *sx, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  const size_t n = (size_t)M * lda16;
-  const int blocks = (int)std::min<size_t>((n + 255) / 256, 4096);
-  to_f16_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(x), M, K, lda16, x16);
+  if (K % 8 != 0 || lda16 < K) return cudaErrorInvalidValue;
+  to_f16_kernel<<<M, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(x), M, K, lda16, x16, sx);
   return cudaGetLastError();
 }
 

@@ -98,12 +98,11 @@ struct GemmArgs {
   const uint16_t *ta;        // gate/up with LoRA: binary16 [M][2r] = lora_scale * x A^T (gate rows, up rows)
   int r;
   const void *lora_b[2];     // bf16 [N][r]
-  const float *rs;           // gate/up: RMSNorm scale per token, or null
+  const float *rs;           // per token: the factor of the fp32 sums (2^-e of the binary16 activations'
+                             // scale, times the RMSNorm scale for gate/up), or null for 1
   const void *residual;      // down: bf16 [M][N] or null
   void *out;                 // bf16 (or fp32 for down with out_f32) [M][N]
   int out_f32;
-  uint16_t *out_f16;         // gate/up: h also as binary16 [M][ldo16] (the down GEMM's A), or null
-  int ldo16;
   int mt;                    // token halves of 128 per CTA (1 or 2; set by launch_gemm)
   // stream-K scratch (null: one CTA per tile): gemm_scratch_floats() fp32 and
   // gemm_counters() arrival counters, zero between launches
@@ -111,11 +110,15 @@ struct GemmArgs {
   unsigned *sk_cnt;
 };
 cudaError_t launch_gemm(GemvKind kind, const GemmArgs &args, cudaStream_t stream);
-// x16 [M][lda16] = binary16(x), rs[m] = 1/sqrt(mean(x^2) + eps), ta [M][r2] = lora_scale * x A^T (r2 > 0)
+// Per token m of x [M, K]: an exact power of two 2^e puts max|x[m]| in
+// [2^4, 2^5); x16 [M][lda16] = binary16(2^e x), ta [M][r2] = binary16(2^e
+// lora_scale x A^T) (r2 > 0), rs[m] = 2^-e / sqrt(mean(x^2) + eps) (prenorm)
+// or 2^-e: the factor the gate/up GEMM's epilogue applies to its sums.
 cudaError_t launch_gemm_prep(const void *x, int M, int K, int lda16, const void *lora_a, int r2, float lora_scale,
-                             uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t stream);
-// x16 [M][lda16] = binary16(x) (zero padded)
-cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, cudaStream_t stream);
+                             int prenorm, uint16_t *x16, float *rs, uint16_t *ta, cudaStream_t stream);
+// x16 [M][lda16] = binary16(2^e x) (zero padded), e per token putting its
+// max|x| in [2^4, 2^5); sx[m] = 2^-e (the down GEMM's epilogue factor).
+cudaError_t launch_to_f16(const void *x, int M, int K, int lda16, uint16_t *x16, float *sx, cudaStream_t stream);
 // Stream-K scratch a GEMM launch of this shape can need: fp32 partial sums
 // and per-tile arrival counters (num_sms: the device's SM count).
 size_t gemm_scratch_floats(int M, int N, int K, int nproj, int num_sms);

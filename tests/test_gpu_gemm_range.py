@@ -1,0 +1,109 @@
+"""The batched dequant-GEMM path on activations far from unit scale.
+
+The tcgen05 path multiplies binary16 copies of the activations.  Each token
+is scaled by an exact power of two before the narrowing (its largest |x| put
+in [16, 32)) and the epilogue undoes it, so tokens of any magnitude keep the
+precision of unit-scale ones: here tokens span 1e-6 .. 1e5 (gate/up with
+and without the RMSNorm, down with bf16 and fp32 output) and a stack without
+the RMSNorm whose h reaches ~1e6 (past the binary16 maximum 65504).  Every
+token is checked against the oracle with its own bound.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from paper_2606_04238_gb300 import synth
+from tests.gpu_util import check_bf16, check_f32, upload_packed
+
+pytestmark = pytest.mark.gpu
+
+MIN_EXACT = 0.6  # the GEMM path's share of outputs equal to the oracle's own bf16 rounding
+
+
+@pytest.fixture(scope="module")
+def wq():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04238_gb300 import wq as mod
+    return mod
+
+
+def _q(shape, group, bits, seed):
+    w = (np.random.default_rng(seed).standard_normal(shape) * 0.02).astype(np.float32)
+    return orc.quantize(w, group, bits)[:3]
+
+
+def _wide(m, n, seed, lo=-6.0, hi=5.0):
+    """bf16 [m, n]: N(0, 1) rows scaled by 10^k, k spread over [lo, hi] across the tokens."""
+    x = synth.activations((m, n), seed).float()
+    k = torch.linspace(lo, hi, m).unsqueeze(1)
+    return (x * torch.pow(10.0, k)).to(torch.bfloat16)
+
+
+def _per_token(got, ref, what, min_exact=MIN_EXACT, f32=False):
+    for i in range(ref.shape[0]):
+        if f32:
+            check_f32(got[i:i + 1], ref[i:i + 1], f"{what} token {i}")
+        else:
+            check_bf16(got[i:i + 1], ref[i:i + 1], f"{what} token {i}", min_exact=min_exact)
+
+
+@pytest.mark.parametrize("m", [65, 512])
+@pytest.mark.parametrize("prenorm", [False, True])
+def test_gateup_wide_range(wq, m, prenorm):
+    d, inter, group, r = 512, 1024, 128, 16
+    qg, qu = _q((inter, d), group, 2, 5), _q((inter, d), group, 2, 6)
+    x = _wide(m, d, 7)
+    a, bg, bu = synth.lora(d, inter, r, 8)
+    h = wq.gateup_w2_lora(x.cuda(), upload_packed(*qg, group, 2), upload_packed(*qu, group, 2), a.cuda(), bg.cuda(),
+                          bu.cuda(), lora_scale=2.0, prenorm=prenorm)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.gateup(synth.bf16_bits(x), qg, qu, group, synth.bf16_bits(a), synth.bf16_bits(bg),
+                        synth.bf16_bits(bu), lora_scale=2.0, prenorm=prenorm)
+    assert np.isfinite(h.float().cpu().numpy()).all()
+    _per_token(h, ref, f"gate/up m={m} prenorm={prenorm}")
+
+
+@pytest.mark.parametrize("m", [65, 512])
+def test_down_wide_range(wq, m):
+    d, inter, group = 512, 1024, 128
+    qd = _q((d, inter), group, 4, 9)
+    h = _wide(m, inter, 10)
+    res = _wide(m, d, 11)
+    dn = upload_packed(*qd, group, 4)
+    y = wq.down_w4(h.cuda(), dn, residual=res.cuda())
+    y32 = wq.down_w4(h.cuda(), dn, residual=res.cuda(), out_f32=True)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.down(synth.bf16_bits(h), qd, group, synth.bf16_bits(res))
+    _per_token(y, ref, f"down m={m}")
+    _per_token(y32, ref, f"down f32 m={m}", f32=True)
+
+
+def test_gemm_stack_without_rmsnorm_large_h(wq):
+    """Two layers on the GEMM chain without the RMSNorm: h grows with |x|^2
+    (to ~1e6 here) and crosses the binary16 range; each layer teacher-forced."""
+    d, inter, group, r, m = 512, 1024, 128, 8, 65
+    layers, ents = [], []
+    for l in range(2):
+        qg, qu, qd = _q((inter, d), group, 2, 20 + l), _q((inter, d), group, 2, 30 + l), _q((d, inter), group, 4, 40 + l)
+        a, bg, bu = synth.lora(d, inter, r, 50 + l)
+        layers.append(wq.MLPLayer(upload_packed(*qg, group, 2), upload_packed(*qu, group, 2), upload_packed(*qd, group, 4),
+                                  lora_a=a.cuda(), lora_b_gate=bg.cuda(), lora_b_up=bu.cuda(), lora_scale=2.0))
+        ents.append(dict(g=qg, u=qu, d=qd, a=synth.bf16_bits(a), bg=synth.bf16_bits(bg), bu=synth.bf16_bits(bu)))
+    x = _wide(m, d, 12, lo=-2.0, hi=3.0)
+    assert wq.mlp_forward_info(m, layers, prenorm=False)["route"] == wq.ROUTE_GEMM_CHAIN
+    _, states, h_states = wq.mlp_forward_states(x.cuda(), layers, prenorm=False, with_h=True)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    assert h_states.float().abs().max().item() > 65504.0  # past the binary16 range
+    prev = synth.bf16_bits(x)
+    for l, ent in enumerate(ents):
+        h_ref, _ = orc.gateup(prev, ent["g"], ent["u"], group, ent["a"], ent["bg"], ent["bu"], lora_scale=2.0,
+                              prenorm=False)
+        _per_token(h_states[l], h_ref, f"stack layer {l} h")
+        y_ref, _ = orc.down(synth.bf16_bits(h_states[l].cpu()), ent["d"], group, prev)
+        _per_token(states[l], y_ref, f"stack layer {l} y")
+        prev = synth.bf16_bits(states[l].cpu())
