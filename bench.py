@@ -215,6 +215,17 @@ def recorded_traffic(kernel, files=GEMV_SOURCES):
     return e.get("dram_bytes_per_launch")
 
 
+def stack_config(cfg, n_layers, m, ws_):
+    """The workload description both arms report."""
+    gu_bytes, dn_bytes = algorithmic_bytes(cfg, m)
+    return {"workload": f"{cfg.name}_mlp_stack_{n_layers}L_m{m}", "model": f"{cfg.name}-shaped MLP stack",
+            "d": cfg.d, "inter": cfg.inter, "layers": n_layers, "m": m, "global_batch": m * ws_,
+            "seq_len": 1, "group": cfg.group_gu, "lora_r": cfg.r, "lora_scale": cfg.lora_scale,
+            "prenorm": True, "parallelism": f"replicas x{ws_}",
+            "l2": f"no flush: {n_layers * (gu_bytes + dn_bytes) / 1e9:.2f} GB of packed weights per step "
+                  "(> 129 MB L2)"}
+
+
 # --------------------------------------------------------------------------- GPU arm
 def build_stack(wq, synth, cfg, n_layers, bits_gu, lora, dev):
     import torch
@@ -371,12 +382,9 @@ def run_gpu(args):
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_, "steps": steps, "warmup": warmup,
            "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "w2/w4 codes x f16 mma, f32 accumulate, bf16 activations", "data": "synthetic",
-           "config": {"workload": f"{cfg.name}_mlp_stack_{n_layers}L_m{m}", "model": f"{cfg.name}-shaped MLP stack",
-                      "d": cfg.d, "inter": cfg.inter, "layers": n_layers, "m": m, "global_batch": m * ws_,
-                      "seq_len": 1, "group": cfg.group_gu, "lora_r": cfg.r, "lora_scale": cfg.lora_scale,
-                      "prenorm": True, "parallelism": f"replicas x{ws_}",
-                      "l2": f"no flush: {n_layers * (gu_bytes + dn_bytes) / 1e9:.2f} GB of packed weights per step "
-                            "(> 129 MB L2)"},
+           "config": stack_config(cfg, n_layers, m, ws_),
+           "route": ("launch chain", "dequant-GEMM chain", "single-launch stack kernel")[
+               wq.mlp_forward_info(m, layers, table=table)["route"]],
            "gpu_launches": launches_per_step * steps, "clocks": clocks, "e2e": e2e,
            "stack_gbs": n_layers * (gu_bytes + dn_bytes) / (ms_step / 1e3) / 1e9}
 
@@ -454,6 +462,8 @@ def run_gpu(args):
         torch.cuda.empty_cache()
         out["prefill"] = run_prefill(wq, synth, dev, args.prefill_layers, max(20, min(steps, 200)), warmup)
         torch.cuda.empty_cache()
+        out["decoder_layer"] = run_decoder(wq, synth, dev, max(10, min(steps, 50)), warmup)
+        out["sweep"] = run_sweep(wq, synth, dev, max(10, min(steps, 50)), warmup, BENCH_SWEEP)["rows"]
         out["cpu_baseline"] = cpu_oracle_sample(cfg, m)
 
     if rank == 0:
@@ -462,9 +472,11 @@ def run_gpu(args):
 
 
 SWEEP = (("qwen3_4b", (1, 2, 4, 8, 16, 32, 64)), ("dense_8b", (1, 4, 16, 32, 64)), ("dense_14b", (1, 16, 64)))
+# the decode token counts of the benchmark configurations (4B stack, 8B and 14B stacks), in the bench line
+BENCH_SWEEP = (("qwen3_4b", (2, 4, 8, 16)), ("dense_8b", (1, 4, 16, 64)), ("dense_14b", (1, 16, 64)))
 
 
-def run_sweep(wq, synth, dev, steps, warmup):
+def run_sweep(wq, synth, dev, steps, warmup, sweep=SWEEP):
     """Decode MLP stacks of the 4B, 8B and 14B shapes (all layers, W2 gate/up
     + LoRA, W4 down, RMSNorm) at their token counts: tokens/s, µs per step and
     the stack's algorithmic bytes per step over the measured HBM bandwidth."""
@@ -472,7 +484,7 @@ def run_sweep(wq, synth, dev, steps, warmup):
     peak, src = measured_peaks()
     out = {"metric": "decode MLP-stack tokens/s over token counts", "peak_gbs": peak, "peak_source": src,
            "data": "synthetic", "rows": []}
-    for name, ms in SWEEP:
+    for name, ms in sweep:
         cfg = synth.CONFIGS[name]
         layers = build_stack(wq, synth, cfg, cfg.layers, 2, True, dev)
         table = wq.LayerTable(layers)
@@ -485,7 +497,10 @@ def run_sweep(wq, synth, dev, steps, warmup):
             t_step = ms_tot / steps / 1e3
             gu, dn = algorithmic_bytes(cfg, m)
             gbs = cfg.layers * (gu + dn) / t_step / 1e9
-            out["rows"].append({"config": name, "layers": cfg.layers, "m": m, "tokens_per_s": m / t_step,
+            out["rows"].append({"config": name, "layers": cfg.layers, "m": m,
+                                "route": ("launch chain", "dequant-GEMM chain", "single-launch stack kernel")[
+                                    wq.mlp_forward_info(m, layers, table=table)["route"]],
+                                "tokens_per_s": m / t_step,
                                 "us_per_step": t_step * 1e6, "us_per_layer": t_step * 1e6 / cfg.layers,
                                 "stack_gbs": gbs, "frac_of_hbm": gbs / peak, "clocks": clocks})
             assert wq.device_status() == 0
@@ -560,10 +575,80 @@ def run_prefill(wq, synth, dev, n_layers, steps, warmup, eager=False):
     }
 
 
+DECODER_CONTEXTS = (1024, 8192, 32768)
+DECODER_HEADS = (32, 8, 128)  # query heads, kv heads, head_dim of the Qwen3-4B attention
+
+
+def run_decoder(wq, synth, dev, steps, warmup, n_layers=None, contexts=DECODER_CONTEXTS, batch=1):
+    """One decode step through whole decoder layers of the Qwen3-4B shape
+    (4-bit q/k/v/o projections, grouped-query attention over a bf16 KV cache,
+    then the MLP block) at several context lengths, with the MLP at
+    W4/W2-GateUp (2-bit gate/up + LoRA) and at uniform W4: the decode rate and
+    the gain of the 2-bit gate/up over context (the attention's cache reads
+    grow with the context while the MLP's bytes stay fixed)."""
+    import torch
+    cfg = synth.CONFIGS["qwen3_4b"]
+    n_layers = n_layers or cfg.layers
+    H, Hkv, hd = DECODER_HEADS
+    max_ctx = max(contexts)
+    attn, caches, mlps = [], [], {2: [], 4: []}
+    for l in range(n_layers):
+        wqkv = synth.weights(((H + 2 * Hkv) * hd, cfg.d), 7000 + 2 * l, device=dev)
+        wo = synth.weights((cfg.d, H * hd), 7001 + 2 * l, device=dev)
+        attn.append((wq.pack(wqkv, 128, 4), wq.pack(wo, 128, 4)))
+        del wqkv, wo
+        g = torch.Generator(device=dev)
+        g.manual_seed(9000 + l)
+        kc = torch.randn((batch, Hkv, max_ctx, hd), generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn((batch, Hkv, max_ctx, hd), generator=g, device=dev).to(torch.bfloat16)
+        caches.append((kc, vc))
+    for bits in (2, 4):
+        mlps[bits] = build_stack(wq, synth, cfg, n_layers, bits, bits == 2, dev)
+    wm = torch.empty((cfg.inter, cfg.d), dtype=torch.float32, device=dev)
+    mlps["merged"] = [wq.merge_layer(L, w_merged=wm) for L in mlps[2]]  # 2-bit codes, adapters merged (r = 0)
+    del wm
+    x = synth.activations((batch, cfg.d), 77, device=dev)
+    bufs = [torch.empty_like(x) for _ in range(2)]
+    rows = []
+    for ctx in contexts:
+        lens = torch.full((batch,), ctx - 1, dtype=torch.int32, device=dev)
+        row = {"context": ctx}
+        for bits, name in ((4, "w4"), (2, "w4w2_gateup"), ("merged", "w4w2_gateup_merged")):
+            layers = [wq.DecoderLayer(attn[l][0], attn[l][1], mlps[bits][l], H, Hkv, hd) for l in range(n_layers)]
+            cls = [L.c() for L in layers]
+            ws = wq.decoder_workspace(batch, layers[0], max_ctx)
+
+            def step():
+                cur = x
+                for l in range(n_layers):
+                    out = bufs[l & 1]
+                    wq.decoder_layer_forward(cur, lens, layers[l], caches[l][0], caches[l][1], y=out, ws=ws, c_layer=cls[l])
+                    cur = out
+
+            ms, _ = time_graph(capture(step), steps, warmup)
+            assert wq.device_status() == 0
+            t = ms / steps / 1e3
+            row[name] = {"tokens_per_s": batch / t, "us_per_layer": t * 1e6 / n_layers}
+            del ws
+        row["gain_pct"] = 100.0 * (row["w4w2_gateup"]["tokens_per_s"] / row["w4"]["tokens_per_s"] - 1.0)
+        row["gain_pct_merged"] = 100.0 * (row["w4w2_gateup_merged"]["tokens_per_s"] / row["w4"]["tokens_per_s"] - 1.0)
+        rows.append(row)
+    del caches, mlps, attn
+    torch.cuda.empty_cache()
+    return {"workload": f"qwen3_4b_decoder_{n_layers}L_b{batch}", "heads": {"q": H, "kv": Hkv, "head_dim": hd},
+            "kv_cache": "bf16, random N(0, 1) contents up to the context",
+            "rows": rows,
+            "note": "one decode step through whole decoder layers (attention projections 4-bit g128; the MLP as "
+                    "standalone gate/up and down calls): uniform W4 (no adapter), W4/W2-GateUp with the unmerged "
+                    "rank-16 adapter, and W4/W2-GateUp with the adapter merged into the 2-bit codes; gain_pct and "
+                    "gain_pct_merged are the decode-rate gains of the last two over uniform W4"}
+
+
 # --------------------------------------------------------------------------- reference arm
 def run_reference(args):
-    """The oracle as it stands, on the host cores: each step is one layer of
-    the stack (a bounded sample); the rate is scaled to the whole stack."""
+    """The oracle as it stands, on the host cores: each timed step is one layer
+    of the stack (a bounded sample; ms_per_step is that measured time); the
+    rate is the whole stack's, m / (layers x the time a step)."""
     ws_ = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -597,14 +682,13 @@ def run_reference(args):
     el = time.perf_counter() - t0
     per_layer = el / max(1, args.steps)
     value = m / (per_layer * n_layers)
-    sample = (f"each step = 1 of the {n_layers} layers at m={m} (fp64 C oracle, OpenMP); rate scaled to the "
-              f"whole stack; {per_layer * 1e3:.1f} ms per layer")
+    sample = (f"each timed step is 1 of the {n_layers} layers at m={m} (fp64 C oracle, OpenMP, {nprep} distinct "
+              f"layers cycled); value = m / ({n_layers} x the measured time a step); {per_layer * 1e3:.1f} ms a step")
     print(json.dumps({"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_,
-                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * n_layers * 1e3,
+                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * 1e3,
+                      "step_unit": f"one layer of the {n_layers}-layer stack",
                       "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-                      "data": "synthetic",
-                      "config": {"workload": f"{cfg.name}_mlp_stack_{n_layers}L_m{m}", "d": cfg.d, "inter": cfg.inter,
-                                 "layers": n_layers, "m": m},
+                      "data": "synthetic", "config": stack_config(cfg, n_layers, m, ws_),
                       "cpu_baseline": {"value": value, "unit": UNIT, "cores": orc.threads(), "kind": "oracle",
                                        "sample": sample},
                       "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))

@@ -22,9 +22,10 @@
  *   - Supported: group in {32, 64, 128}; in-features a multiple of the group
  *     (WQ_ERR_SHAPE otherwise); 1 <= m <= 16384 tokens (m == 0 is a no-op);
  *     LoRA rank r a multiple of 8, r <= 64 (r == 0: no adapter).
- *   - Two paths behind the same calls: up to 16 tokens the dequant-GEMV
- *     kernels (exact products of the codes and binary16 activations on the
- *     mma.sync tensor-core path, fp32 sums); above 16 tokens, and for a layer
+ *   - Two paths behind the same calls: up to 16 tokens (8 for layers of
+ *     hidden size d >= 4096) the dequant-GEMV kernels (exact products of the
+ *     codes and binary16 activations on the mma.sync tensor-core path, fp32
+ *     sums); above that, and for a layer
  *     shape the GEMV kernels have no launch configuration for at the given
  *     token count, the batched dequant-GEMM on the tcgen05 tensor cores
  *     (activations and each dequantized weight s (q - z) rounded once to
@@ -199,13 +200,15 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
  * paper has no counterpart to this call; it is a deployment convenience.
  *
  * Same arguments and results as wq_gateup_w2_lora minus ws / ws_bytes, for
- * the decode token counts 1 <= m <= 16 (the dequant-GEMV path).  The scratch
+ * the decode token counts of the dequant-GEMV path (1 <= m <= 16, or 8 for
+ * d >= 4096).  The scratch
  * it needs (per-16-feature RMSNorm and LoRA-A partial sums of x, split-K
  * partial sums and arrival counters) lives in a fixed array of
  * WQ_NOALLOC_SCRATCH_BYTES bytes inside the library, which every GPU that
  * loads the library keeps until the process exits.  It returns
  * WQ_ERR_UNSUPPORTED and launches nothing when
- *   - m > 16 (wq_gateup_w2_lora takes the dequant-GEMM path there),
+ *   - m above the dequant-GEMV path's limit (wq_gateup_w2_lora takes the
+ *     dequant-GEMM path there),
  *   - the layer shape has no dequant-GEMV launch configuration at this m
  *     (wq_gateup_w2_lora takes the dequant-GEMM path for it), or
  *   - the layer needs more scratch than the array holds.
@@ -270,11 +273,60 @@ wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, c
  *   - the launch chain: 2 kernels per layer (plus one for the first layer's
  *     input statistics) with programmatic dependent launch, each down launch
  *     also producing the next layer's RMSNorm and LoRA-A partial sums;
- *   - the dequant-GEMM chain above 16 tokens.
+ *   - the dequant-GEMM chain above 16 tokens (8 for d >= 4096).
  * Every route can be captured into a CUDA graph.
  */
 wq_status wq_mlp_forward(const void *x, int m, const wq_mlp_layer *layers, int n_layers,
                          unsigned flags, void *y, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * One decode step of grouped-query attention over a bf16 KV cache: the
+ * decoder-layer operator around the MLP block whose cost Sec. 5 counts as
+ * independent of the weight precision (Sec. 7 step 4 puts its projections at
+ * INT4).  Per sequence b (one new token) and query head h (kv head
+ * g = h / (n_heads / n_kv)):
+ *   rs  = 1 / sqrt(mean(x[b]^2) + 1e-6)           (the layer input's RMSNorm)
+ *   q_h = RoPE(headnorm(rs qkv[b, q_h])), k_g = RoPE(headnorm(rs qkv[b, k_g])),
+ *   v_g = rs qkv[b, v_g]; k_g, v_g rounded to bf16 and written to the caches at
+ *   position lens[b]; headnorm: unit-weight RMSNorm over the head (eps 1e-6);
+ *   RoPE: element i with i + head_dim/2, angle lens[b] theta^(-2i/head_dim);
+ *   o[b, h] = bf16( softmax_j(q_h . K[b,g,j] / sqrt(head_dim)) V[b,g,j] ), j = 0..lens[b].
+ *   qkv:     fp32 [batch, (n_heads + 2 n_kv) head_dim] = x deq(Wqkv)^T before the
+ *            RMSNorm scale (e.g. wq_down_w4 with WQ_F32 on the rows of Wq, Wk, Wv).
+ *   x:       bf16 [batch, d], the layer input.
+ *   lens:    int32 [batch] on the device: positions already cached.  A length
+ *            outside [0, max_len) skips that sequence and records WQ_ERR_ARG in
+ *            the device status (wq_device_status).
+ *   caches:  bf16 [batch, n_kv, max_len, head_dim].  o: bf16 [batch, n_heads head_dim].
+ *   Supported: head_dim 64 or 128, n_heads a multiple of n_kv, n_heads / n_kv <= 8.
+ *   Workspace: wq_attn_workspace_bytes (split partial results, no zeroing needed).
+ */
+size_t wq_attn_workspace_bytes(int batch, int n_heads, int n_kv, int head_dim, int max_len);
+wq_status wq_attn_decode(const float *qkv, const void *x, const int32_t *lens, int batch, int d, int n_heads,
+                         int n_kv, int head_dim, float theta, void *k_cache, void *v_cache, int max_len, void *o,
+                         void *ws, size_t ws_bytes, void *stream);
+
+/* A decoder layer: 4-bit attention projections around the MLP block. */
+typedef struct {
+    wq_qweight qkv;        /* bits 4, [(n_heads + 2 n_kv) head_dim, d]: the rows of Wq, then Wk, then Wv */
+    wq_qweight o;          /* bits 4, [d, n_heads head_dim] */
+    wq_mlp_layer mlp;
+    int32_t n_heads, n_kv, head_dim;
+    float rope_theta;
+} wq_decoder_layer;
+
+/*
+ * One decode step of a decoder layer for `batch` sequences:
+ *   qkv = x deq(Wqkv)^T (fp32), o = wq_attn_decode(...), x1 = bf16(x + o deq(Wo)^T),
+ *   y = the MLP block on x1 (as wq_gateup_* then wq_down_w4 with residual x1;
+ *   flags as for wq_mlp_forward, WQ_PRENORM for the MLP's RMSNorm).
+ * Five calls on `stream`; the caches gain position lens[b] (lens is not changed).
+ * Workspace: wq_decoder_workspace_bytes, zero-filled before first use (wq_workspace_init).
+ */
+size_t wq_decoder_workspace_bytes(int batch, const wq_decoder_layer *layer, int max_len);
+wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens, const wq_decoder_layer *layer,
+                                   void *k_cache, void *v_cache, int max_len, unsigned flags, void *y, void *ws,
+                                   size_t ws_bytes, void *stream);
 
 /*
  * wq_mlp_forward that also returns every layer's output (the hidden states of
@@ -322,8 +374,9 @@ wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t 
 /* Message of the last error returned on this host thread ("" if none). */
 const char *wq_last_error(void);
 
-/* Reads and clears the device-side status word (WQ_OK or WQ_ERR_TIMEOUT) of
- * the current device.  Synchronizes the device. */
+/* Reads and clears the device-side status words of the current device: WQ_OK,
+ * WQ_ERR_TIMEOUT (a bounded wait ran out) or WQ_ERR_ARG (wq_attn_decode met a
+ * sequence length outside its cache).  Synchronizes the device. */
 wq_status wq_device_status(int *status);
 
 /* Library version string. */

@@ -84,6 +84,13 @@ struct WsLayout {
 
 size_t up256(size_t v) { return (v + 255) / 256 * 256; }
 
+// Token count above which the calls take the dequant-GEMM path: 16, or 8 for
+// layers of hidden size 4096 and more (measured on GB300: at 16 tokens the
+// launch chain of the d 4096 and d 5120 stacks took 157 and 266 us a layer,
+// the GEMM chain at 64 tokens 119 and 147 us; up to 8 tokens the single-launch
+// stack kernel serves those shapes).
+int gemv_prefer_tokens(int d) { return d >= 4096 ? 8 : kGemvPreferTokens; }
+
 size_t partial_bytes(const GemvPlan &p, int nproj) {
   return p.P > 1 ? (size_t)p.RT * p.P * nproj * 16 * p.M * 4 : 0;
 }
@@ -188,9 +195,9 @@ bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   L->part2 = off; off = up256(off + p2);
   L->total = off;
   if (gemv_only) return true;
-  // above kGemvPreferTokens, or for a shape that lacks a GEMV plan for some
+  // above gemv_prefer_tokens, or for a shape that lacks a GEMV plan for some
   // group or rank at this token count, the calls take the dequant-GEMM path
-  if (m > kGemvPreferTokens || !all_fit) {
+  if (m > gemv_prefer_tokens(d) || !all_fit) {
     if (!gemm_layout(m, d, inter, off, L)) return false;
     off = L->total;
   }
@@ -198,17 +205,18 @@ bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
   return true;
 }
 
-// Whether a call takes the dequant-GEMM path: above kGemvPreferTokens (where
+
+// Whether a call takes the dequant-GEMM path: above gemv_prefer_tokens (where
 // it is the faster path on every measured layer shape; the GEMV kernels'
 // work grows faster than linearly with the token count), or where the GEMV
 // path has no launch plan.  The workspace holds the GEMM buffers then.
 bool gateup_uses_gemm(GemvKind kind, int m, const wq_qweight *gate, int r) {
-  if (m > kGemvPreferTokens) return true;
+  if (m > gemv_prefer_tokens(gate->k)) return true;
   GemvPlan pl;
   return !plan_gemv(kind, gate->n, gate->k, m, gate->group, r, num_sms(), &pl);
 }
 bool down_uses_gemm(int m, const wq_qweight *down, int r_next) {
-  if (m > kGemvPreferTokens) return true;
+  if (m > gemv_prefer_tokens(down->n)) return true;
   GemvPlan pl;
   return !plan_gemv(kDownW4, down->n, down->k, m, down->group, r_next, num_sms(), &pl);
 }
@@ -607,9 +615,9 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
   if (m == 0) return ok();
   if (!x || !h) return fail(WQ_ERR_ARG, "null x or h");
   if (!aligned16(x) || !aligned16(h)) return fail(WQ_ERR_ALIGN, "x or h not 16-byte aligned");
-  if (m > kGemvPreferTokens)
-    return fail(WQ_ERR_UNSUPPORTED, "m=%d: the built-in scratch serves the decode path (m <= %d; use wq_gateup_w2_lora)",
-                m, kGemvPreferTokens);
+  if (m > gemv_prefer_tokens(gate->k))
+    return fail(WQ_ERR_UNSUPPORTED, "m=%d: the built-in scratch serves the decode path (m <= %d here; use wq_gateup_w2_lora)",
+                m, gemv_prefer_tokens(gate->k));
   GemvPlan plan;
   if (!plan_gemv(kGateUpW2, gate->n, gate->k, m, gate->group, r, num_sms(), &plan))
     return fail(WQ_ERR_UNSUPPORTED,
@@ -715,7 +723,7 @@ wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned 
 
 // How a stack runs: the per-layer dequant-GEMV launch chain, the
 // dequant-GEMM launch chain (every layer's launches need a GEMV plan for the
-// first; above kGemvPreferTokens tokens the second), or the single-launch
+// first; above gemv_prefer_tokens tokens the second), or the single-launch
 // stack kernel (1..8 tokens, every layer with the same bits, groups and rank,
 // unless the caller asks for the chain).
 enum StackRoute { kRouteGemvChain = 0, kRouteGemmChain = 1, kRouteStack = 2 };
@@ -757,7 +765,7 @@ StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned
   StackPlan sp;
   if (((flags & WQ_LAUNCH_STACK) || stack_preferred(m, layers[0])) && stack_kernel_plan(m, layers, n_layers, flags, &sp))
     return kRouteStack;
-  if (m > kGemvPreferTokens) return kRouteGemmChain;
+  if (m > gemv_prefer_tokens(layers[0].gate.k)) return kRouteGemmChain;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
@@ -948,6 +956,122 @@ wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, u
   return ok();
 }
 
+size_t wq_attn_workspace_bytes(int batch, int n_heads, int n_kv, int head_dim, int max_len) {
+  const int sms = num_sms();
+  if (batch <= 0 || n_heads <= 0 || n_kv <= 0 || head_dim <= 0 || max_len <= 0 || sms <= 0) return 0;
+  const int S = attn_splits(batch, n_kv, max_len, sms);
+  return up256((size_t)batch * n_heads * S * (head_dim + 2) * 4);
+}
+
+wq_status wq_attn_decode(const float *qkv, const void *x, const int32_t *lens, int batch, int d, int n_heads, int n_kv,
+                         int head_dim, float theta, void *k_cache, void *v_cache, int max_len, void *o, void *ws,
+                         size_t ws_bytes, void *stream) {
+  if (batch < 0 || d <= 0 || d % 8 != 0) return fail(WQ_ERR_SHAPE, "batch %d, d %d (a positive multiple of 8)", batch, d);
+  if (head_dim != 64 && head_dim != 128) return fail(WQ_ERR_UNSUPPORTED, "head_dim %d not 64 or 128", head_dim);
+  if (n_kv <= 0 || n_heads <= 0 || n_heads % n_kv != 0 || n_heads / n_kv > 8)
+    return fail(WQ_ERR_UNSUPPORTED, "n_heads %d / n_kv %d: a multiple, at most 8 query heads a kv head", n_heads, n_kv);
+  if (max_len <= 0) return fail(WQ_ERR_SHAPE, "max_len %d", max_len);
+  if (!(theta > 0.f)) return fail(WQ_ERR_ARG, "rope theta must be positive");
+  if (batch == 0) return ok();
+  if (!qkv || !x || !lens || !k_cache || !v_cache || !o || !ws) return fail(WQ_ERR_ARG, "null pointer");
+  if (!aligned16(qkv) || !aligned16(x) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(o) ||
+      !aligned16(ws))
+    return fail(WQ_ERR_ALIGN, "qkv, x, caches, o or workspace not 16-byte aligned");
+  if (ws_bytes < wq_attn_workspace_bytes(batch, n_heads, n_kv, head_dim, max_len))
+    return fail(WQ_ERR_WORKSPACE, "attention workspace of %zu bytes, %zu needed", ws_bytes,
+                wq_attn_workspace_bytes(batch, n_heads, n_kv, head_dim, max_len));
+  const int S = attn_splits(batch, n_kv, max_len, num_sms());
+  cudaError_t e = launch_attn_decode(qkv, x, reinterpret_cast<const int *>(lens), batch, d, n_heads, n_kv, head_dim,
+                                     (double)theta, k_cache, v_cache, max_len, static_cast<float *>(ws), S, o,
+                                     static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  return ok();
+}
+
+}  // extern "C"
+
+namespace {
+
+// Regions of a decoder layer's workspace: the MLP's, the two projections'
+// (each with its own arrival counters), the attention partials, then the
+// intermediates qkv (fp32), o, x1 and h (bf16).
+struct DecoderWs {
+  size_t mlp, proj_qkv, proj_o, attn, qkv, o, x1, h, total;
+  size_t n_mlp, n_qkv, n_o, n_attn;
+};
+
+bool decoder_ws(int batch, const wq_decoder_layer &Ly, int max_len, DecoderWs *W) {
+  const int d = Ly.mlp.gate.k, inter = Ly.mlp.gate.n;
+  const int H = Ly.n_heads, Hkv = Ly.n_kv, hd = Ly.head_dim;
+  const int nqkv = (H + 2 * Hkv) * hd;
+  W->n_mlp = wq_workspace_bytes(batch, d, inter, Ly.mlp.r);
+  W->n_qkv = wq_workspace_bytes(batch, nqkv, d, 0);
+  W->n_o = wq_workspace_bytes(batch, d, H * hd, 0);
+  W->n_attn = wq_attn_workspace_bytes(batch, H, Hkv, hd, max_len);
+  if (!W->n_mlp || !W->n_qkv || !W->n_o || !W->n_attn) return false;
+  size_t off = 0;
+  W->mlp = off;      off = up256(off + W->n_mlp);
+  W->proj_qkv = off; off = up256(off + W->n_qkv);
+  W->proj_o = off;   off = up256(off + W->n_o);
+  W->attn = off;     off = up256(off + W->n_attn);
+  W->qkv = off;      off = up256(off + (size_t)batch * nqkv * 4);
+  W->o = off;        off = up256(off + (size_t)batch * H * hd * 2);
+  W->x1 = off;       off = up256(off + (size_t)batch * d * 2);
+  W->h = off;        off = up256(off + (size_t)batch * inter * 2);
+  W->total = off;
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t wq_decoder_workspace_bytes(int batch, const wq_decoder_layer *layer, int max_len) {
+  if (!layer || batch <= 0 || max_len <= 0) return 0;
+  DecoderWs W;
+  return decoder_ws(batch, *layer, max_len, &W) ? W.total : 0;
+}
+
+wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens, const wq_decoder_layer *layer,
+                                   void *k_cache, void *v_cache, int max_len, unsigned flags, void *y, void *ws,
+                                   size_t ws_bytes, void *stream) {
+  if (!layer) return fail(WQ_ERR_ARG, "null layer");
+  const wq_decoder_layer &Ly = *layer;
+  const int d = Ly.mlp.gate.k, inter = Ly.mlp.gate.n;
+  const int H = Ly.n_heads, Hkv = Ly.n_kv, hd = Ly.head_dim;
+  wq_status st;
+  if ((st = check_qweight(&Ly.qkv, 4, "qkv")) != WQ_OK || (st = check_qweight(&Ly.o, 4, "o")) != WQ_OK) return st;
+  if (H <= 0 || Hkv <= 0 || hd <= 0 || Ly.qkv.n != (H + 2 * Hkv) * hd || Ly.qkv.k != d || Ly.o.n != d ||
+      Ly.o.k != H * hd || Ly.mlp.down.n != d || Ly.mlp.down.k != inter)
+    return fail(WQ_ERR_SHAPE, "decoder layer shapes disagree (qkv [%d x %d], o [%d x %d], d %d, heads %d/%d x %d)",
+                Ly.qkv.n, Ly.qkv.k, Ly.o.n, Ly.o.k, d, H, Hkv, hd);
+  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (batch < 0) return fail(WQ_ERR_ARG, "batch %d", batch);
+  if (batch == 0) return ok();
+  DecoderWs W;
+  if (!decoder_ws(batch, Ly, max_len, &W)) return fail(WQ_ERR_SHAPE, "no workspace layout for this layer");
+  if (!ws || ws_bytes < W.total)
+    return fail(WQ_ERR_WORKSPACE, "decoder workspace of %zu bytes, %zu needed", ws_bytes, W.total);
+  uint8_t *w8 = static_cast<uint8_t *>(ws);
+  if ((st = wq_down_w4(x, batch, &Ly.qkv, nullptr, w8 + W.qkv, WQ_F32, w8 + W.proj_qkv, W.n_qkv, stream)) != WQ_OK)
+    return fail(st, "qkv projection: %s", g_last_error.c_str());
+  if ((st = wq_attn_decode(reinterpret_cast<const float *>(w8 + W.qkv), x, lens, batch, d, H, Hkv, hd, Ly.rope_theta,
+                           k_cache, v_cache, max_len, w8 + W.o, w8 + W.attn, W.n_attn, stream)) != WQ_OK)
+    return fail(st, "attention: %s", g_last_error.c_str());
+  if ((st = wq_down_w4(w8 + W.o, batch, &Ly.o, x, w8 + W.x1, WQ_BF16, w8 + W.proj_o, W.n_o, stream)) != WQ_OK)
+    return fail(st, "output projection: %s", g_last_error.c_str());
+  const wq_mlp_layer &M = Ly.mlp;
+  if (M.gate.bits == 2)
+    st = wq_gateup_w2_lora(w8 + W.x1, batch, &M.gate, &M.up, M.lora_a, M.lora_b_gate, M.lora_b_up, M.r, M.lora_scale,
+                           flags, w8 + W.h, w8 + W.mlp, W.n_mlp, stream);
+  else
+    st = wq_gateup_w4(w8 + W.x1, batch, &M.gate, &M.up, flags, w8 + W.h, w8 + W.mlp, W.n_mlp, stream);
+  if (st != WQ_OK) return fail(st, "gate/up: %s", g_last_error.c_str());
+  if ((st = wq_down_w4(w8 + W.h, batch, &M.down, w8 + W.x1, y, WQ_BF16, w8 + W.mlp, W.n_mlp, stream)) != WQ_OK)
+    return fail(st, "down: %s", g_last_error.c_str());
+  return ok();
+}
+
 wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t info[10]) {
   if (!info) return fail(WQ_ERR_ARG, "null info array");
   if (kind < 0 || kind > 2) return fail(WQ_ERR_ARG, "kind %d not in {0, 1, 2}", kind);
@@ -981,6 +1105,9 @@ wq_status wq_device_status(int *status) {
   if (e != cudaSuccess) return cuda_fail(e, "device status read");
   if (*status == 0) *status = g;
   e = read_stack_status(&g);
+  if (e != cudaSuccess) return cuda_fail(e, "device status read");
+  if (*status == 0) *status = g;
+  e = read_attn_status(&g);
   if (e != cudaSuccess) return cuda_fail(e, "device status read");
   if (*status == 0) *status = g;
   return ok();

@@ -19,4 +19,16 @@ cudaError_t launch_merge_lora(const uint32_t *codes, const uint16_t *meta, int n
 cudaError_t launch_down_bf16(const void *h, int m, const void *wd, int d, int inter, const void *residual, void *y,
                              bool y_f32, cudaStream_t stream);
 
+// One decode step of grouped-query attention (wq_attn.cu): qkv fp32
+// [B][(H + 2 Hkv) HD] projections of x (not yet RMSNorm-scaled), x bf16 [B][d],
+// lens [B] device ints, caches bf16 [B][Hkv][max_len][HD] (the new k, v
+// written at lens[b]), part fp32 [B][H][S][HD + 2], o bf16 [B][H HD].
+cudaError_t launch_attn_decode(const float *qkv, const void *x, const int *lens, int B, int d, int H, int Hkv, int HD,
+                               double theta, void *k_cache, void *v_cache, int max_len, float *part, int S, void *o,
+                               cudaStream_t s);
+// Context splits of a launch (S above).
+int attn_splits(int B, int Hkv, int max_len, int num_sms);
+// Reads and clears the attention kernels' device status word.
+cudaError_t read_attn_status(int *status);
+
 }  // namespace wq

@@ -43,6 +43,11 @@ class _MLPLayer(ctypes.Structure):
                 ("lora_scale", ctypes.c_float)]
 
 
+class _DecoderLayer(ctypes.Structure):
+    _fields_ = [("qkv", _QWeight), ("o", _QWeight), ("mlp", _MLPLayer), ("n_heads", ctypes.c_int32),
+                ("n_kv", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("rope_theta", ctypes.c_float)]
+
+
 _lib = None
 
 
@@ -78,6 +83,10 @@ def lib():
             "wq_mlp_forward_states": (I, [P, I, ctypes.POINTER(_MLPLayer), I, U, P, P, P, P, S, P]),
             "wq_mlp_forward_info": (I, [I, ctypes.POINTER(_MLPLayer), I, U, ctypes.POINTER(ctypes.c_int64)]),
             "wq_plan_info": (I, [I, I, I, I, I, I, ctypes.POINTER(ctypes.c_int64)]),
+            "wq_attn_workspace_bytes": (S, [I, I, I, I, I]),
+            "wq_attn_decode": (I, [P, P, P, I, I, I, I, I, F, P, P, I, P, P, S, P]),
+            "wq_decoder_workspace_bytes": (S, [I, ctypes.POINTER(_DecoderLayer), I]),
+            "wq_decoder_layer_forward": (I, [P, I, P, ctypes.POINTER(_DecoderLayer), P, P, I, U, P, P, S, P]),
             "wq_last_error": (ctypes.c_char_p, []),
             "wq_device_status": (I, [ctypes.POINTER(I)]),
             "wq_version": (ctypes.c_char_p, []),
@@ -380,6 +389,70 @@ def plan_info(kind: int, n: int, k: int, m: int, group: int, r: int = 0) -> dict
     arr = (ctypes.c_int64 * 10)()
     _check(lib().wq_plan_info(kind, n, k, m, group, r, arr))
     return dict(zip(PLAN_FIELDS, list(arr)))
+
+
+def attn_workspace(batch: int, n_heads: int, n_kv: int, head_dim: int, max_len: int, device="cuda") -> torch.Tensor:
+    nb = int(lib().wq_attn_workspace_bytes(batch, n_heads, n_kv, head_dim, max_len))
+    if nb == 0:
+        raise WQError(-2, "no attention workspace for these sizes")
+    return torch.empty(nb, dtype=torch.uint8, device=device)
+
+
+def attn_decode(qkv, x, lens, k_cache, v_cache, n_heads: int, n_kv: int, theta: float, o=None, ws=None):
+    """wq_attn_decode: one decode step of grouped-query attention; the caches
+    (bf16 [B, n_kv, max_len, head_dim]) gain position lens[b]."""
+    b, d = x.shape
+    _, hkv, max_len, hd = k_cache.shape
+    assert hkv == n_kv and lens.dtype == torch.int32
+    if o is None:
+        o = torch.empty((b, n_heads * hd), dtype=torch.bfloat16, device=x.device)
+    if ws is None:
+        ws = attn_workspace(b, n_heads, n_kv, hd, max_len, device=x.device)
+    _check(lib().wq_attn_decode(_ptr(qkv), _ptr(x), _ptr(lens), b, d, n_heads, n_kv, hd, float(theta), _ptr(k_cache),
+                                _ptr(v_cache), max_len, _ptr(o), _ptr(ws), ws.numel(), _stream()))
+    return o
+
+
+@dataclass
+class DecoderLayer:
+    """A decoder layer: 4-bit qkv (rows of Wq, Wk, Wv) and o projections around an MLPLayer."""
+    qkv: QWeight
+    o: QWeight
+    mlp: MLPLayer
+    n_heads: int
+    n_kv: int
+    head_dim: int
+    rope_theta: float = 1e6
+
+    def c(self) -> _DecoderLayer:
+        return _DecoderLayer(self.qkv.c(), self.o.c(), self.mlp.c(), self.n_heads, self.n_kv, self.head_dim,
+                             float(self.rope_theta))
+
+
+def decoder_workspace(batch: int, layer: DecoderLayer, max_len: int, device="cuda") -> torch.Tensor:
+    cl = layer.c()
+    nb = int(lib().wq_decoder_workspace_bytes(batch, ctypes.byref(cl), max_len))
+    if nb == 0:
+        raise WQError(-2, "no decoder workspace for these sizes")
+    ws = torch.empty(nb, dtype=torch.uint8, device=device)
+    _check(lib().wq_workspace_init(_ptr(ws), nb, _stream()))
+    return ws
+
+
+def decoder_layer_forward(x, lens, layer: DecoderLayer, k_cache, v_cache, prenorm: bool = True, y=None, ws=None,
+                          c_layer=None):
+    """wq_decoder_layer_forward: one decode step of the layer for x bf16 [B, d]."""
+    b, d = x.shape
+    max_len = k_cache.shape[2]
+    if y is None:
+        y = torch.empty_like(x)
+    if ws is None:
+        ws = decoder_workspace(b, layer, max_len, device=x.device)
+    cl = c_layer if c_layer is not None else layer.c()
+    _check(lib().wq_decoder_layer_forward(_ptr(x), b, _ptr(lens), ctypes.byref(cl), _ptr(k_cache), _ptr(v_cache),
+                                          max_len, WQ_PRENORM if prenorm else 0, _ptr(y), _ptr(ws), ws.numel(),
+                                          _stream()))
+    return y
 
 
 def device_status() -> int:
