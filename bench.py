@@ -459,6 +459,22 @@ def run_gpu(args):
                                   "algorithmic_gb_per_step": n_layers * sum(algorithmic_bytes(cfg, m, lora=False)) / 1e9,
                                   "note": "adapters merged into the 2-bit codes and requantized; r = 0 at decode"}
         del merged, tmg, gmg
+        # the BF16/W2-GateUp configuration (Sec. 6.1): the same 2-bit gate/up and adapters, a dense bf16 down
+        bdl = [wq.MLPLayer(L.gate, L.up, wq.dense_weight(synth.weights((cfg.d, cfg.inter), 3 * l + 2, device=dev)
+                                                          .to(torch.bfloat16)),
+                           lora_a=L.lora_a, lora_b_gate=L.lora_b_gate, lora_b_up=L.lora_b_up, lora_scale=L.lora_scale)
+               for l, L in enumerate(layers)]
+        tbd = wq.LayerTable(bdl)
+        gbd = capture(lambda: wq.mlp_forward(x, bdl, prenorm=True, y=y, ws=ws, table=tbd))
+        msb, _ = time_graph(gbd, steps, warmup)
+        tpsb = m * steps / (msb / 1e3)
+        bd_gb = n_layers * (gu_bytes + cfg.d * cfg.inter * 2 + m * cfg.inter * 2 + 2 * m * cfg.d * 2) / 1e9
+        out["bf16_down_stack"] = {"tokens_per_s": tpsb, "ms_per_step": msb / steps, "vs_w4_down": tpsb / tps,
+                                  "algorithmic_gb_per_step": bd_gb,
+                                  "stack_gbs": bd_gb / (msb / steps / 1e3), "frac_of_hbm": bd_gb / (msb / steps / 1e3) / peak,
+                                  "note": "BF16/W2-GateUp: 2-bit gate/up with the adapters, dense bf16 down "
+                                          "(wq_mlp_forward with bits-16 down weights)"}
+        del bdl, tbd, gbd
         torch.cuda.empty_cache()
         out["prefill"] = run_prefill(wq, synth, dev, args.prefill_layers, max(20, min(steps, 200)), warmup)
         torch.cuda.empty_cache()

@@ -105,7 +105,10 @@ typedef struct {
  * with the unmerged LoRA terms a_g = lora_scale * (x A_g^T) B_g^T and a_u likewise
  * (Eq. 1; alpha of Eq. 1 is lora_scale, e.g. alpha/r in the PEFT convention). */
 typedef struct {
-    wq_qweight gate, up, down;   /* gate/up: n = inter, k = d.  down: n = d, k = inter */
+    wq_qweight gate, up, down;   /* gate/up: n = inter, k = d.  down: n = d, k = inter; in
+                                    wq_mlp_forward* the down may also be dense bf16 (the BF16/W2-GateUp
+                                    configuration, Sec. 6.1): bits = 16, codes = the bf16 [d, inter]
+                                    matrix (inter a multiple of 32), meta and group unused */
     const void *lora_a;          /* bf16 [2r, d]: rows 0..r-1 = A_gate, r..2r-1 = A_up; NULL if r == 0 */
     const void *lora_b_gate;     /* bf16 [inter, r] */
     const void *lora_b_up;       /* bf16 [inter, r] */

@@ -67,6 +67,18 @@ wq_status check_qweight(const wq_qweight *q, int bits, const char *name) {
   return WQ_OK;
 }
 
+// A stack layer's down matrix: 4-bit packed, or dense bf16 (bits 16: codes
+// holds the bf16 [n, k] matrix, k a multiple of 32; meta unused).
+wq_status check_down(const wq_qweight *q) {
+  if (q && q->bits == 16) {
+    if (!q->codes) return fail(WQ_ERR_ARG, "down: null bf16 matrix");
+    if (!aligned16(q->codes)) return fail(WQ_ERR_ALIGN, "down: bf16 matrix not 16-byte aligned");
+    if (q->n <= 0 || q->k <= 0 || q->k % 32 != 0) return fail(WQ_ERR_SHAPE, "down: bf16 shape [%d, %d] (k a multiple of 32)", q->n, q->k);
+    return WQ_OK;
+  }
+  return check_qweight(q, 4, "down");
+}
+
 // Byte layout of the workspace for up to m tokens of a (d, inter) layer.
 struct WsLayout {
   // arrival counters: at fixed offsets for every token count (zero once, kept
@@ -701,7 +713,7 @@ wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned 
     const int bits = Ly.gate.bits;
     if (bits != 2 && bits != 4) return fail(WQ_ERR_SHAPE, "layer %d: gate bits %d not in {2, 4}", l, bits);
     if ((st = check_gateup_pair(&Ly.gate, &Ly.up, bits)) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
-    if ((st = check_qweight(&Ly.down, 4, "down")) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    if ((st = check_down(&Ly.down)) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     if (bits == 4 && Ly.r != 0) return fail(WQ_ERR_UNSUPPORTED, "layer %d: LoRA on 4-bit gate/up is not supported", l);
     if ((st = check_lora(Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r)) != WQ_OK)
       return fail(st, "layer %d: %s", l, g_last_error.c_str());
@@ -745,7 +757,7 @@ bool stack_kernel_plan(int m, const wq_mlp_layer *layers, int n_layers, unsigned
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     if (Ly.gate.bits != L0.gate.bits || Ly.gate.group != L0.gate.group || Ly.down.group != L0.down.group ||
-        Ly.r != L0.r)
+        Ly.r != L0.r || Ly.down.bits != 4)
       return false;
   }
   if (!cooperative_ok()) return false;
@@ -770,7 +782,7 @@ StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned
     const wq_mlp_layer &Ly = layers[l];
     const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
     if (gateup_uses_gemm(Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4, m, &Ly.gate, Ly.r) ||
-        down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0))
+        (Ly.down.bits == 4 && down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0)))
       return kRouteGemmChain;
   }
   return kRouteGemvChain;
@@ -871,8 +883,13 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
       st = run_gateup_gemm(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale,
                            flags, layer_h(l), L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
-      st = run_down_gemm(layer_h(l), m, &Ly.down, cur, out, 0, L, w8, s);
-      if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+      if (Ly.down.bits == 16) {
+        cudaError_t e = launch_down_bf16(layer_h(l), m, Ly.down.codes, d, inter, cur, out, false, s);
+        if (e != cudaSuccess) return cuda_fail(e, "bf16 down launch");
+      } else {
+        st = run_down_gemm(layer_h(l), m, &Ly.down, cur, out, 0, L, w8, s);
+        if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+      }
       cur = out;
     }
     return finish();
@@ -887,6 +904,7 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     if (e != cudaSuccess) return cuda_fail(e, "tile-partials launch");
   }
   const void *cur = x;
+  bool tp_ready = true;  // the tile partials of cur are in tp (from tile_prep or the previous down launch)
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     void *out = layer_out(l);
@@ -894,15 +912,24 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
     const bool need_tp = prenorm || Ly.r > 0;
     const wq_mlp_layer *nx = l + 1 < n_layers ? &layers[l + 1] : nullptr;
-    const bool next_tp = nx && (prenorm || nx->r > 0);
+    const bool dense_down = Ly.down.bits == 16;
+    const bool next_tp = nx && (prenorm || nx->r > 0) && !dense_down;
     const int r_next = next_tp ? nx->r : 0;
-    const bool panel = chain_panel_ok(kind, m, Ly.gate, Ly.r, Ly.down, r_next);
+    const bool panel = !dense_down && chain_panel_ok(kind, m, Ly.gate, Ly.r, Ly.down, r_next);
+    // after a bf16 down (which writes no tile partials) the gate/up launch
+    // computes its input's partials itself
     st = run_gateup(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale, flags,
-                    hbuf, need_tp ? tp : nullptr, L, w8, s, panel);
+                    hbuf, need_tp && tp_ready ? tp : nullptr, L, w8, s, panel);
     if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
-    st = run_down(hbuf, m, &Ly.down, cur, out, 0, next_tp ? nx->lora_a : nullptr, r_next, next_tp ? tp : nullptr, L,
-                  w8, s, panel);
-    if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    if (dense_down) {
+      cudaError_t e = launch_down_bf16(hbuf, m, Ly.down.codes, d, inter, cur, out, false, s);
+      if (e != cudaSuccess) return cuda_fail(e, "bf16 down launch");
+    } else {
+      st = run_down(hbuf, m, &Ly.down, cur, out, 0, next_tp ? nx->lora_a : nullptr, r_next, next_tp ? tp : nullptr, L,
+                    w8, s, panel);
+      if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
+    }
+    tp_ready = next_tp;
     cur = out;
   }
   return finish();
@@ -945,12 +972,13 @@ wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, u
     const GemvKind kind = L0.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
     const bool next_tp = n_layers > 1 && ((flags & WQ_PRENORM) || layers[1].r > 0);
     const int r_next = next_tp ? layers[1].r : 0;
-    GemvPlan pg, pd;
+    GemvPlan pg, pd{};
     if (!plan_gemv(kind, L0.gate.n, L0.gate.k, m, L0.gate.group, L0.r, sms, &pg) ||
-        !plan_gemv(kDownW4, L0.down.n, L0.down.k, m, L0.down.group, r_next, sms, &pd))
+        (L0.down.bits == 4 && !plan_gemv(kDownW4, L0.down.n, L0.down.k, m, L0.down.group, r_next, sms, &pd)))
       return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits");
+    if (L0.down.bits == 16) pd.RB = pd.KP = pd.WK = pd.TPW = pd.P = pd.units = -1;  // the bf16 down kernel
     const int64_t v[13] = {pg.RB, pg.KP, pg.WK, pg.TPW, pg.P, pg.units, pd.RB, pd.KP, pd.WK, pd.TPW, pd.P, pd.units,
-                           chain_panel_ok(kind, m, L0.gate, L0.r, L0.down, r_next) ? 1 : 0};
+                           L0.down.bits == 4 && chain_panel_ok(kind, m, L0.gate, L0.r, L0.down, r_next) ? 1 : 0};
     for (int i = 0; i < 13; ++i) info[1 + i] = v[i];
   }
   return ok();

@@ -12,8 +12,10 @@
 //
 // The launch is programmatic-dependent: the first step's loads of Wd are issued
 // before griddepcontrol.wait (they do not depend on the previous kernel), h and
-// the residual only after it, and the next launch is let in once this one's
-// inputs are readable, so its weight stream overlaps this launch's tail.
+// the residual only after it, through L2 (ld.global.cg: a read-only-path load
+// could be moved above the wait and see h before the previous kernel wrote
+// it), and the next launch is let in once this one's inputs are readable, so
+// its weight stream overlaps this launch's tail.
 //
 // A CTA owns one tile of 16 output rows and 16 tokens; its 8 warps split the
 // input features into 8 contiguous ranges of 32-feature chunks and their fp32
@@ -40,8 +42,8 @@ __device__ __forceinline__ uint32_t u4word(const uint4 &v, int q) {
 // up to 8 tokens, 4 for 16: the register budget of 2 CTAs an SM)
 template <int NT, int U>
 __global__ void __launch_bounds__(kDnWarps * 32, 2)
-    down_bf16_kernel(const __nv_bfloat16 *__restrict__ h, int m, const __nv_bfloat16 *__restrict__ w, int d, int K,
-                     const __nv_bfloat16 *__restrict__ res, void *__restrict__ y, int y_f32) {
+    down_bf16_kernel(const __nv_bfloat16 *h, int m, const __nv_bfloat16 *__restrict__ w, int d, int K,
+                     const __nv_bfloat16 *res, void *__restrict__ y, int y_f32) {
   __shared__ float part[kDnWarps][16][17];  // [warp][row][token]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, g = lane >> 2, t = lane & 3;
   const int r0 = blockIdx.x * 16, m0 = blockIdx.y * 16;
@@ -80,7 +82,7 @@ __global__ void __launch_bounds__(kDnWarps * 32, 2)
       const int cc = c + u;
       const bool in = cc < c_hi;
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) vh[u][nt] = in && tin[nt] ? __ldg(hp[nt] + 4 * cc) : zero;
+      for (int nt = 0; nt < NT; ++nt) vh[u][nt] = in && tin[nt] ? ldg_cg128(hp[nt] + 4 * cc) : zero;
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -114,7 +116,7 @@ __global__ void __launch_bounds__(kDnWarps * 32, 2)
 #pragma unroll
     for (int wi = 0; wi < kDnWarps; ++wi) v += part[wi][rl][tl];
     const size_t at = (size_t)tok * d + row;
-    if (res != nullptr) v = __fadd_rn(__bfloat162float(res[at]), v);
+    if (res != nullptr) v = __fadd_rn(__bfloat162float(__ldcg(res + at)), v);
     if (y_f32)
       static_cast<float *>(y)[at] = v;
     else

@@ -131,6 +131,14 @@ class QWeight:
         return self.codes.numel() * 4 + self.meta.numel() * 2
 
 
+def dense_weight(w: torch.Tensor) -> QWeight:
+    """A dense bf16 [n, k] matrix as a down weight of wq_mlp_forward (bits 16;
+    the BF16/W2-GateUp configuration)."""
+    assert w.dtype == torch.bfloat16 and w.is_cuda and w.is_contiguous()
+    n, k = w.shape
+    return QWeight(w.view(torch.int16).view(-1), torch.zeros(8, dtype=torch.int16, device=w.device), n, k, 0, 16)
+
+
 def packed_sizes(bits: int, n: int, k: int, group: int):
     cb, mb = ctypes.c_size_t(), ctypes.c_size_t()
     _check(lib().wq_packed_sizes(bits, n, k, group, ctypes.byref(cb), ctypes.byref(mb)))
