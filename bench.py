@@ -480,6 +480,8 @@ def run_gpu(args):
         torch.cuda.empty_cache()
         out["decoder_layer"] = run_decoder(wq, synth, dev, max(10, min(steps, 50)), warmup)
         out["sweep"] = run_sweep(wq, synth, dev, max(10, min(steps, 50)), warmup, BENCH_SWEEP)["rows"]
+        torch.cuda.empty_cache()
+        out["moe"] = run_moe(wq, synth, dev, max(10, min(steps, 50)), warmup, peak)
         out["cpu_baseline"] = cpu_oracle_sample(cfg, m)
 
     if rank == 0:
@@ -658,6 +660,69 @@ def run_decoder(wq, synth, dev, steps, warmup, n_layers=None, contexts=DECODER_C
                     "standalone gate/up and down calls): uniform W4 (no adapter), W4/W2-GateUp with the unmerged "
                     "rank-16 adapter, and W4/W2-GateUp with the adapter merged into the 2-bit codes; gain_pct and "
                     "gain_pct_merged are the decode-rate gains of the last two over uniform W4"}
+
+
+# GPT-OSS-20B-shaped MoE MLP (Sec. 5's MoE model): hidden 2880, 32 experts of width 2880, top-4, 24 layers,
+# groups of 64 (the paper's INT4 g64 setting for this model)
+MOE_SHAPE = dict(d=2880, inter=2880, experts=32, top_k=4, layers=24, group=64, r=16, lora_scale=2.0)
+
+
+def run_moe(wq, synth, dev, steps, warmup, peak, shape=MOE_SHAPE, m=1):
+    """One decode step through a stack of MoE MLP blocks at W4/W2-GateUp (2-bit
+    gate/up experts with rank-16 adapters, 4-bit down) and at uniform W4: the
+    decode rate, the bytes the selected experts move per token, and the gain of
+    the 2-bit gate/up when routing leaves most experts unread."""
+    import torch
+    d, inter, E, k, L, g, r = (shape[key] for key in ("d", "inter", "experts", "top_k", "layers", "group", "r"))
+    x = synth.activations((m, d), 31, device=dev)
+    logits = [synth.weights((m, E), 8000 + l, std=1.0, device=dev) for l in range(L)]
+    out = {"workload": f"gpt_oss_20b_moe_{L}L_m{m}", "d": d, "expert_width": inter, "experts": E, "top_k": k,
+           "group": g, "lora_rank": r,
+           "routing": "fixed seeded N(0, 1) router logits per layer (top-4 of 32 experts)"}
+    for bits, name in ((2, "w4w2_gateup"), (4, "w4")):
+        blocks = []
+        for l in range(L):
+            wg = synth.weights((E * inter, d), 50_000 + 3 * l, device=dev)
+            wu = synth.weights((E * inter, d), 50_001 + 3 * l, device=dev)
+            wd = synth.weights((E * d, inter), 50_002 + 3 * l, device=dev)
+            kw = {}
+            if bits == 2:
+                _, bg, bu = synth.lora(d, E * inter, r, 60_000 + l, device=dev)
+                a = synth.weights((E * 2 * r, d), 61_000 + l, std=0.01, device=dev).to(torch.bfloat16)
+                kw = dict(lora_a=a, lora_b_gate=bg, lora_b_up=bu, lora_scale=shape["lora_scale"])
+            ex = wq.MLPLayer(wq.pack(wg, g, bits), wq.pack(wu, g, bits), wq.pack(wd, g, 4), **kw)
+            blocks.append(wq.MoELayer(ex, E, k))
+            del wg, wu, wd
+        cls = [b.c() for b in blocks]
+        ws = wq.moe_workspace(m, blocks[0])
+        bufs = [torch.empty_like(x) for _ in range(2)]
+
+        def step():
+            cur = x
+            for l in range(L):
+                o = bufs[l & 1]
+                wq.moe_forward(cur, logits[l], blocks[l], y=o, ws=ws, c_layer=cls[l])
+                cur = o
+
+        ms, _ = time_graph(capture(step), steps, warmup)
+        assert wq.device_status() == 0
+        t = ms / steps / 1e3
+        # bytes of one expert: packed gate, up, down, the adapter's rows; times the experts a token selects
+        ex0 = blocks[0].experts
+        per_expert = (ex0.gate.nbytes + ex0.up.nbytes + ex0.down.nbytes) / E
+        if bits == 2:
+            per_expert += (2 * r * d + 2 * inter * r) * 2
+        active = L * m * k * per_expert  # an upper bound when tokens share experts
+        out[name] = {"tokens_per_s": m / t, "us_per_layer": t * 1e6 / L, "active_gb_per_step": active / 1e9,
+                     "gbs": active / t / 1e9, "frac_of_hbm": active / t / 1e9 / peak,
+                     "all_experts_gb": L * per_expert * E / 1e9}
+        del blocks, cls, ws
+        torch.cuda.empty_cache()
+    out["gain_pct"] = 100.0 * (out["w4w2_gateup"]["tokens_per_s"] / out["w4"]["tokens_per_s"] - 1.0)
+    out["byte_ratio_w4_over_w4w2"] = out["w4"]["active_gb_per_step"] / out["w4w2_gateup"]["active_gb_per_step"]
+    out["note"] = ("wq_moe_forward per layer (routing + tile partials, gate/up and down over the selected "
+                   "experts' slots, combine): only the k selected experts' weights are read")
+    return out
 
 
 # --------------------------------------------------------------------------- reference arm

@@ -332,6 +332,46 @@ wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens
                                    size_t ws_bytes, void *stream);
 
 /*
+ * A mixture-of-experts MLP block (the MoE model of Sec. 5: a router picks a
+ * few experts per token, so a decode step reads only those experts' weights,
+ * which is how expert routing shrinks the realized gain of the 2-bit gate/up).
+ * Each expert is a gated MLP of wq_mlp_layer form; the E experts' matrices
+ * are stacked row-wise and packed as one matrix each:
+ *   experts.gate, experts.up: n = E * inter, k = d (expert e: rows e*inter ..
+ *                             e*inter + inter - 1); bits 2 (bits 4, r = 0: the
+ *                             uniform-W4 comparator);
+ *   experts.down:             bits 4, n = E * d, k = inter;
+ *   experts.lora_a:           bf16 [E][2r][d]; lora_b_gate, lora_b_up: bf16 [E * inter][r].
+ *   d and inter multiples of 16; 1 <= top_k <= min(E, 16); E <= 256.
+ */
+typedef struct {
+    wq_mlp_layer experts;
+    int32_t n_experts, top_k;
+} wq_moe_layer;
+
+/*
+ * One MoE block for m tokens (1 <= m <= 64; m == 0 is a no-op):
+ *   1. routing: per token t, the top_k experts by router logit, the larger
+ *      logit first and the lower expert index first among equal logits; their
+ *      weights w_j = softmax over the selected logits (fp32);
+ *   2. per slot (t, j): h = the gate/up of expert e_j on x[t] (the arithmetic
+ *      of wq_gateup_w2_lora, RMSNorm with WQ_PRENORM), y_j = h deq(Wd_e)^T (fp32);
+ *   3. y[t] = bf16(x[t] + sum_j w_j y_j), j in order (fp32).
+ *   x: bf16 [m, d].  logits: fp32 [m, E], finite.  y: bf16 [m, d].
+ *   expert_idx (int32 [m, top_k]), expert_w (fp32 [m, top_k]), h_slots
+ *   (bf16 [m top_k, inter]) and y_slots (fp32 [m top_k, d]): optional device
+ *   outputs of steps 1-2, slot t*top_k + j (NULL: kept in the workspace).
+ * Four launches on `stream` (routing with the tile partials, gate/up and down
+ * over the slots, combine); only the selected experts' weights are read.
+ * Workspace: wq_moe_workspace_bytes for this layer, token count and flags,
+ * zero-filled before first use (wq_workspace_init).
+ */
+size_t wq_moe_workspace_bytes(int m, const wq_moe_layer *layer, unsigned flags);
+wq_status wq_moe_forward(const void *x, int m, const float *logits, const wq_moe_layer *layer, unsigned flags,
+                         void *y, int32_t *expert_idx, float *expert_w, void *h_slots, float *y_slots, void *ws,
+                         size_t ws_bytes, void *stream);
+
+/*
  * wq_mlp_forward that also returns every layer's output (the hidden states of
  * the stack) and, optionally, every layer's MLP activation h:
  *   states:   bf16 [n_layers][m][d] (device, 16-byte aligned), states[l] = x_{l+1};

@@ -1100,6 +1100,169 @@ wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens
   return ok();
 }
 
+}  // extern "C"
+
+namespace {
+
+// Plans and workspace regions of a mixture-of-experts block for m tokens:
+// the slots' arrival counters first (zero between calls), then the routing
+// outputs, tile partials, h and the experts' fp32 outputs of every slot, then
+// the split-K partials.  Each slot's launches are planned as one token on
+// its share of the SMs (all slots of a launch run side by side).
+struct MoeWs {
+  GemvPlan gu, dn;
+  size_t cnt_gu, cnt_dn, idx, w, tp, h, ys, part_gu, part_dn, total;
+};
+
+bool moe_plan(GemvKind kind, int N, int K, int group, int r, int slots, GemvPlan *p) {
+  const int sms = num_sms();
+  if (sms <= 0) return false;
+  for (int share = std::max(1, sms / slots);; share = std::min(sms, share * 2)) {
+    if (plan_gemv(kind, N, K, 1, group, r, share, p)) return true;
+    if (share == sms) return false;
+  }
+}
+
+wq_status moe_check(int m, const wq_moe_layer *layer) {
+  if (!layer) return fail(WQ_ERR_ARG, "null MoE layer");
+  const wq_mlp_layer &X = layer->experts;
+  const int E = layer->n_experts, k = layer->top_k;
+  if (E < 1 || E > moe_max_experts()) return fail(WQ_ERR_SHAPE, "n_experts %d not in [1, %d]", E, moe_max_experts());
+  if (k < 1 || k > std::min(E, moe_max_top_k()))
+    return fail(WQ_ERR_SHAPE, "top_k %d not in [1, min(n_experts, %d)]", k, moe_max_top_k());
+  const int bits = X.gate.bits == 4 ? 4 : 2;
+  wq_status st;
+  if ((st = check_qweight(&X.gate, bits, "gate")) != WQ_OK || (st = check_qweight(&X.up, bits, "up")) != WQ_OK ||
+      (st = check_qweight(&X.down, 4, "down")) != WQ_OK)
+    return st;
+  const int d = X.gate.k;
+  if (X.gate.n % E != 0) return fail(WQ_ERR_SHAPE, "gate rows %d not a multiple of n_experts %d", X.gate.n, E);
+  const int inter = X.gate.n / E;
+  if (X.up.n != X.gate.n || X.up.k != d || X.up.group != X.gate.group || X.down.n != E * d || X.down.k != inter)
+    return fail(WQ_ERR_SHAPE, "expert shapes disagree (gate [%d x %d], up [%d x %d], down [%d x %d], %d experts)",
+                X.gate.n, X.gate.k, X.up.n, X.up.k, X.down.n, X.down.k, E);
+  if (d % 16 != 0 || inter % 16 != 0)
+    return fail(WQ_ERR_SHAPE, "d %d and the expert width %d must be multiples of 16", d, inter);
+  if (X.r < 0 || X.r > kMaxRank || X.r % 8 != 0) return fail(WQ_ERR_SHAPE, "LoRA rank %d", X.r);
+  if (X.r > 0) {
+    if (bits != 2) return fail(WQ_ERR_UNSUPPORTED, "adapters on 4-bit experts");
+    if (!X.lora_a || !X.lora_b_gate || !X.lora_b_up) return fail(WQ_ERR_ARG, "null LoRA factor");
+    if (!aligned16(X.lora_a) || !aligned16(X.lora_b_gate) || !aligned16(X.lora_b_up))
+      return fail(WQ_ERR_ALIGN, "LoRA factors not 16-byte aligned");
+  }
+  if (m < 0 || m > kMaxTokens) return fail(WQ_ERR_SHAPE, "m = %d tokens not in [0, %d]", m, kMaxTokens);
+  return WQ_OK;
+}
+
+bool moe_ws(int m, const wq_moe_layer &L, unsigned flags, MoeWs *W) {
+  const wq_mlp_layer &X = L.experts;
+  const int E = L.n_experts, S = m * L.top_k, d = X.gate.k, inter = X.gate.n / E, r = X.r;
+  const GemvKind kgu = X.gate.bits == 4 ? kGateUpW4 : kGateUpW2;
+  if (!moe_plan(kgu, inter, d, X.gate.group, r, S, &W->gu) || !moe_plan(kDownW4, d, inter, X.down.group, 0, S, &W->dn))
+    return false;
+  const bool need_tp = (flags & WQ_PRENORM) || r > 0;
+  size_t off = 0;
+  W->cnt_gu = off;  off = up256(off + (size_t)S * W->gu.RT * 4);
+  W->cnt_dn = off;  off = up256(off + (size_t)S * W->dn.RT * 4);
+  W->idx = off;     off = up256(off + (size_t)S * 4);
+  W->w = off;       off = up256(off + (size_t)S * 4);
+  W->tp = off;      off = up256(off + (need_tp ? (size_t)S * (d / 16) * WQ_TP_STRIDE(r) * 4 : 0));
+  W->h = off;       off = up256(off + (size_t)S * inter * 2);
+  W->ys = off;      off = up256(off + (size_t)S * d * 4);
+  W->part_gu = off; off = up256(off + (size_t)S * partial_bytes(W->gu, 2));
+  W->part_dn = off; off = up256(off + (size_t)S * partial_bytes(W->dn, 1));
+  W->total = off;
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t wq_moe_workspace_bytes(int m, const wq_moe_layer *layer, unsigned flags) {
+  if (m <= 0 || moe_check(m, layer) != WQ_OK) return 0;
+  MoeWs W;
+  return moe_ws(m, *layer, flags, &W) ? W.total : 0;
+}
+
+wq_status wq_moe_forward(const void *x, int m, const float *logits, const wq_moe_layer *layer, unsigned flags,
+                         void *y, int32_t *expert_idx, float *expert_w, void *h_slots, float *y_slots, void *ws,
+                         size_t ws_bytes, void *stream) {
+  wq_status st = moe_check(m, layer);
+  if (st != WQ_OK) return st;
+  if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
+  if (m == 0) return ok();
+  if (!x || !logits || !y) return fail(WQ_ERR_ARG, "null x, logits or y");
+  if (!aligned16(x) || !aligned16(logits) || !aligned16(y) || !aligned16(expert_idx) || !aligned16(expert_w) ||
+      !aligned16(h_slots) || !aligned16(y_slots))
+    return fail(WQ_ERR_ALIGN, "a device pointer is not 16-byte aligned");
+  const wq_moe_layer &L = *layer;
+  const wq_mlp_layer &X = L.experts;
+  MoeWs W;
+  if (!moe_ws(m, L, flags, &W)) return fail(WQ_ERR_UNSUPPORTED, "no launch configuration fits the experts");
+  if (!ws || ws_bytes < W.total) return fail(WQ_ERR_WORKSPACE, "MoE workspace of %zu bytes, %zu needed", ws_bytes, W.total);
+  uint8_t *w8 = static_cast<uint8_t *>(ws);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int E = L.n_experts, k = L.top_k, S = m * k, d = X.gate.k, inter = X.gate.n / E, r = X.r;
+  const bool need_tp = (flags & WQ_PRENORM) || r > 0;
+  int *idx = expert_idx ? expert_idx : reinterpret_cast<int *>(w8 + W.idx);
+  float *wt = expert_w ? expert_w : reinterpret_cast<float *>(w8 + W.w);
+  void *h = h_slots ? h_slots : static_cast<void *>(w8 + W.h);
+  float *ys = y_slots ? y_slots : reinterpret_cast<float *>(w8 + W.ys);
+  float *tp = need_tp ? reinterpret_cast<float *>(w8 + W.tp) : nullptr;
+
+  cudaError_t e = launch_moe_prep(x, m, d, logits, E, k, r > 0 ? X.lora_a : nullptr, 2 * r, tp, idx, wt, s);
+  if (e != cudaSuccess) return cuda_fail(e, "MoE routing launch");
+
+  GemvArgs a = {};
+  a.act = x;
+  a.M = 1;
+  a.K = d;
+  a.N = inter;
+  a.group = X.gate.group;
+  a.codes[0] = X.gate.codes;
+  a.codes[1] = X.up.codes;
+  a.meta[0] = X.gate.meta;
+  a.meta[1] = X.up.meta;
+  a.tp = tp;
+  a.ntp = d / 16;
+  a.prenorm = (flags & WQ_PRENORM) ? 1 : 0;
+  a.lora_b[0] = r > 0 ? X.lora_b_gate : nullptr;
+  a.lora_b[1] = r > 0 ? X.lora_b_up : nullptr;
+  a.r = r;
+  a.lora_scale = X.lora_scale;
+  a.out = h;
+  a.partials = reinterpret_cast<float *>(w8 + W.part_gu);
+  a.counters = reinterpret_cast<unsigned *>(w8 + W.cnt_gu);
+  a.slot_expert = idx;
+  a.n_experts = E;
+  a.slot_div = k;
+  e = launch_gemv_slots(X.gate.bits == 4 ? kGateUpW4 : kGateUpW2, W.gu, a, S, s, true);
+  if (e != cudaSuccess) return cuda_fail(e, "MoE gate/up launch");
+
+  GemvArgs b = {};
+  b.act = h;
+  b.M = 1;
+  b.K = inter;
+  b.N = d;
+  b.group = X.down.group;
+  b.codes[0] = X.down.codes;
+  b.meta[0] = X.down.meta;
+  b.out = ys;
+  b.out_f32 = 1;
+  b.partials = reinterpret_cast<float *>(w8 + W.part_dn);
+  b.counters = reinterpret_cast<unsigned *>(w8 + W.cnt_dn);
+  b.slot_expert = idx;
+  b.n_experts = E;
+  b.slot_div = 1;
+  e = launch_gemv_slots(kDownW4, W.dn, b, S, s, true);
+  if (e != cudaSuccess) return cuda_fail(e, "MoE down launch");
+
+  e = launch_moe_combine(x, m, d, k, wt, ys, y, s);
+  if (e != cudaSuccess) return cuda_fail(e, "MoE combine launch");
+  return ok();
+}
+
 wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t info[10]) {
   if (!info) return fail(WQ_ERR_ARG, "null info array");
   if (kind < 0 || kind > 2) return fail(WQ_ERR_ARG, "kind %d not in {0, 1, 2}", kind);

@@ -871,7 +871,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) gemm_prep_kernel(const __nv_b
     }
 #pragma unroll
     for (int u = 0; u < kPrepUnroll; ++u) {
-      const int c = cb + u * kPrepWarps, k = c * 32 + 8 * t;
+      const int c = cb + u * kPrepWarps;
       if (c >= nchunk) break;  // the same for the whole warp
 #pragma unroll
       for (int i = 0; i < 2; ++i) {

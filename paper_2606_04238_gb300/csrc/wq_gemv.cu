@@ -131,7 +131,7 @@ constexpr int kMaxThreads = 512;  // per CTA: up to 128 registers a thread
 //   NPROJ projections).
 // ---------------------------------------------------------------------------
 template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
-__global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1 ? 2 : 1) qgemv_kernel(const GemvArgs a, const GemvPlan p) {
+__device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p) {
   extern __shared__ __align__(128) uint8_t smem[];
   constexpr int BPK = BITS == 2 ? 512 : 1024;  // code bytes per (row tile, 128-feature block)
   constexpr int GPB = 128 / GROUP;             // groups per block
@@ -213,8 +213,9 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
       const int n = rt0 * 16 + rl;
       uint4 v = make_uint4(0u, 0u, 0u, 0u);
       const size_t src = ((size_t)n * r + (size_t)c * 8) * 2;
-      if (n < a.N && WQ_OK_IF(WQ_RANGE(src, 16, a.nb_lora_b[pj], 16), 30, n))
-        v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(a.lora_b[pj]) + src));
+      const void *lb = pj == 0 ? a.lora_b[0] : a.lora_b[NPROJ - 1];  // no dynamic index into the arguments
+      if (n < a.N && WQ_OK_IF(WQ_RANGE(src, 16, pj == 0 ? a.nb_lora_b[0] : a.nb_lora_b[NPROJ - 1], 16), 30, n))
+        v = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const uint8_t *>(lb) + src));
       const size_t dst = p.off_lorab + (((size_t)pj * p.RB * 16 + rl) * r + (size_t)c * 8) * 2;
       if (WQ_OK_IF(WQ_RANGE(dst, 16, p.off_an, 16), 31, i)) *reinterpret_cast<uint4 *>(smem + dst) = v;
     }
@@ -879,6 +880,67 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
   }
 }
 
+template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
+__global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1 ? 2 : 1)
+    qgemv_kernel(const GemvArgs a, const GemvPlan p) {
+  qgemv_body<BITS, NPROJ, GROUP, NT, TPW>(a, p);
+}
+
+// ---------------------------------------------------------------------------
+// The same kernel over the routed experts of a mixture-of-experts block
+// (Sec. 5's MoE model reads only the experts a token selects).  grid.y runs
+// over slots (token t, choice j) -> slot t*top_k + j, one token each; the
+// experts' matrices are stacked row-wise ([E*N, K] packed as one matrix, so
+// expert e owns row tiles e*RT .. e*RT+RT-1) and slot s computes with expert
+// e = slot_expert[s], written by the routing kernel of the same step.  The
+// expert is known only after the previous launch, so the wait comes first
+// and the weight stream follows it.  Per slot: input row s / slot_div of act,
+// tile partials and panel partials / counters of its own, output row s.
+// ---------------------------------------------------------------------------
+template <int BITS, int NPROJ, int GROUP, int TPW>
+__global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && TPW == 1 ? 2 : 1)
+    qgemv_slots_kernel(const GemvArgs a0, const GemvPlan p) {
+  pdl_wait();  // slot_expert and the activations come from the previous launches
+  const int slot = blockIdx.y;
+  const int e = __ldcg(a0.slot_expert + slot);
+  if (e < 0 || e >= a0.n_experts) {
+    if (threadIdx.x == 0) atomicExch(&g_device_status, -1);  // WQ_ERR_ARG: an expert index outside [0, E)
+    return;
+  }
+  constexpr int WPB = BITS == 2 ? 128 : 256;  // code words per (row tile, 128-feature block)
+  const size_t rt = (size_t)p.RT, ng = (size_t)p.KB * (128 / GROUP);
+  const int Qp = WQ_TP_STRIDE(a0.r);
+  GemvArgs a = a0;
+#pragma unroll
+  for (int pj = 0; pj < NPROJ; ++pj) {
+    a.codes[pj] = a0.codes[pj] + (size_t)e * rt * p.KB * WPB;
+    a.meta[pj] = a0.meta[pj] + (size_t)e * rt * ng * 32;
+    a.nb_codes[pj] = rt * p.KB * WPB * 4;
+    a.nb_meta[pj] = rt * ng * 64;
+    if (NPROJ == 2 && a0.r > 0) {
+      a.lora_b[pj] = reinterpret_cast<const uint8_t *>(a0.lora_b[pj]) + (size_t)e * a0.N * a0.r * 2;
+      a.nb_lora_b[pj] = (size_t)a0.N * a0.r * 2;
+    }
+  }
+  a.act = reinterpret_cast<const uint8_t *>(a0.act) + (size_t)(slot / a0.slot_div) * a0.K * 2;
+  a.nb_act = (size_t)a0.K * 2;
+  if (a0.tp != nullptr) {
+    a.tp = a0.tp + (size_t)slot * a0.ntp * Qp;
+    a.nb_tp = (size_t)a0.ntp * Qp * 4;
+  }
+  const size_t osz = a0.out_f32 ? 4 : 2;
+  a.out = reinterpret_cast<uint8_t *>(a0.out) + (size_t)slot * a0.N * osz;
+  a.nb_out = (size_t)a0.N * osz;
+  if (p.P > 1) {
+    const size_t per = rt * p.P * NPROJ * 16;
+    a.partials = a0.partials + (size_t)slot * per;
+    a.counters = a0.counters + (size_t)slot * rt;
+    a.nb_part = per * 4;
+    a.nb_cnt = rt * 4;
+  }
+  qgemv_body<BITS, NPROJ, GROUP, 1, TPW>(a, p);
+}
+
 // ---------------------------------------------------------------------------
 // Tile partials of an input x [M, d] (d a multiple of 16), one warp per tile
 // of 16 features: tp[tile][m][0] = sum_c x_c^2, tp[tile][m][1 + j] =
@@ -1118,6 +1180,36 @@ cudaError_t launch_t(const GemvPlan &p, const GemvArgs &a, cudaStream_t s, bool 
   return cudaLaunchKernelEx(&cfg, kern, a, p);
 }
 
+template <int BITS, int NPROJ, int GROUP, int TPW>
+cudaError_t launch_slots_t(const GemvPlan &p, const GemvArgs &a, int slots, cudaStream_t s, bool pdl) {
+  auto kern = qgemv_slots_kernel<BITS, NPROJ, GROUP, TPW>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.units, slots);
+  cfg.blockDim = dim3(p.threads);
+  cfg.dynamicSmemBytes = p.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, a, p);
+}
+
+template <int BITS, int NPROJ>
+cudaError_t launch_slots_g(const GemvPlan &p, const GemvArgs &a, int slots, cudaStream_t s, bool pdl) {
+  if (p.NT != 1 || p.M != 1) return cudaErrorInvalidValue;
+  const bool t2 = p.TPW == 2;
+  switch (a.group) {
+    case 32: return t2 ? launch_slots_t<BITS, NPROJ, 32, 2>(p, a, slots, s, pdl) : launch_slots_t<BITS, NPROJ, 32, 1>(p, a, slots, s, pdl);
+    case 64: return t2 ? launch_slots_t<BITS, NPROJ, 64, 2>(p, a, slots, s, pdl) : launch_slots_t<BITS, NPROJ, 64, 1>(p, a, slots, s, pdl);
+    case 128: return t2 ? launch_slots_t<BITS, NPROJ, 128, 2>(p, a, slots, s, pdl) : launch_slots_t<BITS, NPROJ, 128, 1>(p, a, slots, s, pdl);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 template <int BITS, int NPROJ, int GROUP>
 const void *kernel_ptr(int NT, int TPW) {
   if (NT == 2) return reinterpret_cast<const void *>(qgemv_kernel<BITS, NPROJ, GROUP, 2, 1>);
@@ -1175,6 +1267,17 @@ cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &arg
     case kGateUpW2: return launch_g<2, 2>(plan, args, stream, pdl);
     case kGateUpW4: return launch_g<4, 2>(plan, args, stream, pdl);
     case kDownW4: return launch_g<4, 1>(plan, args, stream, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemv_slots(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, int slots,
+                              cudaStream_t stream, bool pdl) {
+  if (plan.r != args.r || args.slot_expert == nullptr || slots <= 0 || slots > 65535) return cudaErrorInvalidValue;
+  switch (kind) {
+    case kGateUpW2: return launch_slots_g<2, 2>(plan, args, slots, stream, pdl);
+    case kGateUpW4: return launch_slots_g<4, 2>(plan, args, slots, stream, pdl);
+    case kDownW4: return launch_slots_g<4, 1>(plan, args, slots, stream, pdl);
   }
   return cudaErrorInvalidValue;
 }

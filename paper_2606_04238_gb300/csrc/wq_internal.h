@@ -81,6 +81,12 @@ struct GemvArgs {
   int pre_stride;
   float *partials;           // [RT][P][NPROJ][16][M] fp32 (P > 1)
   unsigned *counters;        // [RT] arrival counters, zero between calls
+  // Routed experts (launch_gemv_slots only): slot s = blockIdx.y runs the
+  // matrix of expert slot_expert[s] (rows e*N .. e*N+N-1 of the stacked
+  // codes, meta and LoRA-B) on input row s / slot_div of act, writing output
+  // row s; tp, partials and counters hold one region per slot.
+  const int *slot_expert;    // [slots], written by the routing kernel
+  int n_experts, slot_div;
   // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
   size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_tp, nb_res, nb_out, nb_an, nb_tp_out, nb_part, nb_cnt;
   size_t nb_hq, nb_hsc, nb_hxs, nb_pre_x, nb_pre_sc, nb_pre_xs;
@@ -138,6 +144,11 @@ int kernel_regs(GemvKind kind, int group, int NT, int TPW);
 // Launches the dequant-GEMV kernel of `kind` (programmatic dependent launch
 // when `pdl`).  Returns the CUDA error of the launch.
 cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, cudaStream_t stream, bool pdl);
+
+// The same kernels over `slots` routed-expert slots (grid.y; one token each,
+// plan made for M = 1 and one expert's N rows).  Needs args.slot_expert.
+cudaError_t launch_gemv_slots(GemvKind kind, const GemvPlan &plan, const GemvArgs &args, int slots,
+                              cudaStream_t stream, bool pdl);
 
 // Launches the tile-partials kernel of an input x [M, d] (d a multiple of
 // 16): tp[tile][m][0] = sum x^2, tp[tile][m][1 + j] = A[j] . x over the

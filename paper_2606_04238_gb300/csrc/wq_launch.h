@@ -31,4 +31,17 @@ int attn_splits(int B, int Hkv, int max_len, int num_sms);
 // Reads and clears the attention kernels' device status word.
 cudaError_t read_attn_status(int *status);
 
+// Mixture-of-experts steps (wq_moe.cu).  Routing and tile partials: per
+// token t of x bf16 [m][d], the top_k of the E fp32 logits [m][E] (larger
+// first, lower index among equal ones) -> idx [m*top_k] and softmax weights
+// w [m*top_k]; with tp non-null, per slot s = t*top_k + j the tile partials
+// of x[t] for expert idx[s] (sum x^2 and the r2 rows of lora_a + idx[s]*r2*d)
+// at tp + s*(d/16)*stride.  Combine: y[t] = bf16(x[t] + sum_j w ys[t*top_k + j]).
+cudaError_t launch_moe_prep(const void *x, int m, int d, const float *logits, int E, int top_k, const void *lora_a,
+                            int r2, float *tp, int *idx, float *w, cudaStream_t s);
+cudaError_t launch_moe_combine(const void *x, int m, int d, int top_k, const float *w, const float *ys, void *y,
+                               cudaStream_t s);
+int moe_max_experts();
+int moe_max_top_k();
+
 }  // namespace wq

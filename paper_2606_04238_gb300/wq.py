@@ -48,6 +48,10 @@ class _DecoderLayer(ctypes.Structure):
                 ("n_kv", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("rope_theta", ctypes.c_float)]
 
 
+class _MoELayer(ctypes.Structure):
+    _fields_ = [("experts", _MLPLayer), ("n_experts", ctypes.c_int32), ("top_k", ctypes.c_int32)]
+
+
 _lib = None
 
 
@@ -87,6 +91,8 @@ def lib():
             "wq_attn_decode": (I, [P, P, P, I, I, I, I, I, F, P, P, I, P, P, S, P]),
             "wq_decoder_workspace_bytes": (S, [I, ctypes.POINTER(_DecoderLayer), I]),
             "wq_decoder_layer_forward": (I, [P, I, P, ctypes.POINTER(_DecoderLayer), P, P, I, U, P, P, S, P]),
+            "wq_moe_workspace_bytes": (S, [I, ctypes.POINTER(_MoELayer), U]),
+            "wq_moe_forward": (I, [P, I, P, ctypes.POINTER(_MoELayer), U, P, P, P, P, P, P, S, P]),
             "wq_last_error": (ctypes.c_char_p, []),
             "wq_device_status": (I, [ctypes.POINTER(I)]),
             "wq_version": (ctypes.c_char_p, []),
@@ -461,6 +467,52 @@ def decoder_layer_forward(x, lens, layer: DecoderLayer, k_cache, v_cache, prenor
                                           max_len, WQ_PRENORM if prenorm else 0, _ptr(y), _ptr(ws), ws.numel(),
                                           _stream()))
     return y
+
+
+@dataclass
+class MoELayer:
+    """A mixture-of-experts block: the experts' matrices stacked row-wise in one
+    MLPLayer (gate/up [E*inter, d], down [E*d, inter], lora_a [E*2r, d],
+    lora_b_* [E*inter, r]), n_experts experts, top_k of them per token."""
+    experts: MLPLayer
+    n_experts: int
+    top_k: int
+
+    def c(self) -> _MoELayer:
+        return _MoELayer(self.experts.c(), self.n_experts, self.top_k)
+
+
+def moe_workspace(m: int, layer: MoELayer, prenorm: bool = True, device="cuda") -> torch.Tensor:
+    cl = layer.c()
+    nb = int(lib().wq_moe_workspace_bytes(m, ctypes.byref(cl), WQ_PRENORM if prenorm else 0))
+    if nb == 0:
+        raise WQError(-2, "no MoE workspace for these sizes")
+    ws = torch.empty(nb, dtype=torch.uint8, device=device)
+    _check(lib().wq_workspace_init(_ptr(ws), nb, _stream()))
+    return ws
+
+
+def moe_forward(x, logits, layer: MoELayer, prenorm: bool = True, y=None, ws=None, with_slots: bool = False,
+                c_layer=None):
+    """wq_moe_forward for x bf16 [m, d] and router logits fp32 [m, E].  Returns y,
+    or with with_slots (y, expert_idx [m, k], expert_w [m, k], h [m*k, inter], y_slots [m*k, d])."""
+    m, d = x.shape
+    k = layer.top_k
+    inter = layer.experts.gate.n // layer.n_experts
+    if y is None:
+        y = torch.empty_like(x)
+    if ws is None:
+        ws = moe_workspace(m, layer, prenorm, device=x.device)
+    idx = wt = hs = ys = None
+    if with_slots:
+        idx = torch.empty((m, k), dtype=torch.int32, device=x.device)
+        wt = torch.empty((m, k), dtype=torch.float32, device=x.device)
+        hs = torch.empty((m * k, inter), dtype=torch.bfloat16, device=x.device)
+        ys = torch.empty((m * k, d), dtype=torch.float32, device=x.device)
+    cl = c_layer if c_layer is not None else layer.c()
+    _check(lib().wq_moe_forward(_ptr(x), m, _ptr(logits), ctypes.byref(cl), WQ_PRENORM if prenorm else 0, _ptr(y),
+                                _ptr(idx), _ptr(wt), _ptr(hs), _ptr(ys), _ptr(ws), ws.numel(), _stream()))
+    return (y, idx, wt, hs, ys) if with_slots else y
 
 
 def device_status() -> int:
