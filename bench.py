@@ -233,7 +233,7 @@ def build_stack(wq, synth, cfg, n_layers, bits_gu, lora, dev):
     for l in range(n_layers):
         wg, wu, wd = synth.layer_weights(cfg, l, device=dev)
         kw = {}
-        if lora and bits_gu == 2:
+        if lora and bits_gu in (2, 3):
             a, bg, bu = synth.lora(cfg.d, cfg.inter, cfg.r, 10_000 + l, device=dev)
             kw = dict(lora_a=a, lora_b_gate=bg, lora_b_up=bu, lora_scale=cfg.lora_scale)
         layers.append(wq.MLPLayer(wq.pack(wg, cfg.group_gu, bits_gu), wq.pack(wu, cfg.group_gu, bits_gu),
@@ -476,6 +476,8 @@ def run_gpu(args):
                                           "(wq_mlp_forward with bits-16 down weights)"}
         del bdl, tbd, gbd
         torch.cuda.empty_cache()
+        out["quant_settings"] = run_quant_settings(wq, synth, dev, cfg, n_layers, m, x, y, ws, steps, warmup, peak)
+        torch.cuda.empty_cache()
         out["prefill"] = run_prefill(wq, synth, dev, args.prefill_layers, max(20, min(steps, 200)), warmup)
         torch.cuda.empty_cache()
         out["decoder_layer"] = run_decoder(wq, synth, dev, max(10, min(steps, 50)), warmup)
@@ -660,6 +662,38 @@ def run_decoder(wq, synth, dev, steps, warmup, n_layers=None, contexts=DECODER_C
                     "standalone gate/up and down calls): uniform W4 (no adapter), W4/W2-GateUp with the unmerged "
                     "rank-16 adapter, and W4/W2-GateUp with the adapter merged into the 2-bit codes; gain_pct and "
                     "gain_pct_merged are the decode-rate gains of the last two over uniform W4"}
+
+
+# gate/up quantization settings of the same stack: the headline W2 g128, the paper's W2 g32 (Sec. 4.1; its
+# scales and zeros cost 1 bit a weight), App. B's W3 g32, and the uniform W4 g128 comparator
+QUANT_SETTINGS = ((2, 128, True), (2, 32, True), (3, 32, True), (4, 128, False))
+
+
+def run_quant_settings(wq, synth, dev, cfg, n_layers, m, x, y, ws, steps, warmup, peak):
+    """The decode stack (same workload, 4-bit g128 down) with each gate/up setting: rate, bytes a step and the
+    fraction of HBM bandwidth those bytes take at that rate."""
+    import dataclasses
+
+    import torch
+    rows = []
+    for bits, g, lora in QUANT_SETTINGS:
+        c2 = dataclasses.replace(cfg, group_gu=g)
+        layers = build_stack(wq, synth, c2, n_layers, bits, lora, dev)
+        table = wq.LayerTable(layers)
+        gr = capture(lambda: wq.mlp_forward(x, layers, prenorm=True, y=y, ws=ws, table=table))
+        ms, _ = time_graph(gr, steps, warmup)
+        assert wq.device_status() == 0
+        gu, dn = algorithmic_bytes(c2, m, bits, lora)
+        t = ms / steps / 1e3
+        gb = n_layers * (gu + dn) / 1e9
+        rows.append({"gate_up": f"W{bits} g{g}" + (" + LoRA r" + str(cfg.r) if lora else ""),
+                     "tokens_per_s": m / t, "us_per_layer": t * 1e6 / n_layers, "gb_per_step": gb,
+                     "frac_of_hbm": gb / t / peak,
+                     "route": ("launch chain", "dequant-GEMM chain", "single-launch stack kernel")[
+                         wq.mlp_forward_info(m, layers, table=table)["route"]]})
+        del layers, table, gr
+        torch.cuda.empty_cache()
+    return {"workload": f"{cfg.name}_stack_{n_layers}L_m{m}", "down": f"W4 g{cfg.group_down}", "rows": rows}
 
 
 # GPT-OSS-20B-shaped MoE MLP (Sec. 5's MoE model): hidden 2880, 32 experts of width 2880, top-4, 24 layers,

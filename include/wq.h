@@ -78,16 +78,21 @@ typedef enum {
  *   feature blocks, NG = KB*128/group groups per row.
  *
  *   codes: uint32 words; block (rt, kb) of 16 rows x 128 features starts at
- *   word (rt*KB + kb) * WPB, WPB = 128 (bits 2) or 256 (bits 4).  The code of
- *   local row i and local feature c sits at
+ *   word (rt*KB + kb) * WPB, WPB = 128 (bits 2), 192 (bits 3) or 256 (bits 4).
+ *   The code of local row i and local feature c sits at
  *       lane = (i%8)*4 + (c%8)/2,  half = c%2
  *       bits 2: word = lane*4 + c/32,
  *               bit  = 16*half + 8*(i/8) + 2*(2*((c%32)/16) + (c%16)/8)
  *       bits 4: word = (c/64)*128 + lane*4 + (c%64)/16,
  *               bit  = 16*half + 8*(i/8) + 4*((c%16)/8)
- *   so that one 16-byte load per lane yields that lane's m16n8k16 tensor-core
- *   A fragments for a whole 128-feature block (64 codes of 2 bits) or a
- *   64-feature half block (32 codes of 4 bits).
+ *       bits 3 (App. B's INT3 gate/up), two bit planes: code % 4 in words
+ *               0..127 exactly where a 2-bit code sits, and code / 4 at
+ *               word = 128 + lane*2 + (c/32)/2,
+ *               bit  = 16*half + 8*((c/32)%2) + 2*(2*((c%32)/16) + (c%16)/8) + i/8
+ *   so that one 16-byte load per lane (plus 8 bytes of the second plane for
+ *   3 bits) yields that lane's m16n8k16 tensor-core A fragments for a whole
+ *   128-feature block (64 codes of 2 or 3 bits) or a 64-feature half block
+ *   (32 codes of 4 bits).
  *
  *   meta: binary16 scale s and zero z per (row, group): 32 values per
  *   (rt, group j) at (rt*NG + j)*32, for e = 0..7:
@@ -122,7 +127,8 @@ wq_status wq_packed_sizes(int bits, int n, int k, int group, size_t *code_bytes,
 
 /*
  * Stage-1 quantization and packing (Sec. 4.1 selective INT2 quantization of
- * gate/up; INT4 for the remaining layers, Sec. 3.3 and Sec. 7 step 4).
+ * gate/up; INT4 for the remaining layers, Sec. 3.3 and Sec. 7 step 4; INT3
+ * for App. B's W3-GateUp variant): bits 2, 3 or 4.
  * Asymmetric min-max round-to-nearest per group of `group` consecutive input
  * features of each row, in IEEE fp32:
  *     s = fp16((max - min) / qmax)  (1.0 if that is zero),
@@ -234,6 +240,17 @@ wq_status wq_gateup_w2_lora_noalloc(const void *x, int m, const wq_qweight *gate
                                     const void *lora_a, const void *lora_b_gate, const void *lora_b_up,
                                     int r, float lora_scale, unsigned flags, void *h, void *stream);
 
+/*
+ * App. B's W3-GateUp variant: wq_gateup_w2_lora with 3-bit gate/up codes
+ * (bits 3, two bit planes; same arguments, same arithmetic).  Runs on the
+ * dequant-GEMV kernels at every token count up to 64 (WQ_ERR_UNSUPPORTED
+ * above: the dequant-GEMM path takes 2- and 4-bit codes).
+ */
+wq_status wq_gateup_w3_lora(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
+                            const void *lora_a, const void *lora_b_gate, const void *lora_b_up,
+                            int r, float lora_scale, unsigned flags, void *h,
+                            void *ws, size_t ws_bytes, void *stream);
+
 /* The uniform-W4 comparator: the same block with 4-bit gate/up and no LoRA. */
 wq_status wq_gateup_w4(const void *x, int m, const wq_qweight *gate, const wq_qweight *up,
                        unsigned flags, void *h, void *ws, size_t ws_bytes, void *stream);
@@ -265,8 +282,10 @@ wq_status wq_down_bf16(const void *h, int m, const void *wd, int d, int inter, c
  * A stack of gated-MLP layers for one decode step of m tokens:
  *     x_0 = x,  x_{l+1} = x_l + down_l( SiLU(gate_l(xin_l)) * up_l(xin_l) ),  y = x_L
  * with xin_l = RMSNorm(x_l) (unrounded, as in wq_gateup_w2_lora) when flags has
- * WQ_PRENORM, else x_l.  Each layer's gate/up are 2-bit (with LoRA) or 4-bit
- * (no LoRA); down is 4-bit.  x, y: bf16 [m, d]; the residual stream is stored
+ * WQ_PRENORM, else x_l.  Each layer's gate/up are 2-bit or 3-bit (App. B; with
+ * LoRA) or 4-bit (no LoRA); down is 4-bit (or dense bf16, see wq_mlp_layer).
+ * Stacks with 3-bit gate/up take the launch chain at every token count up to
+ * 64 (above: WQ_ERR_UNSUPPORTED).  x, y: bf16 [m, d]; the residual stream is stored
  * in bf16 between layers.  Three routes, chosen per call (wq_mlp_forward_info
  * reports which):
  *   - the single-launch stack kernel: every layer in one cooperative launch

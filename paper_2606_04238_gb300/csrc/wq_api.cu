@@ -122,6 +122,7 @@ bool max_partials(int m, int d, int inter, size_t *p1, size_t *p2, bool *all_fit
       if (d % g == 0) {
         if (plan_gemv(kGateUpW2, inter, d, m, g, r, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
         else fit = false;
+        if (plan_gemv(kGateUpW3, inter, d, m, g, r, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
         if (r == 0) {
           if (plan_gemv(kGateUpW4, inter, d, m, g, 0, sms, &pl)) *p1 = std::max(*p1, partial_bytes(pl, 2));
           else fit = false;
@@ -223,6 +224,7 @@ bool ws_layout(int m, int d, int inter, WsLayout *L, bool gemv_only = false) {
 // work grows faster than linearly with the token count), or where the GEMV
 // path has no launch plan.  The workspace holds the GEMM buffers then.
 bool gateup_uses_gemm(GemvKind kind, int m, const wq_qweight *gate, int r) {
+  if (kind == kGateUpW3) return false;  // the dequant-GEMM path takes 2- and 4-bit codes only
   if (m > gemv_prefer_tokens(gate->k)) return true;
   GemvPlan pl;
   return !plan_gemv(kind, gate->n, gate->k, m, gate->group, r, num_sms(), &pl);
@@ -467,7 +469,10 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
                        void *h, void *ws, size_t ws_bytes, void *stream) {
   wq_status st = check_tokens(m);
   if (st != WQ_OK) return st;
-  if ((st = check_gateup_pair(gate, up, kind == kGateUpW2 ? 2 : 4)) != WQ_OK) return st;
+  if ((st = check_gateup_pair(gate, up, kind == kGateUpW2 ? 2 : kind == kGateUpW3 ? 3 : 4)) != WQ_OK) return st;
+  if (kind == kGateUpW3 && m > kMaxTokens)
+    return fail(WQ_ERR_UNSUPPORTED, "3-bit gate/up above %d tokens (the dequant-GEMM path takes 2- and 4-bit codes)",
+                kMaxTokens);
   if ((st = check_lora(lora_a, bg, bu, r)) != WQ_OK) return st;
   if (flags & ~WQ_PRENORM) return fail(WQ_ERR_ARG, "unknown flags 0x%x", flags);
   if (m == 0) return ok();
@@ -489,11 +494,11 @@ wq_status gateup_entry(GemvKind kind, const void *x, int m, const wq_qweight *ga
 extern "C" {
 
 wq_status wq_packed_sizes(int bits, int n, int k, int group, size_t *code_bytes, size_t *meta_bytes) {
-  if (bits != 2 && bits != 4) return fail(WQ_ERR_SHAPE, "bits %d not in {2, 4}", bits);
+  if (bits < 2 || bits > 4) return fail(WQ_ERR_SHAPE, "bits %d not in {2, 3, 4}", bits);
   if (!group_ok(group)) return fail(WQ_ERR_SHAPE, "group %d not in {32, 64, 128}", group);
   if (n < 0 || k < 0 || k % group != 0) return fail(WQ_ERR_SHAPE, "bad shape [%d, %d] for group %d", n, k, group);
   const size_t RT = (size_t)(n + 15) / 16, KB = (size_t)(k + 127) / 128;
-  if (code_bytes) *code_bytes = RT * KB * (bits == 2 ? 512 : 1024);
+  if (code_bytes) *code_bytes = RT * KB * 256 * bits;
   if (meta_bytes) *meta_bytes = RT * (KB * 128 / group) * 64;
   return ok();
 }
@@ -527,7 +532,7 @@ wq_status wq_pack_w4(const float *w, int n, int k, int group, wq_qweight *out, i
 wq_status wq_merge_lora(const wq_qweight *src, const void *lora_b, const void *lora_a, int r, float lora_scale,
                         float *w_merged, wq_qweight *out, int *nonfinite, void *stream) {
   if (!src) return fail(WQ_ERR_ARG, "src: null wq_qweight");
-  if (src->bits != 2 && src->bits != 4) return fail(WQ_ERR_SHAPE, "src: bits %d not in {2, 4}", src->bits);
+  if (src->bits < 2 || src->bits > 4) return fail(WQ_ERR_SHAPE, "src: bits %d not in {2, 3, 4}", src->bits);
   wq_status st = check_qweight(src, src->bits, "src");
   if (st != WQ_OK) return st;
   if (r < 0 || r > kMaxRank) return fail(WQ_ERR_SHAPE, "LoRA rank %d not in [0, %d]", r, kMaxRank);
@@ -582,6 +587,13 @@ wq_status wq_gateup_w2_lora(const void *x, int m, const wq_qweight *gate, const 
                             const void *lora_b_gate, const void *lora_b_up, int r, float lora_scale, unsigned flags,
                             void *h, void *ws, size_t ws_bytes, void *stream) {
   return gateup_entry(kGateUpW2, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, ws, ws_bytes,
+                      stream);
+}
+
+wq_status wq_gateup_w3_lora(const void *x, int m, const wq_qweight *gate, const wq_qweight *up, const void *lora_a,
+                            const void *lora_b_gate, const void *lora_b_up, int r, float lora_scale, unsigned flags,
+                            void *h, void *ws, size_t ws_bytes, void *stream) {
+  return gateup_entry(kGateUpW3, x, m, gate, up, lora_a, lora_b_gate, lora_b_up, r, lora_scale, flags, h, ws, ws_bytes,
                       stream);
 }
 
@@ -711,7 +723,10 @@ wq_status check_stack(int m, const wq_mlp_layer *layers, int n_layers, unsigned 
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     const int bits = Ly.gate.bits;
-    if (bits != 2 && bits != 4) return fail(WQ_ERR_SHAPE, "layer %d: gate bits %d not in {2, 4}", l, bits);
+    if (bits < 2 || bits > 4) return fail(WQ_ERR_SHAPE, "layer %d: gate bits %d not in {2, 3, 4}", l, bits);
+    if (bits == 3 && m > kMaxTokens)
+      return fail(WQ_ERR_UNSUPPORTED, "layer %d: 3-bit gate/up above %d tokens (the dequant-GEMM path takes 2- and "
+                  "4-bit codes)", l, kMaxTokens);
     if ((st = check_gateup_pair(&Ly.gate, &Ly.up, bits)) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     if ((st = check_down(&Ly.down)) != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
     if (bits == 4 && Ly.r != 0) return fail(WQ_ERR_UNSUPPORTED, "layer %d: LoRA on 4-bit gate/up is not supported", l);
@@ -777,11 +792,13 @@ StackRoute stack_route(int m, const wq_mlp_layer *layers, int n_layers, unsigned
   StackPlan sp;
   if (((flags & WQ_LAUNCH_STACK) || stack_preferred(m, layers[0])) && stack_kernel_plan(m, layers, n_layers, flags, &sp))
     return kRouteStack;
+  for (int l = 0; l < n_layers; ++l)
+    if (layers[l].gate.bits == 3) return kRouteGemvChain;  // 3-bit codes run on the GEMV kernels only
   if (m > gemv_prefer_tokens(layers[0].gate.k)) return kRouteGemmChain;
   for (int l = 0; l < n_layers; ++l) {
     const wq_mlp_layer &Ly = layers[l];
     const bool next_tp = l + 1 < n_layers && ((flags & WQ_PRENORM) || layers[l + 1].r > 0);
-    if (gateup_uses_gemm(Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4, m, &Ly.gate, Ly.r) ||
+    if (gateup_uses_gemm(gateup_kind(Ly.gate.bits), m, &Ly.gate, Ly.r) ||
         (Ly.down.bits == 4 && down_uses_gemm(m, &Ly.down, next_tp ? layers[l + 1].r : 0)))
       return kRouteGemmChain;
   }
@@ -879,7 +896,7 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     for (int l = 0; l < n_layers; ++l) {
       const wq_mlp_layer &Ly = layers[l];
       void *out = layer_out(l);
-      const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+      const GemvKind kind = gateup_kind(Ly.gate.bits);
       st = run_gateup_gemm(kind, cur, m, &Ly.gate, &Ly.up, Ly.lora_a, Ly.lora_b_gate, Ly.lora_b_up, Ly.r, Ly.lora_scale,
                            flags, layer_h(l), L, w8, s);
       if (st != WQ_OK) return fail(st, "layer %d: %s", l, g_last_error.c_str());
@@ -909,7 +926,7 @@ wq_status mlp_forward_impl(const void *x, int m, const wq_mlp_layer *layers, int
     const wq_mlp_layer &Ly = layers[l];
     void *out = layer_out(l);
     void *hbuf = layer_h(l);
-    const GemvKind kind = Ly.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+    const GemvKind kind = gateup_kind(Ly.gate.bits);
     const bool need_tp = prenorm || Ly.r > 0;
     const wq_mlp_layer *nx = l + 1 < n_layers ? &layers[l + 1] : nullptr;
     const bool dense_down = Ly.down.bits == 16;
@@ -969,7 +986,7 @@ wq_status wq_mlp_forward_info(int m, const wq_mlp_layer *layers, int n_layers, u
   }
   if (route == kRouteGemvChain) {
     const wq_mlp_layer &L0 = layers[0];
-    const GemvKind kind = L0.gate.bits == 2 ? kGateUpW2 : kGateUpW4;
+    const GemvKind kind = gateup_kind(L0.gate.bits);
     const bool next_tp = n_layers > 1 && ((flags & WQ_PRENORM) || layers[1].r > 0);
     const int r_next = next_tp ? layers[1].r : 0;
     GemvPlan pg, pd{};
@@ -1089,7 +1106,10 @@ wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens
   if ((st = wq_down_w4(w8 + W.o, batch, &Ly.o, x, w8 + W.x1, WQ_BF16, w8 + W.proj_o, W.n_o, stream)) != WQ_OK)
     return fail(st, "output projection: %s", g_last_error.c_str());
   const wq_mlp_layer &M = Ly.mlp;
-  if (M.gate.bits == 2)
+  if (M.gate.bits == 3)
+    st = wq_gateup_w3_lora(w8 + W.x1, batch, &M.gate, &M.up, M.lora_a, M.lora_b_gate, M.lora_b_up, M.r, M.lora_scale,
+                           flags, w8 + W.h, w8 + W.mlp, W.n_mlp, stream);
+  else if (M.gate.bits == 2)
     st = wq_gateup_w2_lora(w8 + W.x1, batch, &M.gate, &M.up, M.lora_a, M.lora_b_gate, M.lora_b_up, M.r, M.lora_scale,
                            flags, w8 + W.h, w8 + W.mlp, W.n_mlp, stream);
   else
@@ -1265,7 +1285,7 @@ wq_status wq_moe_forward(const void *x, int m, const float *logits, const wq_moe
 
 wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t info[10]) {
   if (!info) return fail(WQ_ERR_ARG, "null info array");
-  if (kind < 0 || kind > 2) return fail(WQ_ERR_ARG, "kind %d not in {0, 1, 2}", kind);
+  if (kind < 0 || kind > 3) return fail(WQ_ERR_ARG, "kind %d not in {0, 1, 2, 3}", kind);
   if (!group_ok(group) || k % group != 0) return fail(WQ_ERR_SHAPE, "group %d / k %d unsupported", group, k);
   const int sms = num_sms();
   if (sms <= 0) return fail(WQ_ERR_CUDA, "cannot query the current device");

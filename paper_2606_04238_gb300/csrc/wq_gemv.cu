@@ -124,7 +124,8 @@ constexpr int kMaxThreads = 512;  // per CTA: up to 128 registers a thread
 
 // ---------------------------------------------------------------------------
 // The dequant-GEMV kernel.
-//   BITS  2 or 4 (code width), NPROJ 2 (gate+up) or 1 (down),
+//   BITS  2, 3 or 4 (code width; 3: two bit planes, below), NPROJ 2
+//   (gate+up) or 1 (down),
 //   GROUP 32/64/128 (quantization group), NT 1 or 2 (8-token MMA tiles per
 //   token chunk: chunks of 8 tokens for m <= 8, of 16 otherwise), TPW 1 or 2
 //   (row tiles per warp: with 2, each activation fragment feeds 2 tiles x
@@ -133,7 +134,7 @@ constexpr int kMaxThreads = 512;  // per CTA: up to 128 registers a thread
 template <int BITS, int NPROJ, int GROUP, int NT, int TPW>
 __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p) {
   extern __shared__ __align__(128) uint8_t smem[];
-  constexpr int BPK = BITS == 2 ? 512 : 1024;  // code bytes per (row tile, 128-feature block)
+  constexpr int BPK = BITS == 2 ? 512 : BITS == 3 ? 768 : 1024;  // code bytes per (row tile, 128-feature block)
   constexpr int GPB = 128 / GROUP;             // groups per block
   constexpr int GS = GROUP / 16;               // k-steps (16 features) per group
   constexpr int TOK = 8 * NT;                  // tokens per chunk
@@ -401,7 +402,7 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
   // bit-position class of the codes that meet these features: 4^c for 2-bit
   // codes (c from the k-step parity and the feature half), 16^c for 4-bit
   // codes (c from the feature half)
-  const int sh = BITS == 2 ? 4 * (st & 1) + 2 * hi : 4 * hi;
+  const int sh = BITS != 4 ? 4 * (st & 1) + 2 * hi : 4 * hi;
   const int u0 = 4 * (lane & 1) + hi;  // features (2j, 2j+1) of a half sit in word 2j + half
   const bool lo_half = lane < 16;      // features 0..63 of the block
   for (int it0 = warp * CU; it0 < nitems; it0 += CU * nwarps) {
@@ -521,7 +522,7 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
               b[ks][nt][1] = v.y;
             }
           }
-        constexpr int NW = BITS == 2 ? 4 : 8;  // code words a lane holds per (tile, block)
+        constexpr int NW = BITS == 2 ? 4 : BITS == 3 ? 6 : 8;  // code words a lane holds per (tile, block)
         uint32_t wds[NPROJ][TPW][NW];
 #pragma unroll
         for (int pj = 0; pj < NPROJ; ++pj)
@@ -530,9 +531,14 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
             const uint8_t *cb = cbase + pj * cproj + ((size_t)j * p.KP + kb) * BPK;
 #pragma unroll
             for (int q = 0; q < NW; ++q) wds[pj][j][q] = 0u;
-            if (WQ_OK_IF(WQ_RANGE(cb - smem, BPK == 512 ? 16 : 528, p.off_meta, 16), 16, kb)) {
+            if (WQ_OK_IF(WQ_RANGE(cb - smem, BITS == 2 ? 16 : BITS == 3 ? 520 - 8 * lane : 528, p.off_meta, 16),
+                         16, kb)) {
               const uint4 w0 = lds128(cb);
               wds[pj][j][0] = w0.x; wds[pj][j][1] = w0.y; wds[pj][j][2] = w0.z; wds[pj][j][3] = w0.w;
+              if (BITS == 3) {  // the lane's two words of the high bit plane, at 512 + 8 lane in the block
+                const uint2 w1 = lds64(cb + 512 - 8 * lane);
+                wds[pj][j][4] = w1.x; wds[pj][j][5] = w1.y;
+              }
               if (BITS == 4) {
                 const uint4 w1 = lds128(cb + 512);
                 wds[pj][j][NW - 4] = w1.x; wds[pj][j][NW - 3] = w1.y;
@@ -609,6 +615,21 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
                 af[1] = x8 & (0x00030003u << s4);  // rows g+8
                 af[2] = x & (0x000C000Cu << s4);   // rows g,   features 2t+8..2t+9
                 af[3] = x8 & (0x000C000Cu << s4);  // rows g+8
+              } else if (BITS == 3) {
+                // the low two bits as for 2-bit codes; the high bit of the same
+                // code from the plane word, shifted to bit 2c + 2 (c the class):
+                // << 2 / << 1 for rows g / g+8 of an even 2-bit word, >> 6 / >> 7
+                // of an odd one.  A half then reads q 4^c 2^-24, q < 8.
+                const int wi = (ks >> 1) & 3;
+                const uint32_t x = wds[pj][j][wi];
+                const uint32_t x8 = x >> 8;
+                const uint32_t hw = wds[pj][j][4 + (wi >> 1)];
+                const uint32_t h0 = (wi & 1) ? hw >> 6 : hw << 2, h1 = (wi & 1) ? hw >> 7 : hw << 1;
+                const int s4 = (ks & 1) * 4;
+                af[0] = (x & (0x00030003u << s4)) | (h0 & (0x00040004u << s4));
+                af[1] = (x8 & (0x00030003u << s4)) | (h1 & (0x00040004u << s4));
+                af[2] = (x & (0x000C000Cu << s4)) | (h0 & (0x00100010u << s4));
+                af[3] = (x8 & (0x000C000Cu << s4)) | (h1 & (0x00100010u << s4));
               } else {
                 const uint32_t x = wds[pj][j][ks & (NW - 1)];
                 const uint32_t x8 = x >> 8;
@@ -1004,12 +1025,12 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
 // ---------------------------------------------------------------------------
 uint32_t align_up(uint32_t v, uint32_t a) { return (v + a - 1) / a * a; }
 
-int kind_bits(GemvKind k) { return k == kGateUpW2 ? 2 : 4; }
+int kind_bits(GemvKind k) { return k == kGateUpW2 ? 2 : k == kGateUpW3 ? 3 : 4; }
 int kind_nproj(GemvKind k) { return k == kDownW4 ? 1 : 2; }
 
 void compute_layout(GemvKind kind, int group, int r, GemvPlan *p) {
   const int nproj = kind_nproj(kind);
-  const int BPK = kind_bits(kind) == 2 ? 512 : 1024, GPB = 128 / group;
+  const int BPK = kind_bits(kind) * 256, GPB = 128 / group;
   uint32_t off = 0;
   p->r = r;
   p->off_codes = off;
@@ -1058,7 +1079,7 @@ bool search_plan(GemvKind kind, int N, int K, int M, int group, int r, int num_s
   const int tok = 8 * NT;
   const int MPAD = (M + tok - 1) / tok * tok;
   const int chunks = MPAD / tok;
-  const double blk_bytes = (kind_bits(kind) == 2 ? 512.0 : 1024.0) + 64.0 * (128 / group);
+  const double blk_bytes = 256.0 * kind_bits(kind) + 64.0 * (128 / group);
   const double total_bytes = (double)RT * KB * nproj * blk_bytes;
   const int max_warps = kMaxThreads / 32;
   bool found = false;
@@ -1253,7 +1274,10 @@ int kernel_regs(GemvKind kind, int group, int NT, int TPW) {
     case 5: fn = kernel_ptr<4, 2, 128>(NT, TPW); break;
     case 6: fn = kernel_ptr<4, 1, 32>(NT, TPW); break;
     case 7: fn = kernel_ptr<4, 1, 64>(NT, TPW); break;
-    default: fn = kernel_ptr<4, 1, 128>(NT, TPW); break;
+    case 8: fn = kernel_ptr<4, 1, 128>(NT, TPW); break;
+    case 9: fn = kernel_ptr<3, 2, 32>(NT, TPW); break;
+    case 10: fn = kernel_ptr<3, 2, 64>(NT, TPW); break;
+    default: fn = kernel_ptr<3, 2, 128>(NT, TPW); break;
   }
   cudaFuncAttributes attr{};
   const int regs = cudaFuncGetAttributes(&attr, fn) == cudaSuccess && attr.numRegs > 0 ? attr.numRegs : 128;
@@ -1267,6 +1291,7 @@ cudaError_t launch_gemv(GemvKind kind, const GemvPlan &plan, const GemvArgs &arg
     case kGateUpW2: return launch_g<2, 2>(plan, args, stream, pdl);
     case kGateUpW4: return launch_g<4, 2>(plan, args, stream, pdl);
     case kDownW4: return launch_g<4, 1>(plan, args, stream, pdl);
+    case kGateUpW3: return launch_g<3, 2>(plan, args, stream, pdl);
   }
   return cudaErrorInvalidValue;
 }

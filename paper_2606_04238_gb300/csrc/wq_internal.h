@@ -92,7 +92,9 @@ struct GemvArgs {
   size_t nb_hq, nb_hsc, nb_hxs, nb_pre_x, nb_pre_sc, nb_pre_xs;
 };
 
-enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2 };
+enum GemvKind { kGateUpW2 = 0, kGateUpW4 = 1, kDownW4 = 2, kGateUpW3 = 3 };
+// The gate/up kind of a code width (2, 3 or 4 bits).
+inline GemvKind gateup_kind(int bits) { return bits == 2 ? kGateUpW2 : bits == 3 ? kGateUpW3 : kGateUpW4; }
 
 // Batched (prefill-size) dequant-GEMM on the tcgen05 tensor cores (wq_gemm.cu).
 struct GemmArgs {

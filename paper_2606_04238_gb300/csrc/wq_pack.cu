@@ -9,7 +9,8 @@
 //   q = clamp(rint(w/s) + z, 0, qmax).
 // Two kernels: one warp per (row, group) computes s and z into the packed
 // meta layout; then one thread per packed 32-bit word gathers its 16 (2-bit)
-// or 8 (4-bit) codes.  Offline work: not on the decode path.
+// or 8 (4-bit) codes, or for 3-bit codes (App. B) 16 low-plane fields (q % 4)
+// or 32 high-plane bits (q / 4).  Offline work: not on the decode path.
 // A third kernel merges a trained adapter into a packed matrix before it is
 // quantized again (below).
 #include <cuda_bf16.h>
@@ -66,16 +67,45 @@ __global__ void quant_meta_kernel(const float *__restrict__ w, int n, int k, int
 
 __global__ void pack_codes_kernel(const float *__restrict__ w, int n, int k, int group, int bits, int RT, int KB,
                                   int NG, const uint16_t *__restrict__ meta, uint32_t *__restrict__ codes) {
-  const int WPB = bits == 2 ? 128 : 256;
+  const int WPB = bits == 2 ? 128 : bits == 3 ? 192 : 256;
   const size_t wid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (wid >= (size_t)RT * KB * WPB) return;
   const size_t blk = wid / WPB;
   const int wl = (int)(wid % WPB);
   const int rt = (int)(blk / KB), kb = (int)(blk % KB);
+  const float qmax = (float)((1 << bits) - 1);
+  // code of (local row i, block feature c), or 0 outside the matrix
+  auto code_at = [&](int i, int c) -> uint32_t {
+    const int row = rt * 16 + i, col = kb * 128 + c;
+    if (row >= n || col >= k) return 0u;
+    const size_t mb = ((size_t)rt * NG + col / group) * 32 + 4 * (i & 7) + (i >> 3);
+    const float sf = __half2float(__ushort_as_half(meta[mb]));
+    const float zf = __half2float(__ushort_as_half(meta[mb + 2]));
+    return (uint32_t)fminf(fmaxf(__fadd_rn(rintf(__fdiv_rn(w[(size_t)row * k + col], sf)), zf), 0.f), qmax);
+  };
+  if (bits == 3) {
+    uint32_t word = 0;
+    if (wl < 128) {  // low plane: q % 4 where a 2-bit code would sit
+      const int lane = wl >> 2, wi = wl & 3;
+      for (int bit = 0; bit < 32; bit += 2) {
+        const int half = bit >> 4, rowhalf = (bit >> 3) & 1, cls = (bit & 7) >> 1;
+        const int c = wi * 32 + (cls >> 1) * 16 + (cls & 1) * 8 + (lane & 3) * 2 + half;
+        word |= (code_at((lane >> 2) + 8 * rowhalf, c) & 3u) << bit;
+      }
+    } else {  // high plane: word 128 + 2 lane + p holds q / 4 of the features c with (c / 32) / 2 = p
+      const int lane = (wl - 128) >> 1, pp = (wl - 128) & 1;
+      for (int bit = 0; bit < 32; ++bit) {
+        const int half = bit >> 4, cpar = (bit >> 3) & 1, cls = (bit & 7) >> 1, ihi = bit & 1;
+        const int c = (2 * pp + cpar) * 32 + (cls >> 1) * 16 + (cls & 1) * 8 + (lane & 3) * 2 + half;
+        word |= (code_at((lane >> 2) + 8 * ihi, c) >> 2) << bit;
+      }
+    }
+    codes[wid] = word;
+    return;
+  }
   const int tile = bits == 2 ? 0 : wl >> 7;  // 64-feature half of a 4-bit block
   const int wl2 = wl & 127;
   const int lane = wl2 >> 2, wi = wl2 & 3;
-  const float qmax = (float)((1 << bits) - 1);
   uint32_t word = 0;
   for (int bit = 0; bit < 32; bit += bits) {
     const int half = bit >> 4, rowhalf = (bit >> 3) & 1;
@@ -87,15 +117,7 @@ __global__ void pack_codes_kernel(const float *__restrict__ w, int n, int k, int
       const int hi = (bit & 7) >> 2;
       c = tile * 64 + wi * 16 + hi * 8 + (lane & 3) * 2 + half;
     }
-    const int i = (lane >> 2) + 8 * rowhalf;
-    const int row = rt * 16 + i, col = kb * 128 + c;
-    if (row < n && col < k) {
-      const size_t mb = ((size_t)rt * NG + col / group) * 32 + 4 * (i & 7) + (i >> 3);
-      const float sf = __half2float(__ushort_as_half(meta[mb]));
-      const float zf = __half2float(__ushort_as_half(meta[mb + 2]));
-      const float qf = fminf(fmaxf(__fadd_rn(rintf(__fdiv_rn(w[(size_t)row * k + col], sf)), zf), 0.f), qmax);
-      word |= (uint32_t)qf << bit;
-    }
+    word |= code_at((lane >> 2) + 8 * rowhalf, c) << bit;
   }
   codes[wid] = word;
 }
@@ -118,8 +140,8 @@ __global__ void __launch_bounds__(kMergeThreads)
                       const __nv_bfloat16 *__restrict__ lora_a, int r, double alpha, float *__restrict__ w) {
   __shared__ double brow[kMaxRank];
   const int col = blockIdx.x * kMergeThreads + threadIdx.x;
-  const int wpb = bits == 2 ? 128 : 256;
-  const uint32_t mask = (1u << bits) - 1u;
+  const int wpb = bits == 2 ? 128 : bits == 3 ? 192 : 256;
+  const uint32_t mask = bits == 3 ? 3u : (1u << bits) - 1u;
   for (int row = blockIdx.y; row < n; row += gridDim.y) {
     __syncthreads();  // the previous row's B is read by every thread first
     if (threadIdx.x < r) brow[threadIdx.x] = (double)__bfloat162float(lora_b[(size_t)row * r + threadIdx.x]);
@@ -128,14 +150,19 @@ __global__ void __launch_bounds__(kMergeThreads)
     const int rt = row >> 4, i = row & 15, kb = col >> 7, c = col & 127;
     const int lane = (i & 7) * 4 + ((c & 7) >> 1), half = c & 1;
     int word, bit;
-    if (bits == 2) {
+    if (bits != 4) {
       word = lane * 4 + (c >> 5);
       bit = 16 * half + 8 * (i >> 3) + 2 * (2 * ((c & 31) >> 4) + ((c & 15) >> 3));
     } else {
       word = (c >> 6) * 128 + lane * 4 + ((c & 63) >> 4);
       bit = 16 * half + 8 * (i >> 3) + 4 * ((c & 15) >> 3);
     }
-    const uint32_t q = (codes[((size_t)rt * KB + kb) * wpb + word] >> bit) & mask;
+    const uint32_t *blk = codes + ((size_t)rt * KB + kb) * wpb;
+    uint32_t q = (blk[word] >> bit) & mask;
+    if (bits == 3) {  // the high bit from the second plane
+      const int cls = 2 * ((c & 31) >> 4) + ((c & 15) >> 3);
+      q |= ((blk[128 + lane * 2 + ((c >> 5) >> 1)] >> (16 * half + 8 * ((c >> 5) & 1) + 2 * cls + (i >> 3))) & 1u) << 2;
+    }
     const size_t mb = ((size_t)rt * NG + col / group) * 32 + 4 * (i & 7) + (i >> 3);
     const double sf = (double)__half2float(__ushort_as_half(meta[mb]));
     const double zf = (double)__half2float(__ushort_as_half(meta[mb + 2]));
@@ -170,7 +197,7 @@ cudaError_t launch_pack(const float *w, int n, int k, int group, int bits, uint3
                                                                                  nonfinite);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const long long words = (long long)RT * KB * (bits == 2 ? 128 : 256);
+  const long long words = (long long)RT * KB * (bits == 2 ? 128 : bits == 3 ? 192 : 256);
   pack_codes_kernel<<<(unsigned)((words + tpb - 1) / tpb), tpb, 0, stream>>>(w, n, k, group, bits, RT, KB, NG, meta,
                                                                              codes);
   return cudaGetLastError();

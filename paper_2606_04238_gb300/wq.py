@@ -80,6 +80,7 @@ def lib():
             "wq_workspace_init": (I, [P, S, P]),
             "wq_gateup_w2_lora": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P, S, P]),
             "wq_gateup_w2_lora_noalloc": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P]),
+            "wq_gateup_w3_lora": (I, [P, I, QP, QP, P, P, P, I, F, U, P, P, S, P]),
             "wq_gateup_w4": (I, [P, I, QP, QP, U, P, P, S, P]),
             "wq_down_w4": (I, [P, I, QP, P, P, I, P, S, P]),
             "wq_down_bf16": (I, [P, I, P, I, I, P, P, I, P]),
@@ -223,6 +224,22 @@ def gateup_w2_lora(x, gate: QWeight, up: QWeight, lora_a=None, lora_b_gate=None,
         ws = workspace(max(m, 1), d, gate.n, r, device=x.device)
     cg, cu = gate.c(), up.c()
     _check(lib().wq_gateup_w2_lora(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), _ptr(lora_a), _ptr(lora_b_gate),
+                                   _ptr(lora_b_up), r, float(lora_scale), WQ_PRENORM if prenorm else 0, _ptr(h),
+                                   _ptr(ws), ws.numel(), _stream()))
+    return h
+
+
+def gateup_w3_lora(x, gate: QWeight, up: QWeight, lora_a=None, lora_b_gate=None, lora_b_up=None,
+                   lora_scale: float = 0.0, prenorm: bool = False, h=None, ws=None):
+    """wq_gateup_w3_lora: gateup_w2_lora with 3-bit gate/up codes (App. B)."""
+    m, d = x.shape
+    r = 0 if lora_b_gate is None else lora_b_gate.shape[1]
+    if h is None:
+        h = torch.empty((m, gate.n), dtype=torch.bfloat16, device=x.device)
+    if ws is None:
+        ws = workspace(max(m, 1), d, gate.n, r, device=x.device)
+    cg, cu = gate.c(), up.c()
+    _check(lib().wq_gateup_w3_lora(_ptr(x), m, ctypes.byref(cg), ctypes.byref(cu), _ptr(lora_a), _ptr(lora_b_gate),
                                    _ptr(lora_b_up), r, float(lora_scale), WQ_PRENORM if prenorm else 0, _ptr(h),
                                    _ptr(ws), ws.numel(), _stream()))
     return h

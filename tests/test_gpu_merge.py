@@ -45,7 +45,7 @@ def _assert_packed(qw, codes, meta):
     assert np.array_equal(qw.meta.cpu().numpy().view(np.uint16), meta)
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 @pytest.mark.parametrize("n,k,group,r", [(16, 128, 128, 1), (40, 384, 128, 16), (33, 192, 64, 8),
                                          (200, 384, 32, 64), (1000, 640, 128, 32), (5, 96, 32, 8)])
 @pytest.mark.parametrize("alpha", [2.0, 0.37])
@@ -63,7 +63,7 @@ def test_merge_bit_exact(wq, bits, n, k, group, r, alpha):
     _assert_packed(src, c0, m0)
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_merge_rank0_and_alpha0(wq, bits):
     n, k, group = 48, 256, 64
     qsz, a, b = _case(n, k, group, bits, 8, seed=5 + bits)

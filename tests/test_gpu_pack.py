@@ -35,7 +35,7 @@ def _weights(kind, n, k, rng):
     return w.astype(np.float32)
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 @pytest.mark.parametrize("n,k,group", [(16, 128, 128), (768, 256, 64), (37, 192, 64), (200, 384, 32),
                                        (1000, 640, 128), (5, 96, 32)])
 @pytest.mark.parametrize("dist", ["n002", "n1", "edge"])
