@@ -46,7 +46,9 @@ def test_packed_sizes(wq):
     assert wq.packed_sizes(2, 9728, 2560, 128) == (608 * 20 * 512, 608 * 20 * 64)
     # ragged rows and features pad to 16 x 128
     assert wq.packed_sizes(4, 21, 160, 32) == (2 * 2 * 1024, 2 * 8 * 64)
-    for bad in ((3, 16, 128, 64), (2, 16, 128, 48), (2, 16, 100, 64), (4, 16, 128, 256)):
+    # 3-bit codes (two planes): 192 words a block
+    assert wq.packed_sizes(3, 40, 256, 32) == (3 * 2 * 768, 3 * 8 * 64)
+    for bad in ((5, 16, 128, 64), (1, 16, 128, 64), (2, 16, 128, 48), (2, 16, 100, 64), (4, 16, 128, 256)):
         with pytest.raises(wq.WQError) as e:
             wq.packed_sizes(*bad)
         assert e.value.status == -2
@@ -69,6 +71,9 @@ def test_gateup_host_validation(wq):
     assert call(x, -1, ok_g, ok_u) == -1                                   # negative m
     assert call(x, 16385, ok_g, ok_u) == -4                                # beyond the token limit
     assert call(x, 1, _qw(wq, 64, 256, 64, 4), ok_u) == -2                 # wrong bit width
+    assert L.wq_gateup_w3_lora(x, 65, ctypes.byref(_qw(wq, 64, 256, 64, 3)), ctypes.byref(_qw(wq, 64, 256, 64, 3)),
+                               None, None, None, 0, 0.0, 0, ctypes.c_void_p(16), ctypes.c_void_p(16), 1 << 20,
+                               None) == -4                                  # 3-bit codes above 64 tokens
     assert call(x, 1, ok_g, _qw(wq, 32, 256, 64, 2)) == -2                 # gate / up differ
     assert call(x, 1, _qw(wq, 64, 200, 64, 2), _qw(wq, 64, 200, 64, 2)) == -2  # k % group
     assert call(x, 1, _qw(wq, 64, 256, 48, 2), _qw(wq, 64, 256, 48, 2)) == -2  # group
@@ -104,7 +109,7 @@ def test_down_and_stack_host_validation(wq):
 def test_pack_host_validation(wq):
     L = wq.lib()
     q = _qw(wq, 0, 0, 0, 0, codes=0, meta=0)
-    assert L.wq_pack(ctypes.c_void_p(16), 16, 128, 64, 3, ctypes.byref(q), None, None) == -2
+    assert L.wq_pack(ctypes.c_void_p(16), 16, 128, 64, 5, ctypes.byref(q), None, None) == -2
     assert L.wq_pack(ctypes.c_void_p(16), 16, 96, 64, 2, ctypes.byref(q), None, None) == -2
     assert L.wq_pack(ctypes.c_void_p(16), 16, 128, 64, 2, ctypes.byref(q), None, None) == -1   # null codes
     q2 = _qw(wq, 0, 0, 0, 0, codes=16, meta=40)
@@ -121,7 +126,7 @@ def test_merge_host_validation(wq):
                                scale, ctypes.c_void_p(wm), None if out is None else ctypes.byref(out), None, None)
 
     assert call(None) == -1                                         # null source
-    assert call(_qw(wq, 64, 256, 64, 3)) == -2                      # bits
+    assert call(_qw(wq, 64, 256, 64, 5)) == -2                      # bits
     assert call(_qw(wq, 64, 256, 48, 2)) == -2                      # group
     assert call(_qw(wq, 64, 256, 64, 2, meta=8)) == -3              # misaligned meta
     assert call(src, r=65) == -2                                    # rank above 64
@@ -160,3 +165,28 @@ def test_product_path_has_no_oracle_import():
                 text = open(os.path.join(dirpath, fn)).read()
                 assert "import oracle" not in text and "from oracle" not in text, fn
                 assert "wq_oracle" not in text, fn
+
+
+def test_moe_host_validation(wq):
+    L = wq.lib()
+    ex = wq._MLPLayer(_qw(wq, 4 * 64, 256, 64, 2), _qw(wq, 4 * 64, 256, 64, 2), _qw(wq, 4 * 256, 64, 64, 4), None,
+                      None, None, 0, 0.0)
+
+    def call(E=4, k=2, m=1, flags=1, x=16, experts=ex):
+        layer = wq._MoELayer(experts, E, k)
+        return L.wq_moe_forward(ctypes.c_void_p(x), m, ctypes.c_void_p(16), ctypes.byref(layer), flags,
+                                ctypes.c_void_p(16), None, None, None, None, ctypes.c_void_p(16), 1 << 20, None)
+
+    assert call(k=0) == -2                                           # no expert selected
+    assert call(k=5) == -2                                           # more than the experts
+    assert call(E=3) == -2                                           # rows not a multiple of the experts
+    assert call(E=300, k=2) == -2                                    # above 256 experts
+    assert call(m=65) == -2                                          # above 64 tokens
+    assert call(flags=2) == -1                                       # unknown flag
+    assert call(m=0) == 0                                            # empty batch: no-op
+    assert call(x=0) == -1                                           # null x
+    assert call(x=24) == -3                                          # misaligned x
+    bad_down = wq._MLPLayer(ex.gate, ex.up, _qw(wq, 4 * 256, 128, 64, 4), None, None, None, 0, 0.0)
+    assert call(experts=bad_down) == -2                              # down [E d x inter] mismatch
+    with_lora = wq._MLPLayer(ex.gate, ex.up, ex.down, None, None, None, 8, 2.0)
+    assert call(experts=with_lora) == -1                             # rank without pointers
