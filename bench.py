@@ -53,8 +53,10 @@ def parse():
     ap.add_argument("--no-extras", action="store_true", help="skip the comparator / per-kernel / CPU legs")
     ap.add_argument("--eager", action="store_true",
                     help="profiling aid: run the stack with plain stream launches (no CUDA graph), print no JSON")
-    ap.add_argument("--leg", default="decode", choices=["decode", "prefill"],
-                    help="with --eager: which stack to run (the decode stack or the prefill chunk)")
+    ap.add_argument("--leg", default="decode", choices=["decode", "prefill", "moe", "decoder", "w3", "bf16down"],
+                    help="with --eager: which stack to run (the decode stack, the prefill chunk, the MoE stack, "
+                         "whole decoder layers at --context, the stack with 3-bit g32 gate/up, or with bf16 down)")
+    ap.add_argument("--context", type=int, default=8192, help="with --eager --leg decoder: the KV-cache length")
     ap.add_argument("--prefill-layers", type=int, default=4, help="distinct 14B-shaped layers of the prefill leg")
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the bench line: decode stacks of the 4B/8B/14B shapes over their token counts, "
@@ -335,11 +337,23 @@ def run_gpu(args):
     if args.eager and args.leg == "prefill":
         run_prefill(wq, synth, dev, args.prefill_layers, steps, warmup, eager=True)
         return
+    if args.eager and args.leg in ("moe", "decoder"):
+        run_eager_leg(args, wq, synth, dev, steps, warmup)
+        return
     if args.sweep:
         print(json.dumps(run_sweep(wq, synth, dev, min(steps, 200), warmup)))
         return
 
-    layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
+    if args.eager and args.leg == "w3":
+        import dataclasses
+        layers = build_stack(wq, synth, dataclasses.replace(cfg, group_gu=32), n_layers, 3, True, dev)
+    else:
+        layers = build_stack(wq, synth, cfg, n_layers, 2, True, dev)
+    if args.eager and args.leg == "bf16down":
+        layers = [wq.MLPLayer(L.gate, L.up, wq.dense_weight(synth.weights((cfg.d, cfg.inter), 3 * l + 2, device=dev)
+                                                             .to(torch.bfloat16)),
+                              lora_a=L.lora_a, lora_b_gate=L.lora_b_gate, lora_b_up=L.lora_b_up,
+                              lora_scale=L.lora_scale) for l, L in enumerate(layers)]
     table = wq.LayerTable(layers)
     ws = wq.workspace(m, cfg.d, cfg.inter, cfg.r)
     x = synth.activations((m, cfg.d), 2024 + rank, device=dev)
@@ -757,6 +771,59 @@ def run_moe(wq, synth, dev, steps, warmup, peak, shape=MOE_SHAPE, m=1):
     out["note"] = ("wq_moe_forward per layer (routing + tile partials, gate/up and down over the selected "
                    "experts' slots, combine): only the k selected experts' weights are read")
     return out
+
+
+def run_eager_leg(args, wq, synth, dev, steps, warmup):
+    """Profiling aid (--eager): the MoE stack or whole decoder layers issued with plain stream launches."""
+    import torch
+    n = args.layers or 2
+    m = args.m
+    if args.leg == "moe":
+        sh = MOE_SHAPE
+        d, inter, E, k, g, r = (sh[key] for key in ("d", "inter", "experts", "top_k", "group", "r"))
+        blocks = []
+        for l in range(n):
+            _, bg, bu = synth.lora(d, E * inter, r, 60_000 + l, device=dev)
+            a = synth.weights((E * 2 * r, d), 61_000 + l, std=0.01, device=dev).to(torch.bfloat16)
+            ex = wq.MLPLayer(wq.pack(synth.weights((E * inter, d), 50_000 + 3 * l, device=dev), g, 2),
+                             wq.pack(synth.weights((E * inter, d), 50_001 + 3 * l, device=dev), g, 2),
+                             wq.pack(synth.weights((E * d, inter), 50_002 + 3 * l, device=dev), g, 4),
+                             lora_a=a, lora_b_gate=bg, lora_b_up=bu, lora_scale=sh["lora_scale"])
+            blocks.append(wq.MoELayer(ex, E, k))
+        logits = [synth.weights((m, E), 8000 + l, std=1.0, device=dev) for l in range(n)]
+        x = synth.activations((m, d), 31, device=dev)
+        ws = wq.moe_workspace(m, blocks[0])
+
+        def step():
+            cur = x
+            for l in range(n):
+                cur = wq.moe_forward(cur, logits[l], blocks[l], ws=ws)
+    else:
+        cfg = synth.CONFIGS["qwen3_4b"]
+        H, Hkv, hd = DECODER_HEADS
+        layers = build_stack(wq, synth, cfg, n, 2, True, dev)
+        dl, caches = [], []
+        for l in range(n):
+            wqkv = synth.weights(((H + 2 * Hkv) * hd, cfg.d), 7000 + 2 * l, device=dev)
+            wo = synth.weights((cfg.d, H * hd), 7001 + 2 * l, device=dev)
+            dl.append(wq.DecoderLayer(wq.pack(wqkv, 128, 4), wq.pack(wo, 128, 4), layers[l], H, Hkv, hd))
+            gen = torch.Generator(device=dev)
+            gen.manual_seed(9000 + l)
+            caches.append(tuple(torch.randn((m, Hkv, args.context, hd), generator=gen, device=dev)
+                                .to(torch.bfloat16) for _ in range(2)))
+        lens = torch.full((m,), args.context - 1, dtype=torch.int32, device=dev)
+        x = synth.activations((m, cfg.d), 77, device=dev)
+        ws = wq.decoder_workspace(m, dl[0], args.context)
+
+        def step():
+            cur = x
+            for l in range(n):
+                cur = wq.decoder_layer_forward(cur, lens, dl[l], caches[l][0], caches[l][1], ws=ws)
+    for _ in range(warmup + steps):
+        step()
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    print(f"eager: {warmup + steps} {args.leg} steps of {n} layers done", flush=True)
 
 
 # --------------------------------------------------------------------------- reference arm
