@@ -15,7 +15,10 @@
 //   4. o = softmax(q K^T / sqrt(hd)) V over positions 0..lens[b].
 // The context is cut into S splits (grid.y); a CTA of 8 warps takes one
 // (b, g) and one split; each warp takes chunks of 8 positions, the lanes the
-// head dimension (coalesced 8-byte loads of every K and V row).  The 32
+// head dimension.  A warp copies its next chunk's K and V rows into a shared-
+// memory buffer of its own (cp.async, 16 bytes a lane and copy) while it
+// computes the current chunk from the other buffer, so two chunks' rows are
+// in flight at a time.  The 32
 // partial dot products of a chunk (8 positions x 4 query heads) are reduced
 // by a butterfly reduce-scatter (31 shuffles), the softmax runs online (max,
 // sum, rescaled accumulators) in fp32.  The splits' partial results (max,
@@ -46,14 +49,15 @@ constexpr int kPos = 8;  // positions a chunk takes (kHG * kPos = 32 lanes)
 __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
-// HD/32 consecutive bf16 values of a row (8 bytes for HD 128, 4 for HD 64)
+// HD/32 consecutive bf16 values of a row in shared memory (8 bytes for HD
+// 128, 4 for HD 64)
 template <int HD>
-__device__ __forceinline__ void load_row(const __nv_bfloat16 *p, float (&v)[HD / 32]) {
+__device__ __forceinline__ void load_row_s(const __nv_bfloat16 *p, float (&v)[HD / 32]) {
   if (HD == 128) {
-    const uint2 w = __ldg(reinterpret_cast<const uint2 *>(p));
+    const uint2 w = *reinterpret_cast<const uint2 *>(p);
     v[0] = bf_lo(w.x); v[1] = bf_hi(w.x); v[2] = bf_lo(w.y); v[3] = bf_hi(w.y);
   } else {
-    const uint32_t w = __ldg(reinterpret_cast<const uint32_t *>(p));
+    const uint32_t w = *reinterpret_cast<const uint32_t *>(p);
     v[0] = bf_lo(w); v[1] = bf_hi(w);
   }
 }
@@ -67,11 +71,35 @@ struct RopeFreq {
 
 // grid (B * n_kv, S), block kAttnWarps * 32.  part: [B][H][S][HD + 2] fp32
 // (accumulator, max, sum) of every split.
+// Copies of one chunk (positions cb .. cb + kPos - 1) of K and V rows into a
+// warp's buffer dst ([K, V][kPos][HD], already offset by the lane's column):
+// copy i of a lane takes row i * (32 / CPR) + lrow; positions outside
+// [p0, p1) and the new position pos are zero-filled.
 template <int HD>
-__global__ void __launch_bounds__(kAttnWarps * 32) attn_split_kernel(
+__device__ __forceinline__ void attn_issue(__nv_bfloat16 *dst, const __nv_bfloat16 *kbase,
+                                           const __nv_bfloat16 *vbase, int lrow, int cb, int p0, int p1, int pos) {
+  constexpr int CPR = HD * 2 / 16;
+#pragma unroll
+  for (int i = 0; i < 2 * kPos * CPR / 32; ++i) {
+    const int r = i * (32 / CPR) + lrow;
+    const int p = cb + r % kPos;
+    const bool in = p < p1 && p != pos;
+    const __nv_bfloat16 *src = (r < kPos ? kbase : vbase) + (size_t)(in ? p : p0) * HD;
+    cp_async16_zfill(dst + (size_t)r * HD, src, in ? 16u : 0u);
+  }
+}
+
+// Dynamic shared memory: per warp two chunk buffers of K and V rows,
+// [warp][buffer][K, V][kPos][HD] bf16.
+template <int HD>
+constexpr int attn_smem_bytes() { return kAttnWarps * 2 * 2 * kPos * HD * 2; }
+
+template <int HD>
+__global__ void __launch_bounds__(kAttnWarps * 32, 2) attn_split_kernel(
     const float *qkv, const __nv_bfloat16 *x, const int *lens, int d, int H, int Hkv, const RopeFreq fr,
     __nv_bfloat16 *k_cache, __nv_bfloat16 *v_cache, int max_len, float *part, int S) {
   constexpr int E = HD / 32;  // dimensions a lane holds
+  extern __shared__ __align__(16) uint8_t attn_dyn[];
   __shared__ float qs[kHG * 2][HD];  // the group's query heads (up to 8), scaled by 1/sqrt(HD)
   __shared__ float kvn[2][HD];       // the new token's k (normalized, rotated, bf16-rounded) and v
   __shared__ float red[kAttnWarps];
@@ -174,7 +202,26 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_split_kernel(
     for (int hq = 0; hq < kHG; ++hq)
 #pragma unroll
       for (int e = 0; e < E; ++e) acc[hq][e] = 0.f;
-    for (int c0 = p0 + warp * kPos; c0 < p1; c0 += kAttnWarps * kPos) {
+    // this warp's chunk buffers; positions outside [p0, p1) and the new
+    // position (taken from kvn) are zero-filled
+    __nv_bfloat16 *wbuf = reinterpret_cast<__nv_bfloat16 *>(attn_dyn) + (size_t)warp * 2 * 2 * kPos * HD;
+    constexpr int CPR = HD * 2 / 16;  // 16-byte copies a row
+    // copy i of a lane: row r = i * (32 / CPR) + lane / CPR of the [K, V][kPos]
+    // rows, 16 bytes at column lane % CPR
+    const int lrow = lane / CPR, lcol = (lane % CPR) * 8;
+    const __nv_bfloat16 *kbase = k_cache + cache_off + lcol, *vbase = v_cache + cache_off + lcol;
+    constexpr int stride = kAttnWarps * kPos;
+    int bi = 0;
+    if (p0 + warp * kPos < p1)
+      attn_issue<HD>(wbuf + lcol, kbase, vbase, lrow, p0 + warp * kPos, p0, p1, pos);
+    cp_async_commit();
+    for (int c0 = p0 + warp * kPos; c0 < p1; c0 += stride, bi ^= 1) {
+      if (c0 + stride < p1)
+        attn_issue<HD>(wbuf + (size_t)(bi ^ 1) * 2 * kPos * HD + lcol, kbase, vbase, lrow, c0 + stride, p0, p1, pos);
+      cp_async_commit();
+      cp_async_wait_group1();  // this chunk's rows have landed
+      __syncwarp();
+      const __nv_bfloat16 *cur = wbuf + (size_t)bi * 2 * kPos * HD;
       // partial dots of 8 positions x 4 heads: index pp * 4 + hq
       float sv[32];
       float vv[kPos][E];
@@ -182,14 +229,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_split_kernel(
       for (int pp = 0; pp < kPos; ++pp) {
         const int p = c0 + pp;
         float kr[E];
-        if (p < p1 && p != pos) {
-          load_row<HD>(k_cache + cache_off + (size_t)p * HD + lane * E, kr);
-          load_row<HD>(v_cache + cache_off + (size_t)p * HD + lane * E, vv[pp]);
+        if (p != pos) {
+          load_row_s<HD>(cur + (size_t)pp * HD + lane * E, kr);
+          load_row_s<HD>(cur + (size_t)(kPos + pp) * HD + lane * E, vv[pp]);
         } else {
 #pragma unroll
           for (int e = 0; e < E; ++e) {
-            kr[e] = p == pos ? kvn[0][lane * E + e] : 0.f;
-            vv[pp][e] = p == pos ? kvn[1][lane * E + e] : 0.f;
+            kr[e] = kvn[0][lane * E + e];
+            vv[pp][e] = kvn[1][lane * E + e];
           }
         }
 #pragma unroll
@@ -242,7 +289,9 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_split_kernel(
 #pragma unroll
           for (int e = 0; e < E; ++e) acc[hq][e] = fmaf(pw, vv[pp][e], acc[hq][e]);
         }
+      __syncwarp();  // every lane is done with this buffer before it is filled again
     }
+    cp_async_wait_all();
     // merge the warps (fixed order) and write the split's partials
     if (lane < kHG) {
       ws_m[warp][lane] = m_run;
@@ -314,10 +363,16 @@ cudaError_t launch_attn_decode(const float *qkv, const void *x, const int *lens,
   auto *kc = reinterpret_cast<__nv_bfloat16 *>(k_cache), *vc = reinterpret_cast<__nv_bfloat16 *>(v_cache);
   auto *ob = reinterpret_cast<__nv_bfloat16 *>(o);
   if (HD == 128) {
-    attn_split_kernel<128><<<grid, kAttnWarps * 32, 0, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
+    constexpr int sm = attn_smem_bytes<128>();
+    cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+    if (e != cudaSuccess) return e;
+    attn_split_kernel<128><<<grid, kAttnWarps * 32, sm, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
     attn_combine_kernel<128><<<B * H, 128, 0, s>>>(part, lens, H, S, max_len, ob);
   } else if (HD == 64) {
-    attn_split_kernel<64><<<grid, kAttnWarps * 32, 0, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
+    constexpr int sm = attn_smem_bytes<64>();
+    cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+    if (e != cudaSuccess) return e;
+    attn_split_kernel<64><<<grid, kAttnWarps * 32, sm, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
     attn_combine_kernel<64><<<B * H, 64, 0, s>>>(part, lens, H, S, max_len, ob);
   } else {
     return cudaErrorInvalidValue;
