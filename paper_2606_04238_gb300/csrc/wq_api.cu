@@ -1103,9 +1103,44 @@ wq_status wq_decoder_layer_forward(const void *x, int batch, const int32_t *lens
   if ((st = wq_attn_decode(reinterpret_cast<const float *>(w8 + W.qkv), x, lens, batch, d, H, Hkv, hd, Ly.rope_theta,
                            k_cache, v_cache, max_len, w8 + W.o, w8 + W.attn, W.n_attn, stream)) != WQ_OK)
     return fail(st, "attention: %s", g_last_error.c_str());
+  const wq_mlp_layer &M = Ly.mlp;
+  // Decode sizes: the output projection's epilogue also writes the MLP
+  // input's tile partials (RMSNorm sums and LoRA-A products of x1, as the
+  // stack's down launches do for the next layer), so the gate/up launch needs
+  // no partials kernel, and gate/up hands down the ready binary16 panel of h.
+  {
+    const int bits = M.gate.bits;
+    const bool gu_ok = bits >= 2 && bits <= 4 && check_gateup_pair(&M.gate, &M.up, bits) == WQ_OK &&
+                       check_lora(M.lora_a, M.lora_b_gate, M.lora_b_up, M.r) == WQ_OK && !(bits == 4 && M.r != 0) &&
+                       M.down.bits == 4 && check_down(&M.down) == WQ_OK;
+    const GemvKind kind = gateup_kind(bits);
+    const bool need_tp = (flags & WQ_PRENORM) || M.r > 0;
+    const int r_o = need_tp ? M.r : 0;
+    if (gu_ok && !gateup_uses_gemm(kind, batch, &M.gate, M.r) && !down_uses_gemm(batch, &M.down, 0) &&
+        !down_uses_gemm(batch, &Ly.o, r_o) && (r_o == 0 || d % 8 == 0)) {
+      if (!y) return fail(WQ_ERR_ARG, "null y");
+      if (!aligned16(y)) return fail(WQ_ERR_ALIGN, "y not 16-byte aligned");
+      WsLayout Lm, Lo;
+      if ((st = check_ws(w8 + W.mlp, W.n_mlp, batch, d, inter, &Lm)) != WQ_OK ||
+          (st = check_ws(w8 + W.proj_o, W.n_o, batch, d, H * hd, &Lo)) != WQ_OK)
+        return st;
+      cudaStream_t s = static_cast<cudaStream_t>(stream);
+      float *tp = need_tp ? reinterpret_cast<float *>(w8 + W.mlp + Lm.tp) : nullptr;
+      if ((st = run_down(w8 + W.o, batch, &Ly.o, x, w8 + W.x1, 0, need_tp ? M.lora_a : nullptr, r_o, tp, Lo,
+                         w8 + W.proj_o, s)) != WQ_OK)
+        return fail(st, "output projection: %s", g_last_error.c_str());
+      const bool panel = chain_panel_ok(kind, batch, M.gate, M.r, M.down, 0);
+      if ((st = run_gateup(kind, w8 + W.x1, batch, &M.gate, &M.up, M.lora_a, M.lora_b_gate, M.lora_b_up, M.r,
+                           M.lora_scale, flags, w8 + W.h, tp, Lm, w8 + W.mlp, s, panel)) != WQ_OK)
+        return fail(st, "gate/up: %s", g_last_error.c_str());
+      if ((st = run_down(w8 + W.h, batch, &M.down, w8 + W.x1, y, 0, nullptr, 0, nullptr, Lm, w8 + W.mlp, s,
+                         panel)) != WQ_OK)
+        return fail(st, "down: %s", g_last_error.c_str());
+      return ok();
+    }
+  }
   if ((st = wq_down_w4(w8 + W.o, batch, &Ly.o, x, w8 + W.x1, WQ_BF16, w8 + W.proj_o, W.n_o, stream)) != WQ_OK)
     return fail(st, "output projection: %s", g_last_error.c_str());
-  const wq_mlp_layer &M = Ly.mlp;
   if (M.gate.bits == 3)
     st = wq_gateup_w3_lora(w8 + W.x1, batch, &M.gate, &M.up, M.lora_a, M.lora_b_gate, M.lora_b_up, M.r, M.lora_scale,
                            flags, w8 + W.h, w8 + W.mlp, W.n_mlp, stream);

@@ -168,6 +168,27 @@ def test_decoder_layer_end_to_end(wq):
         check_bf16(kd[i, :, n], orc.bf16_bits_to_f64(ref["k_cache"][i, :, n]), f"cache k, sequence {i}", min_exact=0.9)
 
 
+@pytest.mark.parametrize("lora", [True, False])
+def test_qwen3_4b_decoder_layer_end_to_end(wq, lora):
+    """The composite call at the Qwen3-4B shape, where the output projection
+    hands the MLP its input's tile partials and gate/up hands down the ready
+    binary16 panel of h (the decode route of the benchmark's decoder leg)."""
+    cfg = synth.CONFIGS["qwen3_4b"]
+    H, Hkv, hd = 32, 8, 128
+    layer, ora = _build(wq, cfg.d, cfg.inter, H, Hkv, hd, 128, 128, 16 if lora else 0, 111)
+    lens, max_len = [1000], 1024
+    x = synth.activations((1, cfg.d), 112)
+    kc, vc = _caches(1, Hkv, max_len, hd, lens, 113)
+    kd, vd = _dev(kc), _dev(vc)
+    y = wq.decoder_layer_forward(x.cuda(), torch.tensor(lens, dtype=torch.int32, device="cuda"), layer, kd, vd)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref = odec.decoder_layer_decode(synth.bf16_bits(x), lens, kc, vc, odec.AttnShape(H, Hkv, hd, layer.rope_theta),
+                                    ora["wq"], ora["wk"], ora["wv"], ora["wo"], 128, ora["gate"], ora["up"], ora["wd"],
+                                    128, 128, lora=ora["lora"], lora_scale=2.0)
+    check_bf16(y, ref["y"], "qwen3_4b decoder layer y", min_exact=0.5, depth=3)
+
+
 def test_length_outside_the_cache_is_refused_on_the_device(wq):
     d, H, Hkv, hd, max_len = 256, 4, 2, 64, 16
     x = synth.activations((1, d), 5).cuda()
