@@ -412,7 +412,7 @@ def mlp_forward_info(m: int, layers, prenorm: bool = True, table: LayerTable | N
 
 
 PLAN_FIELDS = ("row_tiles", "kblocks", "rb", "kp", "wk", "panels", "ctas", "threads", "smem", "tok_chunk")
-KIND_GATEUP_W2, KIND_GATEUP_W4, KIND_DOWN_W4 = 0, 1, 2
+KIND_GATEUP_W2, KIND_GATEUP_W4, KIND_DOWN_W4, KIND_GATEUP_W3 = 0, 1, 2, 3
 
 
 def plan_info(kind: int, n: int, k: int, m: int, group: int, r: int = 0) -> dict:
