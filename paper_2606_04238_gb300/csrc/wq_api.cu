@@ -1310,6 +1310,7 @@ wq_status wq_moe_forward(const void *x, int m, const float *logits, const wq_moe
   b.slot_expert = idx;
   b.n_experts = E;
   b.slot_div = 1;
+  b.slot_expert_ready = 1;  // the routing launch is two launches back: the down weights stream before the wait
   e = launch_gemv_slots(kDownW4, W.dn, b, S, s, true);
   if (e != cudaSuccess) return cuda_fail(e, "MoE down launch");
 

@@ -913,15 +913,20 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && NT == 1 && TPW == 1
 // over slots (token t, choice j) -> slot t*top_k + j, one token each; the
 // experts' matrices are stacked row-wise ([E*N, K] packed as one matrix, so
 // expert e owns row tiles e*RT .. e*RT+RT-1) and slot s computes with expert
-// e = slot_expert[s], written by the routing kernel of the same step.  The
-// expert is known only after the previous launch, so the wait comes first
-// and the weight stream follows it.  Per slot: input row s / slot_div of act,
-// tile partials and panel partials / counters of its own, output row s.
+// e = slot_expert[s], written by the routing kernel of the same step.  When
+// the routing kernel is the previous launch (gate/up), the expert is known
+// only after the wait, so the wait comes first and the weight stream follows
+// it.  When it ran two launches earlier (down, `slot_expert_ready`), it has
+// completed before this launch could start -- the gate/up launch lets its
+// dependents start only after its own wait on the routing kernel -- so the
+// index is read at once and the weights stream before the wait, overlapping
+// the gate/up launch.  Per slot: input row s / slot_div of act, tile
+// partials and panel partials / counters of its own, output row s.
 // ---------------------------------------------------------------------------
 template <int BITS, int NPROJ, int GROUP, int TPW>
 __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && TPW == 1 ? 2 : 1)
     qgemv_slots_kernel(const GemvArgs a0, const GemvPlan p) {
-  pdl_wait();  // slot_expert and the activations come from the previous launches
+  if (!a0.slot_expert_ready) pdl_wait();  // slot_expert comes from the previous launch
   const int slot = blockIdx.y;
   const int e = __ldcg(a0.slot_expert + slot);
   if (e < 0 || e >= a0.n_experts) {

@@ -87,6 +87,7 @@ struct GemvArgs {
   // row s; tp, partials and counters hold one region per slot.
   const int *slot_expert;    // [slots], written by the routing kernel
   int n_experts, slot_div;
+  int slot_expert_ready;     // the routing kernel completed before this launch can start (not the previous launch)
   // buffer sizes in bytes (checked by the debug build, WQ_DEBUG_CHECKS)
   size_t nb_codes[2], nb_meta[2], nb_lora_b[2], nb_act, nb_tp, nb_res, nb_out, nb_an, nb_tp_out, nb_part, nb_cnt;
   size_t nb_hq, nb_hsc, nb_hxs, nb_pre_x, nb_pre_sc, nb_pre_xs;
