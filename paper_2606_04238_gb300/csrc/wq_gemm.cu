@@ -1036,6 +1036,279 @@ __global__ void __launch_bounds__(256) to_f16_kernel(const __nv_bfloat16 *x, int
   for (int k = K + tid; k < lda16; k += blockDim.x) x16[(size_t)m * lda16 + k] = 0;
 }
 
+// ---------------------------------------------------------------------------
+// Few tokens (M <= 64): the operands swapped.  The dequantized weight tile is
+// the MMA's A operand (M = 128 rows, the K-major no-swizzle layout the
+// dequantizing warps already write) and the activation tile its B operand
+// (N = NT tokens, NT = M rounded up to 16; one TMA box of 64 features x NT
+// tokens a stage, 128-byte swizzled), so the tensor cores spend no work on
+// padding tokens: with 128-token tiles a 16-token call did 8x the MMA work it
+// needs.  TMEM holds D[row][token]: lane = output row, column = token (gate in
+// columns 0..NT-1, up in NT..2NT-1).  The feature blocks are split KS ways
+// (grid.y) when there are fewer row tiles than SMs: each split writes its fp32
+// partial sums to the workspace and the split that brings the row tile's
+// arrival counter to KS adds them in split order and finishes the tile
+// (deterministic; the counter is left at zero).  The LoRA stages run in split
+// 0.
+// ---------------------------------------------------------------------------
+constexpr int kSwapMaxTok = 64;
+
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+struct SwapCfg {
+  using G = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  static constexpr int BPK = G::BPK, GPB = G::GPB, RAWP = G::RAWP, RAW = G::RAW, BT = G::BT;
+  static constexpr int AT = kSwapMaxTok * 128;  // an activation stage: up to 64 token rows of 128 bytes
+  static constexpr int AVAIL = (int)kGemmSmemLimit - 2048;
+  static constexpr int SB = (AVAIL - 3 * BT - 3 * RAW) / AT >= 4 ? 3 : 2;
+  static constexpr int SA = std::min(8, (AVAIL - SB * BT - 3 * RAW) / AT);
+  static constexpr int R = std::min(6, (AVAIL - SA * AT - SB * BT) / RAW);
+  static_assert(SA >= 2 && R >= 2, "swapped GEMM pipeline does not fit");
+  static constexpr int OFF_A = 0;
+  static constexpr int OFF_B = SA * AT;
+  static constexpr int OFF_RAW = OFF_B + SB * BT;
+  static constexpr int OFF_BAR = OFF_RAW + R * RAW;
+  static constexpr int SMEM = OFF_BAR + (2 * SA + 2 * SB + 2 * R + 2) * 8 + 16 + 1024;
+  static constexpr int NCOLS = 128;  // NPROJ x NT fp32 columns, NT <= 64
+  static_assert(SMEM <= (int)kGemmSmemLimit, "swapped GEMM stage does not fit");
+};
+
+// LoRA stage l, token side: lora_scale * t of tokens 0 .. NT-1 (rank columns
+// 32 l .. 32 l + 31 of gate, then of up), zeros past M and r; lane 0 arrives
+// on `full` once all landed.
+template <int NPROJ>
+__device__ __forceinline__ void swap_lora_t_stage(const GemmArgs &a, uint8_t *As, int NT, int l, int lane,
+                                                  uint64_t *full) {
+  for (int i = lane; i < NPROJ * NT * 4; i += 32) {
+    const int p = i / (NT * 4), rem = i - p * NT * 4;
+    const int ml = rem >> 2, c = rem & 3;
+    const int col = l * kLoraK + c * 8;
+    const bool in = ml < a.M && col < a.r;
+    const uint16_t *src = in ? a.ta + (size_t)ml * 2 * a.r + p * a.r + col : a.ta;
+    cp_async16_zfill(As + p * (NT * kLoraK * 2) + kmajor_off(ml, c * 8, 4 * 128u), src, in ? 16u : 0u);
+  }
+  cp_async_wait_all();
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(full);
+}
+
+// The MMAs of one stage (one thread): per projection, D[p] (+)= W_p x^T over
+// the stage's 4 k-steps (EXACT: the low parts of the weights as well).
+template <int NPROJ, bool EXACT>
+__device__ __forceinline__ void swap_issue_stage(uint32_t tmem, uint32_t as, uint32_t bs, int NT, bool wstage,
+                                                 bool first) {
+  const uint32_t idesc = umma_idesc_f16(128, NT);
+  if (wstage) {
+#pragma unroll
+    for (int p = 0; p < NPROJ; ++p)
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks) {
+        const uint64_t xdesc = umma_desc_kmajor_sw128(as + ks * 32, 1024);
+        umma_f16(tmem + p * NT, umma_desc_kmajor(bs + p * kTileBytes + ks * 256, 128, kSboTile), xdesc, idesc,
+                 (first && ks == 0) ? 0u : 1u);
+        if (EXACT)  // the low parts of the same weights
+          umma_f16(tmem + p * NT, umma_desc_kmajor(bs + (NPROJ + p) * kTileBytes + ks * 256, 128, kSboTile), xdesc,
+                   idesc, 1u);
+      }
+  } else {
+    constexpr uint32_t sbo = 4 * 128u;  // 32 rank columns a LoRA stage
+    for (int p = 0; p < NPROJ; ++p)
+      for (int ks = 0; ks < kLoraK / 16; ++ks)
+        umma_f16(tmem + p * NT, umma_desc_kmajor(bs + p * (kBN * kLoraK * 2) + ks * 256, 128, sbo),
+                 umma_desc_kmajor(as + p * (NT * kLoraK * 2) + ks * 256, 128, sbo), idesc,
+                 (first && ks == 0) ? 0u : 1u);
+  }
+}
+
+// Output row n for tokens mb .. mb + 7 from the fp32 sums g (and u):
+// h = SiLU(rs g) * (rs u), or y = rs g + residual (bf16 or fp32); the lanes
+// of a warp hold consecutive rows, so each token's stores are contiguous.
+template <int NPROJ>
+__device__ __forceinline__ void swap_finish(const GemmArgs &a, int n, int mb, const float (&g)[8],
+                                            const float (&u)[8]) {
+  if (n >= a.N) return;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int m = mb + e;
+    if (m >= a.M) break;
+    const float rs = a.rs != nullptr ? a.rs[m] : 1.f;
+    const size_t o = (size_t)m * a.N + n;
+    if (NPROJ == 2) {
+      const float gv = rs * g[e], uv = rs * u[e];
+      reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(__fdividef(gv, 1.f + __expf(-gv)) * uv);
+    } else {
+      float v = rs * g[e];
+      if (a.residual) v += __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(a.residual)[o]);
+      if (a.out_f32)
+        reinterpret_cast<float *>(a.out)[o] = v;
+      else
+        reinterpret_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(v);
+    }
+  }
+}
+
+template <int BITS, int NPROJ, int GROUP, bool EXACT>
+__global__ void __launch_bounds__(kGemmThreads, 1) qgemm_swap_kernel(const GemmArgs a, const __grid_constant__ GemmMaps tm,
+                                                                     int NT, int KS) {
+  using C = SwapCfg<BITS, NPROJ, GROUP, EXACT>;
+  constexpr int SA = C::SA, SB = C::SB, R = C::R, GPB = C::GPB;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  GemmSmem<C> sm(smem_raw);
+  uint8_t *smem = sm.base;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tile = blockIdx.x, n0 = tile * kBN, ks = blockIdx.y;
+  const int KB = (a.K + 127) / 128;
+  const int kb0 = (int)((long long)KB * ks / KS), kb1 = (int)((long long)KB * (ks + 1) / KS);
+  const int nws = 2 * (kb1 - kb0);  // weight stages (64 features each)
+  const int nlora = NPROJ == 2 && a.r > 0 && ks == 0 ? (a.r + kLoraK - 1) / kLoraK : 0;
+  const int nit = nws + nlora;
+  sm.init(tid, warp);
+  const uint32_t tmem = *sm.tmem_s;
+
+  auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
+    if (*sm.abort_s) return false;
+    if (mbar_wait_sleep(bar, parity)) return true;
+    *sm.abort_s = 1;
+    if (lane == 0) gemm_timeout();
+    return false;
+  };
+
+  if (warp == kRawWarp) {
+    if (lane == 0)
+      for (int it = 0; it < kb1 - kb0; ++it) {
+        const int q = it % R;
+        if (it >= R && !wait(&sm.raw_empty[q], (it / R - 1) & 1)) break;
+        mbar_arrive_expect_tx(&sm.raw_full[q], (uint32_t)C::RAW);
+        for (int p = 0; p < NPROJ; ++p) {
+          uint8_t *dst = smem + C::OFF_RAW + q * C::RAW + p * C::RAWP;
+          tma_load_3d(dst, &tm.codes[p], 0, (kb0 + it) * (C::BPK / 128), n0 / 16, &sm.raw_full[q]);
+          tma_load_3d(dst + 8 * C::BPK, &tm.meta[p], 0, (kb0 + it) * GPB, n0 / 16, &sm.raw_full[q]);
+        }
+      }
+    __syncwarp();
+  } else if (warp == kProducerWarp) {
+    for (int it = 0; it < nit; ++it) {
+      const int s = it % SA;
+      if (it >= SA && !wait(&sm.a_empty[s], (it / SA - 1) & 1)) break;
+      uint8_t *As = smem + C::OFF_A + s * C::AT;
+      if (it < nws) {
+        if (lane == 0) {
+          // one box of 64 features x NT tokens, a 128-byte swizzled row per token
+          mbar_arrive_expect_tx(&sm.a_full[s], (uint32_t)(NT * 128));
+          tma_load_2d(As, &tm.act, (2 * kb0 + it) * 64, 0, &sm.a_full[s]);
+        }
+      } else {
+        swap_lora_t_stage<NPROJ>(a, As, NT, it - nws, lane, &sm.a_full[s]);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      for (int it = 0; it < nit; ++it) {
+        const int sa = it % SA, sb = it % SB;
+        if (!wait(&sm.a_full[sa], (it / SA) & 1) || !wait(&sm.b_full[sb], (it / SB) & 1)) break;
+        tc_fence_after();
+        swap_issue_stage<NPROJ, EXACT>(tmem, smem_addr(smem + C::OFF_A + sa * C::AT),
+                                       smem_addr(smem + C::OFF_B + sb * C::BT), NT, it < nws, it == 0);
+        umma_commit(&sm.a_empty[sa]);
+        umma_commit(&sm.b_empty[sb]);
+      }
+      umma_commit(sm.acc_full);
+    }
+    __syncwarp();
+  } else {
+    // ---- dequantization into the weight tiles ----
+    for (int it = 0; it < nit; ++it) {
+      const int s = it % SB, lb = it >> 1, hb = it & 1, q = lb % R;
+      if (it < nws && !wait(&sm.raw_full[q], (lb / R) & 1)) break;
+      if (it >= SB && !wait(&sm.b_empty[s], (it / SB - 1) & 1)) break;
+      uint8_t *Bs = smem + C::OFF_B + s * C::BT;
+      if (it < nws)
+        gemm_deq_stage<BITS, NPROJ, GROUP, EXACT>(smem + C::OFF_RAW + q * C::RAW, Bs, hb, tid);
+      else
+        gemm_lora_b_stage<NPROJ>(a, Bs, n0, it - nws, tid);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&sm.b_full[s]);
+        if (it < nws && hb == 1) mbar_arrive(&sm.raw_empty[q]);
+      }
+    }
+
+    // ---- epilogue: warp w reads TMEM lanes 32 (w % 4) .. (the rows) and the
+    // token groups of 8 columns w / 4, w / 4 + 4, .. ----
+    const bool ok = wait(sm.acc_full, 0);
+    tc_fence_after();
+    const int quarter = warp & 3, rl = quarter * 32 + lane, n = n0 + rl;
+    constexpr int SLOT = NPROJ * kBN * kSwapMaxTok;  // floats of a split's partial tile: [p][128 rows][NT]
+    float *mine = KS > 1 && a.sk_part ? a.sk_part + ((size_t)tile * KS + ks) * SLOT : nullptr;
+    for (int tg = warp >> 2; tg * 8 < NT; tg += 4) {
+      uint32_t gw[8], uw[8];
+      const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16) + tg * 8;
+      tmem_ld8(tl, gw);
+      if (NPROJ == 2) tmem_ld8(tl + NT, uw);
+      tmem_ld_wait();
+      if (!ok) continue;
+      float g[8], u[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        g[e] = __uint_as_float(gw[e]);
+        u[e] = NPROJ == 2 ? __uint_as_float(uw[e]) : 0.f;
+      }
+      if (mine == nullptr) {
+        swap_finish<NPROJ>(a, n, tg * 8, g, u);
+      } else {
+#pragma unroll
+        for (int p = 0; p < NPROJ; ++p) {
+          float4 *dst = reinterpret_cast<float4 *>(mine + ((size_t)p * kBN + rl) * kSwapMaxTok + tg * 8);
+          const float *v = p == 0 ? g : u;
+          __stcg(dst, make_float4(v[0], v[1], v[2], v[3]));
+          __stcg(dst + 1, make_float4(v[4], v[5], v[6], v[7]));
+        }
+      }
+    }
+    if (mine != nullptr) {
+      named_barrier_sync(1, kDeqWarps * 32);
+      if (tid == 0) {
+        int last = 0;
+        if (ok && !*sm.abort_s) {
+          __threadfence();
+          last = atomicAdd(&a.sk_cnt[tile], 1u) == (unsigned)(KS - 1) ? 1 : 0;
+          if (last) {
+            a.sk_cnt[tile] = 0;  // ready for the next launch
+            __threadfence();
+          }
+        }
+        *sm.last_s = last;
+      }
+      named_barrier_sync(1, kDeqWarps * 32);
+      if (*sm.last_s) {
+        for (int tg = warp >> 2; tg * 8 < NT; tg += 4) {
+          float g[8], u[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) g[e] = u[e] = 0.f;
+          for (int k2 = 0; k2 < KS; ++k2) {  // the splits in order
+            const float *src = a.sk_part + ((size_t)tile * KS + k2) * SLOT;
+#pragma unroll
+            for (int p = 0; p < NPROJ; ++p) {
+              const float4 *pv = reinterpret_cast<const float4 *>(src + ((size_t)p * kBN + rl) * kSwapMaxTok + tg * 8);
+              const float4 v0 = __ldcg(pv), v1 = __ldcg(pv + 1);
+              float *d = p == 0 ? g : u;
+              d[0] += v0.x; d[1] += v0.y; d[2] += v0.z; d[3] += v0.w;
+              d[4] += v1.x; d[5] += v1.y; d[6] += v1.z; d[7] += v1.w;
+            }
+          }
+          swap_finish<NPROJ>(a, n, tg * 8, g, u);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == kMmaWarp) tmem_dealloc(tmem, C::NCOLS);
+}
+
 // cuTensorMapEncodeTiled from the driver (looked up once).
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static std::once_flag once;
@@ -1054,14 +1327,14 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 //   activations [M][lda] binary16, boxes of 8 features x 128 tokens;
 //   codes [RT][KB * BPK / 128][128 B], boxes of one block of 8 row tiles;
 //   scales/zeros [RT][KB * GPB][64 B], boxes of one block of 8 row tiles.
-cudaError_t make_maps(const GemmArgs &a, int nproj, int bits, GemmMaps *m) {
+cudaError_t make_maps(const GemmArgs &a, int nproj, int bits, GemmMaps *m, int box_rows = kBM) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   const cuuint32_t e1[3] = {1, 1, 1};
   {
     const cuuint64_t dims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
     const cuuint64_t strides[1] = {(cuuint64_t)a.lda * 2};
-    const cuuint32_t box[2] = {64, (cuuint32_t)kBM};
+    const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
     if (fn(&m->act, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t *>(a.act), dims, strides, box, e1,
            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
@@ -1131,9 +1404,38 @@ GemmSched gemm_schedule(int M, int N, int K, int nproj, int r, int sms) {
   return g;
 }
 
+// The swapped-operand launch for few tokens: NT = M rounded up to 16; the
+// feature blocks split KS ways when the row tiles alone leave SMs idle (each
+// split at least 2 blocks).
+struct SwapSched {
+  int NT, KS, tiles;
+};
+SwapSched swap_schedule(int M, int N, int K, int sms) {
+  SwapSched w;
+  w.NT = (std::min(M, kSwapMaxTok) + 15) / 16 * 16;
+  w.tiles = (N + kBN - 1) / kBN;
+  const int KB = (K + 127) / 128;
+  w.KS = std::max(1, std::min(sms / std::max(1, w.tiles), KB / 2));
+  return w;
+}
+
 template <int BITS, int NPROJ, int GROUP, bool EXACT>
 cudaError_t launch_gemm_t(const GemmArgs &a, cudaStream_t s) {
   using C = GemmCfg<BITS, NPROJ, GROUP, EXACT>;
+  if (a.M <= kSwapMaxTok) {
+    using SC = SwapCfg<BITS, NPROJ, GROUP, EXACT>;
+    auto kern = qgemm_swap_kernel<BITS, NPROJ, GROUP, EXACT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SC::SMEM);
+    if (e != cudaSuccess) return e;
+    int sms = 0;
+    if ((e = num_sms_cached(&sms)) != cudaSuccess) return e;
+    SwapSched w = swap_schedule(a.M, a.N, a.K, sms);
+    if (!(a.sk_part && a.sk_cnt)) w.KS = 1;
+    GemmMaps maps;
+    if ((e = make_maps(a, NPROJ, BITS, &maps, w.NT)) != cudaSuccess) return e;
+    kern<<<dim3(w.tiles, w.KS), kGemmThreads, SC::SMEM, s>>>(a, maps, w.NT, w.KS);
+    return cudaGetLastError();
+  }
   auto tile_kern = qgemm_tile_kernel<BITS, NPROJ, GROUP, EXACT>;
   auto sk_kern = qgemm_sk_kernel<BITS, NPROJ, GROUP, EXACT>;
   cudaError_t e = cudaFuncSetAttribute(tile_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -1179,7 +1481,12 @@ cudaError_t launch_gemm(GemvKind kind, const GemmArgs &a, cudaStream_t s) {
 size_t gemm_scratch_floats(int M, int N, int K, int nproj, int num_sms) {
   if (M <= 0 || N <= 0 || K <= 0 || num_sms <= 0) return 0;
   const GemmSched g = gemm_schedule(M, N, K, nproj, kMaxRank, num_sms);
-  return g.sk ? (size_t)2 * g.P * kHalves * kBM * nproj * kBN : 0;
+  const size_t sk = g.sk ? (size_t)2 * g.P * kHalves * kBM * nproj * kBN : 0;
+  // the swapped-operand launch of any token count up to this one (a
+  // workspace serves every smaller call too)
+  const SwapSched w = swap_schedule(M, N, K, num_sms);
+  const size_t sw = w.KS > 1 ? (size_t)w.tiles * w.KS * nproj * kBN * kSwapMaxTok : 0;
+  return std::max(sk, sw);
 }
 
 size_t gemm_counters(int M, int N) { return (size_t)((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN); }
