@@ -22,7 +22,7 @@
 // partial dot products of a chunk (8 positions x 4 query heads) are reduced
 // by a butterfly reduce-scatter (31 shuffles), the softmax runs online (max,
 // sum, rescaled accumulators) in fp32.  The splits' partial results (max,
-// sum, accumulator) are merged in split order by a second kernel.
+// sum, accumulator) are merged in a fixed order by a second kernel.
 #include <algorithm>
 #include <cmath>
 #include <cstdint>
@@ -325,25 +325,51 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 2) attn_split_kernel(
   }
 }
 
-// o[b][h * HD + e] = bf16( sum_s O_s e^(M_s - M) / sum_s L_s e^(M_s - M) ),
-// the splits in order.  grid B * H, block HD.
+// o[b][h * HD + e] = bf16( sum_s O_s e^(M_s - M) / sum_s L_s e^(M_s - M) ).
+// grid B * H, 8 warps: warp w merges the splits w, w + 8, .. in order (its
+// own max first), lane l the features l * HD/32 ..; then the warps' results
+// are merged in warp order -- a fixed order, so the result is deterministic.
 template <int HD>
-__global__ void __launch_bounds__(HD) attn_combine_kernel(const float *part, const int *lens, int H, int S, int max_len,
-                                                          __nv_bfloat16 *o) {
-  const int bh = blockIdx.x, e = threadIdx.x;
+__global__ void __launch_bounds__(kAttnWarps * 32) attn_combine_kernel(const float *part, const int *lens, int H, int S,
+                                                                       int max_len, __nv_bfloat16 *o) {
+  constexpr int E = HD / 32;
+  __shared__ float wm[kAttnWarps], wl[kAttnWarps], wo[kAttnWarps][HD];
+  const int bh = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int pos = lens[bh / H];
   if (pos < 0 || pos >= max_len) return;  // skipped by the split kernel
   const float *pt = part + (size_t)bh * S * (HD + 2);
   float M = -INFINITY;
-  for (int s = 0; s < S; ++s) M = fmaxf(M, pt[(size_t)s * (HD + 2) + HD]);
-  float Ls = 0.f, O = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const float ms = pt[(size_t)s * (HD + 2) + HD];
+  for (int s = warp; s < S; s += kAttnWarps) M = fmaxf(M, pt[(size_t)s * (HD + 2) + HD]);
+  float L = 0.f, O[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) O[e] = 0.f;
+#pragma unroll 4
+  for (int s = warp; s < S; s += kAttnWarps) {
+    const float *ps = pt + (size_t)s * (HD + 2);
+    const float ms = ps[HD];
     const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
-    Ls = fmaf(pt[(size_t)s * (HD + 2) + HD + 1], f, Ls);
-    O = fmaf(pt[(size_t)s * (HD + 2) + e], f, O);
+    L = fmaf(ps[HD + 1], f, L);
+#pragma unroll
+    for (int e = 0; e < E; ++e) O[e] = fmaf(ps[lane * E + e], f, O[e]);
   }
-  o[(size_t)bh * HD + e] = __float2bfloat16_rn(O / Ls);
+  if (lane == 0) {
+    wm[warp] = M;
+    wl[warp] = L;
+  }
+#pragma unroll
+  for (int e = 0; e < E; ++e) wo[warp][lane * E + e] = O[e];
+  __syncthreads();
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+    float Mt = -INFINITY;
+    for (int w = 0; w < kAttnWarps; ++w) Mt = fmaxf(Mt, wm[w]);
+    float Lt = 0.f, Ot = 0.f;
+    for (int w = 0; w < kAttnWarps; ++w) {
+      const float f = wm[w] == -INFINITY ? 0.f : __expf(wm[w] - Mt);
+      Lt = fmaf(wl[w], f, Lt);
+      Ot = fmaf(wo[w][e], f, Ot);
+    }
+    o[(size_t)bh * HD + e] = __float2bfloat16_rn(Ot / Lt);
+  }
 }
 
 int attn_splits(int B, int Hkv, int max_len, int num_sms) {
@@ -367,13 +393,13 @@ cudaError_t launch_attn_decode(const float *qkv, const void *x, const int *lens,
     cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
     if (e != cudaSuccess) return e;
     attn_split_kernel<128><<<grid, kAttnWarps * 32, sm, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
-    attn_combine_kernel<128><<<B * H, 128, 0, s>>>(part, lens, H, S, max_len, ob);
+    attn_combine_kernel<128><<<B * H, kAttnWarps * 32, 0, s>>>(part, lens, H, S, max_len, ob);
   } else if (HD == 64) {
     constexpr int sm = attn_smem_bytes<64>();
     cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
     if (e != cudaSuccess) return e;
     attn_split_kernel<64><<<grid, kAttnWarps * 32, sm, s>>>(qkv, xb, lens, d, H, Hkv, fr, kc, vc, max_len, part, S);
-    attn_combine_kernel<64><<<B * H, 64, 0, s>>>(part, lens, H, S, max_len, ob);
+    attn_combine_kernel<64><<<B * H, kAttnWarps * 32, 0, s>>>(part, lens, H, S, max_len, ob);
   } else {
     return cudaErrorInvalidValue;
   }
