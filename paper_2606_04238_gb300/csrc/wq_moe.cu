@@ -11,6 +11,7 @@
 //      and one expert each) -> h per slot;
 //   3. the down dequant-GEMV over the slots -> y_j per slot in fp32;
 //   4. moe_combine_kernel: y[t] = bf16(x[t] + sum_j w_j y_j), j in order.
+#include <climits>
 #include <cstdint>
 
 #include <cuda_bf16.h>
@@ -86,7 +87,7 @@ __global__ void __launch_bounds__(kPrepWarps * 32) moe_prep_kernel(const __nv_bf
         }
       }
       if (be != INT_MAX && (be & 31) == lane) live &= ~(1u << (be >> 5));
-      sel_l[c < kMoeMaxTopK ? c : 0] = bl;
+      sel_l[c] = bl;  // top_k <= kMoeMaxTopK (checked by the launcher)
       if (lane == 0) sel_s[c] = be;
     }
     if (lane == 0) {
