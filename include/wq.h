@@ -51,7 +51,7 @@ typedef enum {
     WQ_ERR_ARG = -1,          /* null pointer, negative size, bad flag */
     WQ_ERR_SHAPE = -2,        /* shapes inconsistent or outside the supported set */
     WQ_ERR_ALIGN = -3,        /* a device pointer is not 16-byte aligned */
-    WQ_ERR_UNSUPPORTED = -4,  /* valid request this build does not implement */
+    WQ_ERR_UNSUPPORTED = -4,  /* valid request this library does not implement */
     WQ_ERR_CUDA = -5,         /* a CUDA runtime call or launch failed */
     WQ_ERR_TIMEOUT = -6,      /* a bounded device-side wait ran out */
     WQ_ERR_WORKSPACE = -7     /* workspace missing or smaller than required */

@@ -433,7 +433,7 @@ bool chain_panel_ok(GemvKind kind, int m, const wq_qweight &gate, int r, const w
 
 wq_status check_tokens(int m) {
   if (m < 0) return fail(WQ_ERR_ARG, "m=%d is negative", m);
-  if (m > kMaxGemmTokens) return fail(WQ_ERR_UNSUPPORTED, "m=%d exceeds the %d-token limit of this build", m, kMaxGemmTokens);
+  if (m > kMaxGemmTokens) return fail(WQ_ERR_UNSUPPORTED, "m=%d exceeds the %d-token limit of the library", m, kMaxGemmTokens);
   return WQ_OK;
 }
 
