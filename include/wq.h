@@ -391,6 +391,16 @@ wq_status wq_moe_forward(const void *x, int m, const float *logits, const wq_moe
                          size_t ws_bytes, void *stream);
 
 /*
+ * Self-check of the kernels' bounded waits (failure detection without a GPU
+ * fault): one launch whose single CTA waits, with the library's own wait
+ * routines, on an mbarrier that nothing arrives on and at a grid barrier that
+ * nothing advances.  Each wait gives up after its limit (2 s), records
+ * WQ_ERR_TIMEOUT and lets the launch end; wq_device_status() then returns
+ * WQ_ERR_TIMEOUT and the context stays usable.  About 4 s on `stream`.
+ */
+wq_status wq_wait_check(void *stream);
+
+/*
  * wq_mlp_forward that also returns every layer's output (the hidden states of
  * the stack) and, optionally, every layer's MLP activation h:
  *   states:   bf16 [n_layers][m][d] (device, 16-byte aligned), states[l] = x_{l+1};

@@ -1333,6 +1333,12 @@ wq_status wq_plan_info(int kind, int n, int k, int m, int group, int r, int64_t 
   return ok();
 }
 
+wq_status wq_wait_check(void *stream) {
+  cudaError_t e = launch_wait_check(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "wait self-check launch");
+  return ok();
+}
+
 const char *wq_last_error(void) { return g_last_error.c_str(); }
 
 // Debug builds: first failed in-kernel bounds / alignment check.

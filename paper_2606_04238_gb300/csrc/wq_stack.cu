@@ -1052,6 +1052,32 @@ cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, const StackMaps
   return a.bits_gu == 2 ? launch_stack_b<2>(a, p, maps, s) : launch_stack_b<4>(a, p, maps, s);
 }
 
+// Self-check of the bounded waits (no GPU fault, no hang): one CTA of the
+// stack kernel's shape waits on an mbarrier that nothing arrives on, then at
+// a grid barrier whose counter nothing advances; each wait gives up after its
+// limit (kWaitLimitNs), records WQ_ERR_TIMEOUT in the status word and lets
+// the kernel end, so the context stays usable.
+__device__ unsigned long long g_wait_check_ctr = 0;
+
+__global__ void __launch_bounds__(kSThreads) wait_check_kernel() {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+    abort_flag = 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !mbar_wait(&bar, 0)) record_timeout();  // phase 0 never completes
+  __syncthreads();
+  if (threadIdx.x < kSMathThreads) grid_wait(&g_wait_check_ctr, ld_acquire_u64(&g_wait_check_ctr) + 1, &abort_flag);
+}
+
+cudaError_t launch_wait_check(cudaStream_t s) {
+  wait_check_kernel<<<1, kSThreads, 0, s>>>();
+  return cudaGetLastError();
+}
+
 cudaError_t read_stack_status(int *status) {
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return e;

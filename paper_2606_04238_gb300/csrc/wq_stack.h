@@ -78,5 +78,7 @@ cudaError_t stack_layer_maps(const void *gate_codes, const void *up_codes, const
 cudaError_t launch_stack(const StackArgs &a, const StackPlan &p, const StackMaps &maps, cudaStream_t s);
 // Reads and clears the stack kernel's device status word.
 cudaError_t read_stack_status(int *status);
+// The bounded-wait self-check (wq_wait_check).
+cudaError_t launch_wait_check(cudaStream_t s);
 
 }  // namespace wq

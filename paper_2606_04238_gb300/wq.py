@@ -94,6 +94,7 @@ def lib():
             "wq_decoder_layer_forward": (I, [P, I, P, ctypes.POINTER(_DecoderLayer), P, P, I, U, P, P, S, P]),
             "wq_moe_workspace_bytes": (S, [I, ctypes.POINTER(_MoELayer), U]),
             "wq_moe_forward": (I, [P, I, P, ctypes.POINTER(_MoELayer), U, P, P, P, P, P, P, S, P]),
+            "wq_wait_check": (I, [P]),
             "wq_last_error": (ctypes.c_char_p, []),
             "wq_device_status": (I, [ctypes.POINTER(I)]),
             "wq_version": (ctypes.c_char_p, []),
@@ -530,6 +531,11 @@ def moe_forward(x, logits, layer: MoELayer, prenorm: bool = True, y=None, ws=Non
     _check(lib().wq_moe_forward(_ptr(x), m, _ptr(logits), ctypes.byref(cl), WQ_PRENORM if prenorm else 0, _ptr(y),
                                 _ptr(idx), _ptr(wt), _ptr(hs), _ptr(ys), _ptr(ws), ws.numel(), _stream()))
     return (y, idx, wt, hs, ys) if with_slots else y
+
+
+def wait_check():
+    """wq_wait_check: a launch whose bounded waits run out (WQ_ERR_TIMEOUT in the device status)."""
+    _check(lib().wq_wait_check(_stream()))
 
 
 def device_status() -> int:
