@@ -972,7 +972,7 @@ __global__ void __launch_bounds__(kMaxThreads, NPROJ == 1 && TPW == 1 ? 2 : 1)
 // of 16 features: tp[tile][m][0] = sum_c x_c^2, tp[tile][m][1 + j] =
 // sum_c A[j, c] x_c, each as s = fma(w_c, x_c, s) over c in order.  The
 // gate/up kernel adds them up into the RMSNorm scale and the LoRA-A
-// products x A^T of Eq. 1.
+// products x A^T of Eq. 1.  A lane takes the values lane, lane + 32, ..
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, int M, int d,
                                                          const __nv_bfloat16 *lora_a, int r2, float *tp,
@@ -981,14 +981,30 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
   const int ntp = d / 16;
   const int tile = blockIdx.x * (blockDim.x >> 5) + warp;
   const int Q = 1 + r2, Qp = (Q + 3) & ~3;
+  constexpr int QI = (1 + 2 * kMaxRank + 3) / 32 + 1;  // values a lane takes, at most
   pdl_launch_dependents();
-  pdl_wait();
-  if (tile >= ntp) return;
+  // The LoRA-A rows of this lane's values (weights, not written by the
+  // previous kernel) are loaded before the wait; only x waits for it.
   const uint8_t *x8 = reinterpret_cast<const uint8_t *>(x);
   const uint8_t *a8 = reinterpret_cast<const uint8_t *>(lora_a);
   (void)nb_x;
   (void)nb_a;
   (void)nb_tp;
+  uint4 av[QI][2];
+#pragma unroll
+  for (int i = 0; i < QI; ++i) {
+    const int q = lane + 32 * i;
+    av[i][0] = av[i][1] = make_uint4(0u, 0u, 0u, 0u);
+    if (tile < ntp && q >= 1 && q < Q) {
+      const size_t ao = ((size_t)(q - 1) * d + (size_t)tile * 16) * 2;
+      if (WQ_OK_IF(WQ_RANGE(ao, 32, nb_a, 16), 45, ao)) {
+        av[i][0] = __ldg(reinterpret_cast<const uint4 *>(a8 + ao));
+        av[i][1] = __ldg(reinterpret_cast<const uint4 *>(a8 + ao + 16));
+      }
+    }
+  }
+  pdl_wait();
+  if (tile >= ntp) return;
   for (int m = 0; m < M; ++m) {
     float v[16];
     const size_t xo = ((size_t)m * d + (size_t)tile * 16) * 2;
@@ -999,26 +1015,21 @@ __global__ void __launch_bounds__(256) tile_prep_kernel(const __nv_bfloat16 *x, 
     }
     unpack_bf16x8(x0, *reinterpret_cast<float(*)[8]>(v));
     unpack_bf16x8(x1, *reinterpret_cast<float(*)[8]>(v + 8));
-    for (int q = lane; q < Qp; q += 32) {
+#pragma unroll
+    for (int i = 0; i < QI; ++i) {
+      const int q = lane + 32 * i;
+      if (q >= Qp) break;
       float s = 0.f;
-      if (q >= Q) {
-        s = 0.f;  // padding
-      } else if (q == 0) {
+      if (q == 0) {
 #pragma unroll
         for (int c = 0; c < 16; ++c) s = fmaf(v[c], v[c], s);
-      } else {
-        const size_t ao = ((size_t)(q - 1) * d + (size_t)tile * 16) * 2;
-        uint4 a0 = make_uint4(0u, 0u, 0u, 0u), a1 = a0;
-        if (WQ_OK_IF(WQ_RANGE(ao, 32, nb_a, 16), 45, ao)) {
-          a0 = __ldg(reinterpret_cast<const uint4 *>(a8 + ao));
-          a1 = __ldg(reinterpret_cast<const uint4 *>(a8 + ao + 16));
-        }
+      } else if (q < Q) {
         float w[16];
-        unpack_bf16x8(a0, *reinterpret_cast<float(*)[8]>(w));
-        unpack_bf16x8(a1, *reinterpret_cast<float(*)[8]>(w + 8));
+        unpack_bf16x8(av[i][0], *reinterpret_cast<float(*)[8]>(w));
+        unpack_bf16x8(av[i][1], *reinterpret_cast<float(*)[8]>(w + 8));
 #pragma unroll
         for (int c = 0; c < 16; ++c) s = fmaf(w[c], v[c], s);
-      }
+      }  // else padding: 0
       const size_t o = ((size_t)tile * M + m) * Qp + q;
       if (WQ_OK_IF(WQ_RANGE(o * 4, 4, nb_tp, 4), 46, o)) tp[o] = s;
     }
