@@ -4,9 +4,10 @@ The tcgen05 path multiplies binary16 copies of the activations.  Each token
 is scaled by an exact power of two before the narrowing (its largest |x| put
 in [16, 32)) and the epilogue undoes it, so tokens of any magnitude keep the
 precision of unit-scale ones: here tokens span 1e-6 .. 1e5 (gate/up with
-and without the RMSNorm, down with bf16 and fp32 output) and a stack without
-the RMSNorm whose h reaches ~1e6 (past the binary16 maximum 65504).  Every
-token is checked against the oracle with its own bound.
+and without the RMSNorm, down with bf16 and fp32 output; 24 tokens on the
+swapped-operand launch, 65 and 512 on the token-tile ones) and a stack
+without the RMSNorm whose h reaches ~1e6 (past the binary16 maximum 65504).
+Every token is checked against the oracle with its own bound.
 """
 import numpy as np
 import pytest
@@ -49,7 +50,7 @@ def _per_token(got, ref, what, min_exact=MIN_EXACT, f32=False):
             check_bf16(got[i:i + 1], ref[i:i + 1], f"{what} token {i}", min_exact=min_exact)
 
 
-@pytest.mark.parametrize("m", [65, 512])
+@pytest.mark.parametrize("m", [24, 65, 512])
 @pytest.mark.parametrize("prenorm", [False, True])
 def test_gateup_wide_range(wq, m, prenorm):
     d, inter, group, r = 512, 1024, 128, 16
@@ -66,7 +67,7 @@ def test_gateup_wide_range(wq, m, prenorm):
     _per_token(h, ref, f"gate/up m={m} prenorm={prenorm}")
 
 
-@pytest.mark.parametrize("m", [65, 512])
+@pytest.mark.parametrize("m", [24, 65, 512])
 def test_down_wide_range(wq, m):
     d, inter, group = 512, 1024, 128
     qd = _q((d, inter), group, 4, 9)

@@ -3,11 +3,12 @@ operands (weights as the M = 128 operand, tokens as N = 16..64) vs the fp64
 oracle.
 
 Covers token counts that round up to every N (9, 16, 17, 33, 48, 64), ragged
-row tiles and feature blocks, the adapter's stages, the RMSNorm, split
-feature axes (2 to 32 splits whose fp32 partial sums the last split adds in
-order) and a single split, down with a residual in bf16 and fp32 (the exact
-two-part weights), and a stack of two 8B-shaped layers at 16 tokens.  Calls
-with d >= 4096 take the GEMM path above 8 tokens, the others above 16.
+row tiles and feature blocks, every group size, the adapter's stages, the
+RMSNorm, split feature axes (2 to 32 splits whose fp32 partial sums the last
+split adds in order) and a single split, 4-bit gate/up (two projections of
+4-bit codes), down with a residual in bf16 and fp32 (the exact two-part
+weights), and a stack of two 8B-shaped layers at 16 tokens.  Calls with
+d >= 4096 take the GEMM path above 8 tokens, the others above 16.
 """
 import numpy as np
 import pytest
@@ -62,6 +63,18 @@ def test_swap_gateup(wq, d, inter, group, r, ms, prenorm):
         ref, _ = orc.gateup(synth.bf16_bits(x), qg, qu, group, okw.get("lora_a"), okw.get("lora_b_gate"),
                             okw.get("lora_b_up"), lora_scale=2.0, prenorm=prenorm)
         check_bf16(h, ref, f"swap h d={d} I={inter} g={group} r={r} m={m} prenorm={prenorm}", min_exact=MIN_EXACT)
+
+
+@pytest.mark.parametrize("m", [17, 64])
+def test_swap_gateup_w4(wq, m):
+    d, inter, group = 512, 384, 64
+    qg, qu = _q((inter, d), group, 4, 15), _q((inter, d), group, 4, 16)
+    x = synth.activations((m, d), 17 + m)
+    h = wq.gateup_w4(x.cuda(), upload_packed(*qg, group, 4), upload_packed(*qu, group, 4), prenorm=True)
+    torch.cuda.synchronize()
+    assert wq.device_status() == 0
+    ref, _ = orc.gateup(synth.bf16_bits(x), qg, qu, group, None, None, None, lora_scale=0.0, prenorm=True)
+    check_bf16(h, ref, f"swap W4 h m={m}", min_exact=MIN_EXACT)
 
 
 DOWN_CASES = [
