@@ -388,6 +388,34 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
   // launch computes, not while its latency-bound input loads above are in
   // flight.
   pdl_launch_dependents();
+  // The tile partials summed over the chunks (fixed order) and, with the
+  // RMSNorm, each token's scale rs = 1/sqrt(mean(x^2) + eps) in place of its
+  // sum of squares: their inputs are complete here, so this runs before the
+  // dot products instead of behind two more barriers after them, on the
+  // last threads (their warps convert the fewest items below).
+  if (use_tp && (nchk > 1 || a.prenorm)) {
+    const size_t cst = (size_t)M * Qp;  // stride between chunks
+    for (int pair = (int)blockDim.x - 1 - tid; pair < M * Qp; pair += blockDim.x) {
+      float s = 0.f;
+      if (nchk > 1) {
+        // four loads in flight, added in chunk order
+        int c = 0;
+        for (; c + 4 <= nchk; c += 4) {
+          const float v0 = red_s[c * cst + pair], v1 = red_s[(c + 1) * cst + pair];
+          const float v2 = red_s[(c + 2) * cst + pair], v3 = red_s[(c + 3) * cst + pair];
+          s += v0;
+          s += v1;
+          s += v2;
+          s += v3;
+        }
+        for (; c < nchk; ++c) s += red_s[c * cst + pair];
+      } else {
+        s = rt_s[pair];
+      }
+      if (a.prenorm && pair % Qp == 0) s = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(s, (float)a.K), kRmsEps)));
+      if (WQ_OK_IF(WQ_RANGE(p.off_rt + (size_t)pair * 4, 4, p.off_yv, 4), 37, pair)) rt_s[pair] = s;
+    }
+  }
   // Activation panel -> binary16 in place, one (block, token) item per warp.
   // Scale 2^e puts the block's max|x| in [2^14, 2^15): binary16 then holds
   // every scaled bf16 value exactly (bf16 has 8 significant bits), far from
@@ -728,38 +756,7 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
     }
     if (tid < nrt && last_s[tid]) a.counters[rt0 + tid] = 0u;
     __syncthreads();
-  } else {
-    if (tid < nrt) last_s[tid] = 1;
-    __syncthreads();
-  }
-
-  // the tile partials summed over tiles: add the chunk sums (fixed order)
-  if (use_tp && nchk > 1) {
-    const size_t cst = (size_t)M * Qp;  // stride between chunks
-    for (int pair = tid; pair < M * Qp; pair += blockDim.x) {
-      // four loads in flight, added in chunk order
-      float s = 0.f;
-      int c = 0;
-      for (; c + 4 <= nchk; c += 4) {
-        const float v0 = red_s[c * cst + pair], v1 = red_s[(c + 1) * cst + pair];
-        const float v2 = red_s[(c + 2) * cst + pair], v3 = red_s[(c + 3) * cst + pair];
-        s += v0;
-        s += v1;
-        s += v2;
-        s += v3;
-      }
-      for (; c < nchk; ++c) s += red_s[c * cst + pair];
-      if (WQ_OK_IF(WQ_RANGE(p.off_rt + (size_t)pair * 4, 4, p.off_yv, 4), 37, pair)) rt_s[pair] = s;
-    }
-    __syncthreads();
-  }
-
-  // RMSNorm scale of each token, rs = 1/sqrt(mean(x^2) + eps), in place of its sum of squares
-  if (use_tp && a.prenorm) {
-    for (int m = tid; m < M; m += blockDim.x)
-      rt_s[(size_t)m * Qp] = __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(rt_s[(size_t)m * Qp], (float)a.K), kRmsEps)));
-    __syncthreads();
-  }
+  }  // one panel: every row tile is finished here (last_s is not read)
 
   // ---- epilogue: RMSNorm scale, LoRA-B + SiLU(g) * u; or residual add ----
   const int rows = nrt * 16;
@@ -848,7 +845,7 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
     for (int i = tid; i < rows * M; i += blockDim.x) {
       const int m = i / rows, rl = i % rows;
       const int rti = rl >> 4, r16 = rl & 15;
-      if (!last_s[rti]) continue;
+      if (p.P > 1 && !last_s[rti]) continue;
       const int n = (rt0 + rti) * 16 + r16;
       if (n >= a.N) continue;
       if (NPROJ == 2) {
@@ -881,7 +878,7 @@ __device__ __forceinline__ void qgemv_body(const GemvArgs &a, const GemvPlan &p)
     for (int i = tid; i < nrt * M * Qp; i += blockDim.x) {
       const int rti = i / (M * Qp), rem = i % (M * Qp);
       const int m = rem / Qp, q = rem % Qp;
-      if (!last_s[rti]) continue;
+      if (p.P > 1 && !last_s[rti]) continue;
       const int tile = rt0 + rti;
       const int nv = q < Q ? max(0, min(16, a.N - tile * 16)) : 0;  // rows of the tile inside the matrix
       float vv[16], wv[16];
